@@ -1,0 +1,233 @@
+"""CPU oracle for the thresholded gated MLP and token routing (test infrastructure).
+
+This package is TEST INFRASTRUCTURE.  Only ``tests/``, ``__graft_entry__.smoke()``
+and the ``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import
+it.  It shares no code with the CUDA library in ``paper_2607_08991_gb300``:
+the arithmetic lives in ``sats_oracle.c`` (plain C, IEEE double), compiled
+with gcc into ``liboracle.so`` and called through ctypes.  This module only
+marshals numpy arrays.
+
+Paper: "Sensitivity-Aware Thresholding and Token Routing for Activation
+Sparsification in Large Language Models" (arXiv 2607.08991).  Each wrapper
+names the section / equation its C routine states.
+
+Parity status: every function here is pinned by ``tests/test_oracle_*.py``
+(closed forms, brute force on tiny inputs, library cross-checks and
+invariants).  No function is "parity unpinned".
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+from typing import Optional, Sequence
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "sats_oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile sats_oracle.c into liboracle.so with gcc (portable flags only)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + ".tmp.%d" % os.getpid()
+        subprocess.check_call(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        build()
+        lib = ctypes.CDLL(_LIB)
+        P = ctypes.c_void_p
+        I = ctypes.c_int
+        I64 = ctypes.c_int64
+        D = ctypes.c_double
+        lib.oracle_bf16_to_f64.argtypes = [I64, P, P]
+        lib.oracle_silu.argtypes = [D]
+        lib.oracle_silu.restype = D
+        lib.oracle_gate_act.argtypes = [I, I, I, P, P, P]
+        lib.oracle_up_proj.argtypes = [I, I, I, P, P, P]
+        lib.oracle_cats_mask.argtypes = [I, I, P, P, P, D, P]
+        lib.oracle_cats_mask.restype = I64
+        lib.oracle_masked_mlp.argtypes = [I, I, I, P, P, P, P, P, P]
+        lib.oracle_sparse_mlp.argtypes = [I, I, I, P, P, P, P, P, P, D, P, P, P]
+        lib.oracle_sparse_mlp.restype = I64
+        lib.oracle_dense_mlp.argtypes = [I, I, I, P, P, P, P, P]
+        lib.oracle_percentile_threshold.argtypes = [P, I64, D]
+        lib.oracle_percentile_threshold.restype = D
+        lib.oracle_route.argtypes = [I, P, I, P, P, P]
+        lib.oracle_route.restype = I
+        lib.oracle_rmsnorm.argtypes = [I, I, P, P, D, P]
+        lib.oracle_mlp_stack.argtypes = [I, I, I, I, P, P, P, P, P, D, P, P, I, P, P, D, P]
+        lib.oracle_mlp_stack.restype = I64
+        _lib = lib
+    return _lib
+
+
+def _ptr(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data
+
+
+def _f64(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.float64)
+
+
+def _u16(a) -> np.ndarray:
+    a = np.ascontiguousarray(a)
+    assert a.dtype == np.uint16, "weights are bf16 bit patterns (uint16)"
+    return a
+
+
+def bf16_to_f64(bits: np.ndarray) -> np.ndarray:
+    """Exact value of each bf16 bit pattern, as float64."""
+    bits = _u16(bits)
+    out = np.empty(bits.shape, dtype=np.float64)
+    _load().oracle_bf16_to_f64(bits.size, _ptr(bits), _ptr(out))
+    return out
+
+
+def silu(z: float) -> float:
+    """Sec. 2, Eq. 2."""
+    return _load().oracle_silu(float(z))
+
+
+def gate_act(x: np.ndarray, Wg: np.ndarray) -> np.ndarray:
+    """Sec. 2, Eqs. 1-2: SiLU(x W_gate); x [B][H] float64, Wg [H][N] bf16 bits."""
+    x = _f64(x)
+    Wg = _u16(Wg)
+    B, H = x.shape
+    N = Wg.shape[1]
+    a = np.empty((B, N), dtype=np.float64)
+    _load().oracle_gate_act(B, H, N, _ptr(x), _ptr(Wg), _ptr(a))
+    return a
+
+
+def up_proj(x: np.ndarray, Wu: np.ndarray) -> np.ndarray:
+    """Sec. 2, Eq. 1: x W_up."""
+    x = _f64(x)
+    Wu = _u16(Wu)
+    B, H = x.shape
+    N = Wu.shape[1]
+    u = np.empty((B, N), dtype=np.float64)
+    _load().oracle_up_proj(B, H, N, _ptr(x), _ptr(Wu), _ptr(u))
+    return u
+
+
+def cats_mask(a: np.ndarray, t, keep_hint: Optional[np.ndarray] = None, band_rel: float = 0.0):
+    """Sec. 2, Eqs. 4-5: keep iff |a| >= t.  Returns (keep uint8 [B][N], in_band)."""
+    a = _f64(a)
+    B, N = a.shape
+    tt = _f64(np.broadcast_to(np.asarray(t, dtype=np.float64), (B,)))
+    keep = np.empty((B, N), dtype=np.uint8)
+    hint = None if keep_hint is None else np.ascontiguousarray(keep_hint, dtype=np.uint8)
+    nb = _load().oracle_cats_mask(B, N, _ptr(a), _ptr(tt), _ptr(hint), float(band_rel), _ptr(keep))
+    return keep, int(nb)
+
+
+def masked_mlp(x, Wg, Wu, Wd, keep) -> np.ndarray:
+    """Sec. 2, Eqs. 1 and 5 with a given mask."""
+    x = _f64(x)
+    Wg, Wu, Wd = _u16(Wg), _u16(Wu), _u16(Wd)
+    B, H = x.shape
+    N = Wg.shape[1]
+    keep = np.ascontiguousarray(keep, dtype=np.uint8)
+    y = np.empty((B, H), dtype=np.float64)
+    _load().oracle_masked_mlp(B, H, N, _ptr(x), _ptr(Wg), _ptr(Wu), _ptr(Wd), _ptr(keep), _ptr(y))
+    return y
+
+
+def sparse_mlp(x, Wg, Wu, Wd, t, keep_hint=None, band_rel: float = 0.0):
+    """Sec. 2, Eqs. 1-5: the CATS-thresholded gated MLP with per-token threshold t.
+
+    Returns (y [B][H] float64, a [B][N] float64, keep [B][N] uint8, in_band).
+    """
+    x = _f64(x)
+    Wg, Wu, Wd = _u16(Wg), _u16(Wu), _u16(Wd)
+    B, H = x.shape
+    N = Wg.shape[1]
+    assert Wg.shape == (H, N) and Wu.shape == (H, N) and Wd.shape == (N, H)
+    tt = _f64(np.broadcast_to(np.asarray(t, dtype=np.float64), (B,)))
+    hint = None if keep_hint is None else np.ascontiguousarray(keep_hint, dtype=np.uint8)
+    y = np.empty((B, H), dtype=np.float64)
+    a = np.empty((B, N), dtype=np.float64)
+    keep = np.empty((B, N), dtype=np.uint8)
+    nb = _load().oracle_sparse_mlp(B, H, N, _ptr(x), _ptr(Wg), _ptr(Wu), _ptr(Wd), _ptr(tt),
+                                   _ptr(hint), float(band_rel), _ptr(y), _ptr(a), _ptr(keep))
+    return y, a, keep, int(nb)
+
+
+def dense_mlp(x, Wg, Wu, Wd) -> np.ndarray:
+    """Sec. 2, Eq. 1: the base gated MLP, no mask."""
+    x = _f64(x)
+    Wg, Wu, Wd = _u16(Wg), _u16(Wu), _u16(Wd)
+    B, H = x.shape
+    N = Wg.shape[1]
+    y = np.empty((B, H), dtype=np.float64)
+    _load().oracle_dense_mlp(B, H, N, _ptr(x), _ptr(Wg), _ptr(Wu), _ptr(Wd), _ptr(y))
+    return y
+
+
+def percentile_threshold(values: np.ndarray, k: float) -> float:
+    """Sec. 2, Eq. 3: t = min{t' : F(t') >= k} over the magnitudes of `values`."""
+    v = _f64(values).ravel()
+    return float(_load().oracle_percentile_threshold(_ptr(v), v.size, float(k)))
+
+
+def route(ids: np.ndarray, lut: np.ndarray):
+    """Sec. 3.2, Eq. 13 as a LUT: returns (perm int32 [B], n_dense) or raises on a bad id."""
+    ids = np.ascontiguousarray(ids, dtype=np.int32)
+    lut = np.ascontiguousarray(lut, dtype=np.uint8)
+    B = ids.size
+    perm = np.empty(max(B, 1), dtype=np.int32)
+    nd = np.zeros(1, dtype=np.int32)
+    rc = _load().oracle_route(B, _ptr(ids), lut.size, _ptr(lut), _ptr(perm), _ptr(nd))
+    if rc != 0:
+        raise ValueError("token id outside the vocabulary")
+    return perm[:B].copy(), int(nd[0])
+
+
+def rmsnorm(x, w, eps: float) -> np.ndarray:
+    x = _f64(x)
+    B, H = x.shape
+    w = np.ascontiguousarray(w, dtype=np.float32)
+    out = np.empty_like(x)
+    _load().oracle_rmsnorm(B, H, _ptr(x), _ptr(w), float(eps), _ptr(out))
+    return out
+
+
+def mlp_stack(x, Wg: Sequence, Wu: Sequence, Wd: Sequence, norm_w: Sequence, t, eps: float,
+              ids=None, lut=None, keep_hint=None, band_rel: float = 0.0, want_keep: bool = False):
+    """Stack of L RMSNorm -> gated MLP -> residual blocks with per-token routing.
+
+    Returns (x_out [B][H] float64, keep [L][B][N] uint8 or None, in_band).
+    """
+    x = _f64(x).copy()
+    B, H = x.shape
+    L = len(Wg)
+    N = Wg[0].shape[1]
+    keep_ref = [_u16(w) for w in Wg], [_u16(w) for w in Wu], [_u16(w) for w in Wd]
+    nw = [np.ascontiguousarray(w, dtype=np.float32) for w in norm_w]
+    arr = lambda lst: (ctypes.c_void_p * L)(*[a.ctypes.data for a in lst])
+    tt = _f64(np.broadcast_to(np.asarray(t, dtype=np.float64), (L,)))
+    if ids is not None:
+        ids_a = np.ascontiguousarray(ids, dtype=np.int32)
+        lut_a = np.ascontiguousarray(lut, dtype=np.uint8)
+        V = lut_a.size
+    else:
+        ids_a = lut_a = None
+        V = 0
+    hint = None if keep_hint is None else np.ascontiguousarray(keep_hint, dtype=np.uint8)
+    keep = np.empty((L, B, N), dtype=np.uint8) if want_keep else None
+    nb = _load().oracle_mlp_stack(L, B, H, N, arr(keep_ref[0]), arr(keep_ref[1]), arr(keep_ref[2]),
+                                  arr(nw), _ptr(tt), float(eps), _ptr(ids_a), _ptr(lut_a), V,
+                                  _ptr(x), _ptr(hint), float(band_rel), _ptr(keep))
+    if nb < 0:
+        raise ValueError("token id outside the vocabulary")
+    return x, keep, int(nb)

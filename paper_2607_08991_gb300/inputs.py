@@ -1,0 +1,133 @@
+"""Seeded synthetic inputs shared by the tests, the bench and the oracle checks.
+
+This module only draws random numbers and packs them into the bit layouts the
+two sides take (bf16 bit patterns as uint16, fp32, int32, uint8).  It holds
+none of the method's arithmetic: no projection, activation, threshold,
+percentile or routing rule.  Thresholds are chosen by the method's own
+calibration routine on each side (Eq. 3 of arXiv 2607.08991).
+
+Shapes and distributions follow the workloads the paper runs on
+(Llama-3.1-8B: hidden 4096, intermediate 14336, vocab 128256, 32 blocks;
+Qwen3-8B: hidden 4096, intermediate 12288, vocab 151936, 36 blocks), with
+synthetic weights ~ N(0, 0.02) in bf16 standing in for the trained weights.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Dict, List
+
+import numpy as np
+
+LLAMA_H, LLAMA_N, LLAMA_L, LLAMA_V = 4096, 14336, 32, 128256
+QWEN_H, QWEN_N, QWEN_L, QWEN_V = 4096, 12288, 36, 151936
+SMALL_H, SMALL_N = 512, 1408
+
+# Seed bases: weights of layer l use SEED_WEIGHTS + l (gate / up / down are
+# sub-streams 0 / 1 / 2), evaluation activations SEED_X, calibration
+# activations SEED_CALIB, routing table SEED_LUT, token ids SEED_IDS,
+# RMSNorm weights SEED_NORM + l.
+SEED_WEIGHTS = 1000
+SEED_X = 2000
+SEED_CALIB = 3000
+SEED_LUT = 4000
+SEED_IDS = 5000
+SEED_NORM = 6000
+SEED_SHUFFLE = 7000
+
+
+def _rng(*seed: int) -> np.random.Generator:
+    return np.random.default_rng(list(seed))
+
+
+def to_bf16_bits(a: np.ndarray) -> np.ndarray:
+    """Round float32 values to bf16 (nearest, ties to even); returns uint16 bit patterns."""
+    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32)
+    r = (u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))) >> np.uint32(16)
+    return r.astype(np.uint16)
+
+
+def bf16_bits_to_f32(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns -> float32 (exact)."""
+    return (np.ascontiguousarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+def normal_bf16(shape, std: float, *seed: int) -> np.ndarray:
+    z = _rng(*seed).standard_normal(size=shape, dtype=np.float32)
+    z *= np.float32(std)
+    return to_bf16_bits(z)
+
+
+@dataclasses.dataclass
+class MLPWeights:
+    """One gated-MLP block in the paper's layout: Wg, Wu [H][N]; Wd [N][H] (bf16 bits)."""
+    Wg: np.ndarray
+    Wu: np.ndarray
+    Wd: np.ndarray
+
+    @property
+    def H(self) -> int:
+        return self.Wg.shape[0]
+
+    @property
+    def N(self) -> int:
+        return self.Wg.shape[1]
+
+
+def mlp_weights(H: int, N: int, layer: int = 0, std: float = 0.02, seed: int = SEED_WEIGHTS) -> MLPWeights:
+    return MLPWeights(
+        Wg=normal_bf16((H, N), std, seed + layer, 0),
+        Wu=normal_bf16((H, N), std, seed + layer, 1),
+        Wd=normal_bf16((N, H), std, seed + layer, 2),
+    )
+
+
+def activations_bf16(B: int, H: int, seed: int = SEED_X) -> np.ndarray:
+    """x ~ N(0, 1) rounded to bf16: [B][H] uint16 bit patterns."""
+    return normal_bf16((B, H), 1.0, seed)
+
+
+def activations_f32(B: int, H: int, seed: int = SEED_X) -> np.ndarray:
+    return _rng(seed, 1).standard_normal(size=(B, H), dtype=np.float32)
+
+
+def norm_weight(H: int, layer: int = 0, seed: int = SEED_NORM) -> np.ndarray:
+    """RMSNorm gain 1 + N(0, 0.02), float32 [H]."""
+    return (1.0 + 0.02 * _rng(seed + layer).standard_normal(size=H)).astype(np.float32)
+
+
+def routing_lut(V: int, p_dense: float, seed: int = SEED_LUT) -> np.ndarray:
+    """Bernoulli(p_dense) table over the vocabulary; 1 = base (dense) path."""
+    return (_rng(seed).random(V) < p_dense).astype(np.uint8)
+
+
+def token_ids_uniform(B: int, V: int, seed: int = SEED_IDS) -> np.ndarray:
+    return _rng(seed).integers(0, V, size=B, dtype=np.int64).astype(np.int32)
+
+
+def token_ids_zipf(B: int, V: int, s: float = 1.1, seed: int = SEED_IDS) -> np.ndarray:
+    """Zipf(s) truncated to V ranks via its explicit CDF; rank r -> token id r-1."""
+    ranks = np.arange(1, V + 1, dtype=np.float64)
+    p = ranks ** (-s)
+    cdf = np.cumsum(p)
+    cdf /= cdf[-1]
+    u = _rng(seed).random(B)
+    return np.minimum(np.searchsorted(cdf, u, side="right"), V - 1).astype(np.int32)
+
+
+def stack_sparsity_targets(L: int, lo: float, hi: float, seed: int = SEED_SHUFFLE) -> np.ndarray:
+    """L evenly spaced targets in [lo, hi] (mean (lo+hi)/2), assigned to layers by a seeded shuffle."""
+    base = lo + (hi - lo) * (np.arange(L) + 0.5) / L
+    return base[_rng(seed).permutation(L)]
+
+
+# The five workloads, by what they are.
+WORKLOADS: Dict[str, dict] = {
+    "small_layer_512x1408_b1": dict(H=SMALL_H, N=SMALL_N, B=1, calib=64, sparsity=[0.5]),
+    "llama_layer_4096x14336_b1": dict(H=LLAMA_H, N=LLAMA_N, B=1, calib=256, sparsity=[0.5, 0.7, 0.9]),
+    "llama_stack_32x4096x14336_b1x128": dict(H=LLAMA_H, N=LLAMA_N, L=LLAMA_L, B=1, tokens=128,
+                                            sparsity_range=(0.55, 0.85), eps=1e-5),
+    "qwen_stack_36x4096x12288_routed": dict(H=QWEN_H, N=QWEN_N, L=QWEN_L, V=QWEN_V, batches=[1, 8, 32, 64],
+                                           p_dense=0.3, sparsity=0.5, eps=1e-6),
+    "llama_layer_prefill_routed": dict(H=LLAMA_H, N=LLAMA_N, V=LLAMA_V, batches=[256, 2048], zipf_s=1.1,
+                                       p_dense=0.2, sparsity=[0.4, 0.6, 0.8, 0.9]),
+}
