@@ -1,0 +1,385 @@
+"""Benchmark of the thresholded gated-MLP decode path on one GB300.
+
+Workload (by what it is): one Llama-3.1-8B-shaped MLP block (hidden 4096,
+intermediate 14336), bf16 weights ~ N(0, 0.02), one decode token x ~ N(0, 1)
+in bf16, thresholds t_l from 256 seeded calibration vectors (Eq. 3) at 50 %,
+70 % and 90 % target sparsity.  One step = three sats_sparse_mlp calls, one
+per sparsity level, each writing y and the compacted active-index list.
+Each call reads a different one of four device copies of the layer, so a copy
+is reused only after >= 420 MB of other weights have streamed (inputs larger
+than the 129 MB L2).
+
+Prints one JSON line.  `--impl reference` times the CPU oracle instead (the
+reference arm of this comparison), on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2607_08991_gb300 import inputs  # noqa: E402
+
+WORKLOAD = "llama_layer_4096x14336_b1"
+SPARSITY = (0.5, 0.7, 0.9)
+METRIC = "MLP decode us/token & achieved HBM GB/s vs peak at 50/70/90% sparsity"
+LAYER_COPIES = 4
+N_CALIB = 256
+FUSED_SRC = os.path.join(ROOT, "paper_2607_08991_gb300", "csrc", "fused_mlp.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fused_mlp_llama_layer_b1.md")
+NOMINAL_HBM_GBS = 8000.0
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        return float(pk["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _src_hash(path):
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def _ncu_traffic():
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on this kernel source."""
+    try:
+        lines = open(TRAFFIC_FILE).read().splitlines()
+    except OSError:
+        return None
+    vals = {}
+    for ln in lines:
+        if ":" in ln and ln.strip().startswith("- "):
+            k, v = ln.strip()[2:].split(":", 1)
+            vals[k.strip()] = v.strip().strip("`")
+    if vals.get("kernel_source_sha256_16") != _src_hash(FUSED_SRC):
+        return None
+    try:
+        return {s: float(vals["dram_bytes_per_launch_s%d" % int(round(100 * s))]) for s in SPARSITY}
+    except (KeyError, ValueError):
+        return None
+
+
+class Clocks:
+    """Samples SM clocks and throttle reasons with nvidia-smi during the timed region."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, local: int):
+        vis = [v.strip() for v in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if v.strip()]
+        self.index = vis[local] if local < len(vis) else str(local)
+        self.proc = None
+        self.path = os.path.join("/tmp", "sats_clocks_%d_%d.csv" % (os.getpid(), local))
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", self.index, "--query-gpu=" + self.QUERY,
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        try:
+            for ln in open(self.path):
+                f = [c.strip() for c in ln.split(",")]
+                if len(f) < 9:
+                    continue
+                try:
+                    sm.append(float(f[1]))
+                    mx.append(float(f[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, f[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        finally:
+            try:
+                os.unlink(self.path)
+            except OSError:
+                pass
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def _dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+# ---------------------------------------------------------------------------- CPU oracle arm
+def _oracle_sample(budget_s: float, max_calls: int = 64):
+    """Times the oracle on the workload: one token through the layer per call, cycling sparsity levels."""
+    import oracle
+    oracle.build()
+    H, N = inputs.LLAMA_H, inputs.LLAMA_N
+    w = inputs.mlp_weights(H, N)
+    x = oracle.bf16_to_f64(inputs.activations_bf16(1, H))
+    cal = oracle.bf16_to_f64(inputs.activations_bf16(4, H, seed=inputs.SEED_CALIB))
+    a_cal = oracle.gate_act(cal, w.Wg)
+    ts = [oracle.percentile_threshold(a_cal, s) for s in SPARSITY]
+    times = []
+    t_all = time.perf_counter()
+    i = 0
+    while i < max_calls and (i < len(SPARSITY) or time.perf_counter() - t_all < budget_s):
+        t0 = time.perf_counter()
+        oracle.sparse_mlp(x, w.Wg, w.Wu, w.Wd, ts[i % len(SPARSITY)])
+        times.append(time.perf_counter() - t0)
+        i += 1
+    us = 1e6 * sum(times) / len(times)
+    return us, len(times), "%d single-token calls (hidden 4096, intermediate 14336, thresholds at %s " \
+                           "sparsity from 4 calibration vectors)" % (len(times), "/".join(str(s) for s in SPARSITY))
+
+
+def run_reference(args):
+    ws, rank, _ = _dist_env()
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    H, N = inputs.LLAMA_H, inputs.LLAMA_N
+    w = inputs.mlp_weights(H, N)
+    x = oracle.bf16_to_f64(inputs.activations_bf16(1, H))
+    cal = oracle.bf16_to_f64(inputs.activations_bf16(4, H, seed=inputs.SEED_CALIB))
+    a_cal = oracle.gate_act(cal, w.Wg)
+    ts = [oracle.percentile_threshold(a_cal, s) for s in SPARSITY]
+    # one step = one token through the layer at one sparsity level (cycling), a bounded sample
+    for i in range(args.warmup):
+        oracle.sparse_mlp(x, w.Wg, w.Wu, w.Wd, ts[i % 3])
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        oracle.sparse_mlp(x, w.Wg, w.Wu, w.Wd, ts[i % 3])
+    el = time.perf_counter() - t0
+    us = 1e6 * el / args.steps
+    sample = "%d single-token calls of the layer, sparsity cycling %s" % (args.steps, "/".join(map(str, SPARSITY)))
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": us, "unit": "us/token", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": WORKLOAD, "hidden": H, "intermediate": N, "tokens": 1,
+                                        "sparsity": list(SPARSITY)},
+        "cpu_baseline": {"value": us, "unit": "us/token", "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": us, "unit": "us/token", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+# ---------------------------------------------------------------------------- GPU arm
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_08991_gb300 import sats
+
+    world, rank, local = _dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    H, N = inputs.LLAMA_H, inputs.LLAMA_N
+    stream = torch.cuda.Stream(device=dev)
+    w = inputs.mlp_weights(H, N)
+    with torch.cuda.stream(stream):
+        src = [torch.from_numpy(m.view(np.int16)).to(dev) for m in (w.Wg, w.Wu, w.Wd)]
+        layers = [sats.Layer(*src, stream=stream) for _ in range(LAYER_COPIES)]
+        del src
+        ws = sats.Workspace(H, N, 1, device=dev, stream=stream)
+        # thresholds: Eq. 3 on the post-gate activations of 256 calibration vectors
+        xc = torch.from_numpy(inputs.activations_bf16(N_CALIB, H, seed=inputs.SEED_CALIB).view(np.int16)).to(dev)
+        a = torch.empty(N_CALIB, N, dtype=torch.float32, device=dev)
+        sats.gate_act(layers[0], xc, a, stream=stream)
+        sel = torch.empty(sats.select_workspace_bytes(), dtype=torch.uint8, device=dev)
+        ts = [sats.percentile_threshold(a, s, sel, stream=stream) for s in SPARSITY]
+        del a, xc
+        x = torch.from_numpy(inputs.activations_bf16(1, H).view(np.int16)).to(dev)
+        y = torch.empty(1, H, dtype=torch.float32, device=dev)
+        idx = torch.empty(1, N, dtype=torch.int32, device=dev)
+        cnt = torch.empty(1, dtype=torch.int32, device=dev)
+    stream.synchronize()
+
+    calls = [(i, ts[i]) for i in range(len(SPARSITY))]
+    copy = [0]
+
+    def one_call(si, t, ev0=None, ev1=None):
+        layer = layers[copy[0] % LAYER_COPIES]
+        copy[0] += 1
+        if ev0 is not None:
+            ev0.record(stream)
+        sats.sparse_mlp(layer, x, t, y, ws, idx, cnt, stream=stream)
+        if ev1 is not None:
+            ev1.record(stream)
+
+    # realised sparsity per level
+    realised = []
+    for si, t in calls:
+        one_call(si, t)
+        stream.synchronize()
+        realised.append(1.0 - int(cnt.item()) / N)
+    assert sats.get_error(ws, stream=stream) == sats.OK
+
+    for _ in range(max(args.warmup, 3)):
+        for si, t in calls:
+            one_call(si, t)
+    K = args.steps
+    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in calls]
+           for _ in range(K)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = Clocks(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    time.sleep(0.3)
+    start.record(stream)
+    for k in range(K):
+        for (si, t), (e0, e1) in zip(calls, evs[k]):
+            one_call(si, t, e0, e1)
+    stop.record(stream)
+    stop.synchronize()
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    status = sats.get_error(ws, stream=stream)
+    if status != sats.OK:
+        raise RuntimeError("device status after the timed region: " + sats.status_string(status))
+    total_ms = start.elapsed_time(stop)
+    per_call_us = [[1e3 * evs[k][i][0].elapsed_time(evs[k][i][1]) for k in range(K)] for i in range(len(calls))]
+    mean_us = [sum(v) / len(v) for v in per_call_us]
+
+    # dense path on the same copies, for the speedup
+    dense_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    for i in range(3 + K):
+        layer = layers[i % LAYER_COPIES]
+        if i >= 3:
+            dense_ev[i - 3][0].record(stream)
+        sats.dense_mlp(layer, x, y, ws, stream=stream)
+        if i >= 3:
+            dense_ev[i - 3][1].record(stream)
+    stream.synchronize()
+    dense_us = 1e3 * sum(a.elapsed_time(b) for a, b in dense_ev) / K
+
+    # end to end through the C ABI with host buffers: x host->device, y and count device->host
+    xh = torch.from_numpy(inputs.activations_bf16(1, H).view(np.int16)).pin_memory()
+    yh = torch.empty(1, H, dtype=torch.float32).pin_memory()
+    ch = torch.empty(1, dtype=torch.int32).pin_memory()
+    Ke = max(10, K // 4)
+    e2e_s, e2e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for rep in range(2):
+        if rep == 1:
+            e2e_s.record(stream)
+        for k in range(Ke if rep else 3):
+            for si, t in calls:
+                with torch.cuda.stream(stream):
+                    x.copy_(xh, non_blocking=True)
+                one_call(si, t)
+                with torch.cuda.stream(stream):
+                    yh.copy_(y, non_blocking=True)
+                    ch.copy_(cnt, non_blocking=True)
+            stream.synchronize()
+        if rep == 1:
+            e2e_e.record(stream)
+    stream.synchronize()
+    e2e_us = 1e3 * e2e_s.elapsed_time(e2e_e) / (Ke * len(calls))
+
+    # aggregate over ranks (replicas): max time
+    if world > 1:
+        tt = torch.tensor([total_ms, e2e_us], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms, e2e_us = float(tt[0]), float(tt[1])
+    if rank == 0:
+        hbm_peak, peak_kind = _peaks()
+        per = {}
+        bytes_all, us_all = 0.0, 0.0
+        for i, s in enumerate(SPARSITY):
+            kept = (1.0 - realised[i]) * N
+            algo = 2.0 * H * N + kept * 4.0 * H + 2.0 * H + 4.0 * H + 4.0 * kept + 4.0
+            gbs = algo / (mean_us[i] * 1e-6) / 1e9
+            per[str(s)] = {"us": mean_us[i], "realised_sparsity": realised[i], "algo_bytes": algo,
+                           "achieved_gbs": gbs, "frac_of_%s" % peak_kind: gbs / hbm_peak,
+                           "frac_of_8tbs": gbs / NOMINAL_HBM_GBS, "speedup_vs_dense": dense_us / mean_us[i]}
+            bytes_all += algo
+            us_all += mean_us[i]
+        achieved = bytes_all / (us_all * 1e-6) / 1e9
+        traffic = _ncu_traffic()
+        value = total_ms * 1e3 / (K * len(calls) * world)
+        line = {
+            "metric": METRIC, "value": value, "unit": "us/token", "n_gpus": world, "steps": K,
+            "warmup": max(args.warmup, 3), "ms_per_step": total_ms / K, "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "hidden": H, "intermediate": N, "tokens": 1,
+                       "sparsity": list(SPARSITY), "calibration_vectors": N_CALIB,
+                       "l2": "inputs larger than L2: %d rotating device copies of the layer (%.2f GB)"
+                             % (LAYER_COPIES, LAYER_COPIES * 6.0 * H * N / 1e9),
+                       "parallelism": "replicas" if world > 1 else "single"},
+            "per_sparsity": per,
+            "dense": {"us": dense_us},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                         "frac": achieved / hbm_peak, "peak_kind": peak_kind,
+                         "traffic": None if traffic is None else
+                         sum(traffic[s] for s in SPARSITY) / len(SPARSITY),
+                         "kernel": "fused_mlp_kernel<1,2>"},
+            "e2e": {"value": e2e_us, "unit": "us/token", "h2d_bytes_per_step": len(calls) * 2 * H,
+                    "d2h_bytes_per_step": len(calls) * (4 * H + 4)},
+            "gpu_launches": K * len(calls),
+            "clocks": clk,
+        }
+        if not args.no_cpu_baseline:
+            us, n, sample = _oracle_sample(args.cpu_seconds)
+            line["cpu_baseline"] = {"value": us, "unit": "us/token", "cores": 1, "kind": "oracle", "sample": sample}
+        print(json.dumps(line))
+    for l in layers:
+        l.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="sats", choices=["sats", "reference"])
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,207 @@
+/*
+ * sats.h -- C ABI of the GB300 (sm_103a) library for the runtime path of
+ * "Sensitivity-Aware Thresholding and Token Routing for Activation
+ * Sparsification in Large Language Models" (arXiv 2607.08991).
+ *
+ * The path: the CATS-thresholded gated MLP (Sec. 2, Eqs. 1-5; SATS, Sec. 3.1,
+ * keeps this runtime mask and only chooses the per-layer threshold t_l), run
+ * under per-token routing between the base (dense) and sparse MLP through a
+ * vocabulary lookup table (Sec. 3.2, Eq. 13 and Fig. 2), chained over a
+ * stack of decoder MLP blocks with RMSNorm and a residual add.
+ *
+ * Conventions for every call
+ *   - Matrices follow the paper's row-vector convention y = x W: W_gate and
+ *     W_up are [H][N] (hidden x intermediate), W_down is [N][H]; activations
+ *     are [B][H].  All arrays are row-major and contiguous.
+ *   - bf16 data is passed as its 16-bit patterns (const void*, 2 bytes each).
+ *   - Pointers marked "device" are CUDA device pointers on the current device;
+ *     "host" pointers are ordinary host memory.  The caller owns every buffer
+ *     it passes; the library keeps no pointer to caller memory after a call
+ *     returns, except that work it enqueued on `stream` reads/writes them.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Every call
+ *     that takes a stream only enqueues work on it and returns without
+ *     synchronising, unless stated otherwise.
+ *   - Argument errors are detected on the host and returned before anything is
+ *     enqueued.  Errors found by a kernel (a token id outside the vocabulary, a
+ *     wait that ran out of time) are recorded in a status word in the
+ *     workspace (or in the caller's status word for sats_route) and returned by
+ *     sats_get_error.  No call aborts, throws, or traps on the device.
+ *   - Calls never allocate device memory, except sats_layer_create.
+ *   - Requirements: H a multiple of 8 and 8 <= H <= 8192; N >= 1; B >= 0.
+ */
+#ifndef SATS_H
+#define SATS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SATS_API __attribute__((visibility("default")))
+#else
+#define SATS_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    SATS_OK = 0,
+    SATS_EINVAL = 1,    /* null pointer, negative size, NaN or negative threshold, bad k */
+    SATS_ESHAPE = 2,    /* H not a multiple of 8, H or N out of range */
+    SATS_ECUDA = 3,     /* a CUDA runtime call failed (launch, copy, allocation) */
+    SATS_EDEVICE = 4,   /* a kernel reported bad input (token id outside [0, V)) */
+    SATS_ETIMEOUT = 5,  /* a bounded device-side wait gave up */
+    SATS_ENOSPACE = 6   /* workspace smaller than sats_workspace_bytes() */
+} sats_status;
+
+/* Opaque handle of one MLP block; owns its repacked device weights. */
+typedef struct sats_layer sats_layer;
+
+/* Library version, (major << 16) | minor. */
+SATS_API int sats_version(void);
+
+/* Human-readable name of a status code (static string, never NULL). */
+SATS_API const char *sats_status_string(sats_status s);
+
+/*
+ * sats_layer_create -- repack one gated-MLP block (Sec. 2, Eq. 1) for the
+ * runtime path.
+ *   W_gate, W_up : device bf16 [H][N];  W_down : device bf16 [N][H].
+ * The handle stores two device arrays that it allocates (the only allocation
+ * in this library): Wg_t [N][H] (row j = column j of W_gate) and
+ * W_ud [N][2H] (row j = column j of W_up followed by row j of W_down), so that
+ * the weights a kept neuron needs are one contiguous 4H-byte row and a
+ * skipped neuron costs no memory traffic.  The repacking runs on `stream`;
+ * the call synchronises `stream` before returning, after which the caller may
+ * free the three source arrays.  *out receives the handle.
+ */
+SATS_API sats_status sats_layer_create(const void *W_gate, const void *W_up, const void *W_down,
+                              int H, int N, void *stream, sats_layer **out);
+
+/* Frees the handle's device arrays (synchronises the device first). */
+SATS_API sats_status sats_layer_destroy(sats_layer *layer);
+
+/* Reads back H and N of a layer (host outputs, may be NULL). */
+SATS_API sats_status sats_layer_shape(const sats_layer *layer, int *H, int *N);
+
+/*
+ * Workspace.  Every compute call takes a device workspace `ws` of at least
+ * sats_workspace_bytes(H, N, B) bytes (B = the largest batch the caller will
+ * pass).  It holds cross-block partial sums, scheduling counters, the
+ * compacted per-chunk index lists and the device status word.  It must be
+ * zero-filled once before first use (sats_workspace_init does that on
+ * `stream`); every call leaves its counters at zero for the next call.  Calls
+ * that share one workspace must not overlap on the GPU.
+ */
+SATS_API size_t sats_workspace_bytes(int H, int N, int B);
+SATS_API sats_status sats_workspace_init(void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * sats_sparse_mlp -- the CATS-thresholded gated MLP (Sec. 2, Eqs. 1-5):
+ *   a = SiLU(x W_gate);  keep_j = |a_j| >= t_l;  y = ((keep * a) * (x W_up)) W_down
+ * for each of B tokens, bf16 weights with fp32 accumulation.  Only the
+ * W_up columns and W_down rows of kept neurons are read.
+ *   x          : device bf16 [B][H]
+ *   t_l        : threshold, >= 0 (0 keeps every neuron: the dense MLP;
+ *                +inf keeps none and gives y = 0).  NaN or < 0 -> SATS_EINVAL.
+ *   y          : device fp32 [B][H], written.
+ *   active_idx : device int32 [B][N] or NULL.  Row b receives the kept neuron
+ *                indices of token b in increasing order (entries past the
+ *                count are unspecified).
+ *   active_cnt : device int32 [B] or NULL; the number of kept neurons per token.
+ * active_idx and active_cnt must both be NULL or both be given.
+ */
+SATS_API sats_status sats_sparse_mlp(const sats_layer *layer, const void *x, int B, float t_l,
+                            float *y, int32_t *active_idx, int32_t *active_cnt,
+                            void *ws, size_t ws_bytes, void *stream);
+
+/* As sats_sparse_mlp, with fp32 activations x: device fp32 [B][H]. */
+SATS_API sats_status sats_sparse_mlp_f32(const sats_layer *layer, const float *x, int B, float t_l,
+                                float *y, int32_t *active_idx, int32_t *active_cnt,
+                                void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * sats_dense_mlp -- the base gated MLP of Sec. 2, Eq. 1 (every neuron kept):
+ *   x : device bf16 [B][H];  y : device fp32 [B][H].
+ */
+SATS_API sats_status sats_dense_mlp(const sats_layer *layer, const void *x, int B, float *y,
+                           void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * sats_route -- token routing by lookup table (Sec. 3.2, Eq. 13; Fig. 2).
+ *   token_ids : device int32 [B]
+ *   lut       : device uint8 [V]; lut[v] != 0 sends token id v to the base
+ *               (dense) path, 0 to the sparse path.
+ *   perm      : device int32 [B], written: the positions b of base-path tokens
+ *               in increasing order, then those of sparse-path tokens in
+ *               increasing order (a stable partition, bit-exact).
+ *   n_dense   : device int32 [1], written: the number of base-path tokens.
+ *   dev_status: device int32 [1] or NULL.  If a token id lies outside [0, V)
+ *               the kernel ORs 1 into *dev_status and routes that token to the
+ *               base path; sats_get_status_word reads it back.
+ */
+SATS_API sats_status sats_route(const int32_t *token_ids, int B, const uint8_t *lut, int V,
+                       int32_t *perm, int32_t *n_dense, int32_t *dev_status, void *stream);
+
+/*
+ * sats_mlp_stack -- L decoder MLP blocks on a residual stream:
+ *   for l in 0..L-1:  x <- x + MLP_l( RMSNorm(x) * norm_w[l] )
+ * with RMSNorm(x) = x / sqrt(mean(x^2) + eps).  Routing (Sec. 3.2) is decided
+ * once per token from its id and holds in every block: a base-path token uses
+ * the dense MLP (Eq. 1), a sparse-path token the CATS mask with threshold t[l]
+ * (Eq. 5).  token_ids == NULL sends every token to the sparse path.
+ *   layers    : host array of L layer handles (all with the same H, N)
+ *   norm_w    : host array of L device fp32 [H] RMSNorm gains
+ *   t         : host fp32 [L], per-layer thresholds (>= 0, not NaN)
+ *   token_ids : device int32 [B] or NULL;  lut : device uint8 [V] (V >= 1 when ids given)
+ *   x         : device fp32 [B][H], read and overwritten in place.
+ *   keep_trace: device uint8 [L][B][N] or NULL; receives each block's keep mask
+ *               per token (1 = neuron used), for verification.
+ * A token id outside [0, V) is routed to the base path and sets the
+ * workspace status word (SATS_EDEVICE from sats_get_error).
+ */
+SATS_API sats_status sats_mlp_stack(const sats_layer *const *layers, const float *const *norm_w,
+                           const float *t, int L, float eps,
+                           const int32_t *token_ids, const uint8_t *lut, int V,
+                           float *x, int B, uint8_t *keep_trace,
+                           void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * sats_gate_act -- calibration helper: a = SiLU(x W_gate) (Sec. 2, Eqs. 1-2)
+ * for B tokens, the post-gate activations from which thresholds are chosen
+ * (Eq. 3 for CATS; candidate set T_l for SATS, Sec. 3.1).
+ *   x : device bf16 [B][H];  a : device fp32 [B][N], written.
+ */
+SATS_API sats_status sats_gate_act(const sats_layer *layer, const void *x, int B, float *a,
+                          void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * sats_percentile_threshold -- Eq. 3: t = min{t' : F(t') >= k}, F the empirical
+ * CDF of |a_i| over n values, i.e. the m-th smallest |a_i| with m = ceil(k n)
+ * (k read as a decimal fraction; k*n is taken down by a relative 2^-50 before
+ * the ceiling).  k <= 0 gives 0, k > 1 gives +inf.
+ *   a      : device fp32 [n] (NaN not allowed)
+ *   t_out  : host fp32 [1], written.
+ *   ws     : device workspace of at least sats_select_workspace_bytes() bytes.
+ * Synchronises `stream` (the result is returned on the host).
+ */
+SATS_API size_t sats_select_workspace_bytes(void);
+SATS_API sats_status sats_percentile_threshold(const float *a, int64_t n, double k, float *t_out,
+                                      void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * sats_get_error -- synchronises `stream`, reads the status word in the
+ * workspace, clears it, and returns SATS_OK, SATS_EDEVICE (bad token id) or
+ * SATS_ETIMEOUT (a device wait gave up).
+ */
+SATS_API sats_status sats_get_error(void *ws, size_t ws_bytes, void *stream);
+
+/* Same for a caller-owned status word (as passed to sats_route). */
+SATS_API sats_status sats_get_status_word(int32_t *dev_status, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SATS_H */

@@ -1,0 +1,306 @@
+// api.cu -- the C ABI declared in include/sats.h: argument checks, the
+// workspace layout, and the host-side drivers that split a batch into passes
+// of the fused kernel and chain the blocks of a stack.
+#include <cmath>
+#include <cstring>
+#include <new>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace sats {
+
+static size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+static int nchunks_of(int N) { return (N + kChunk - 1) / kChunk; }
+
+WsLayout ws_layout(int H, int N, int B)
+{
+    WsLayout L{};
+    const size_t nc = (size_t)nchunks_of(N);
+    size_t off = 0;
+    L.ctl = off;
+    off += align256(kCtlInts * sizeof(int));
+    L.partials = off;
+    off += align256((size_t)kMaxGrid * kMaxTokensPerPass * H * sizeof(float));
+    L.chunk_cnt = off;
+    off += align256(nc * kMaxTokensPerPass * sizeof(int));
+    L.idx_tmp = off;
+    off += align256((size_t)kMaxTokensPerPass * nc * kChunk * sizeof(int));
+    L.route_perm = off;
+    off += align256((size_t)(B > 0 ? B : 1) * sizeof(int32_t));
+    L.route_flags = off;
+    off += align256((size_t)(B > 0 ? B : 1));
+    L.total = off;
+    return L;
+}
+
+static bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+static sats_status from_cuda(cudaError_t e) { return e == cudaSuccess ? SATS_OK : SATS_ECUDA; }
+
+static bool bad_threshold(float t) { return std::isnan(t) || t < 0.0f; }
+
+// Runs the fused kernel over B tokens in passes of up to 4 (H <= 4096) or 2.
+static sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B, const float *t_per_pass_l,
+                             const float *norm_w, float eps, const uint8_t *dense_flags, int out_mode, float *out,
+                             int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws,
+                             cudaStream_t stream)
+{
+    const int H = layer->H, N = layer->N;
+    const WsLayout L = ws_layout(H, N, B);
+    char *base = static_cast<char *>(ws);
+    const int per_pass = H > 4096 ? 2 : kMaxTokensPerPass;
+    const size_t x_elem = (x_mode == kXBf16) ? 2 : 4;
+    for (int b0 = 0; b0 < B; b0 += per_pass) {
+        FusedParams p{};
+        p.wg_t = layer->wg_t;
+        p.w_ud = layer->w_ud;
+        p.H = H;
+        p.N = N;
+        p.nchunks = nchunks_of(N);
+        p.nb = B - b0 < per_pass ? B - b0 : per_pass;
+        p.x_mode = x_mode;
+        p.x = static_cast<const char *>(x) + (size_t)b0 * H * x_elem;
+        p.norm_w = norm_w;
+        p.eps = eps;
+        p.t_l = *t_per_pass_l;
+        p.dense_flags = dense_flags ? dense_flags + b0 : nullptr;
+        p.out_mode = out_mode;
+        p.out = out + (size_t)b0 * H;
+        p.ctl = reinterpret_cast<int *>(base + L.ctl);
+        p.partials = reinterpret_cast<float *>(base + L.partials);
+        p.chunk_cnt = reinterpret_cast<int *>(base + L.chunk_cnt);
+        p.idx_tmp = reinterpret_cast<int *>(base + L.idx_tmp);
+        p.active_idx = active_idx ? active_idx + (size_t)b0 * N : nullptr;
+        p.active_cnt = active_cnt ? active_cnt + b0 : nullptr;
+        p.keep_trace = keep_trace ? keep_trace + (size_t)b0 * N : nullptr;
+        const cudaError_t e = launch_fused(p, stream);
+        if (e != cudaSuccess) return SATS_ECUDA;
+    }
+    return SATS_OK;
+}
+
+static sats_status check_layer(const sats_layer *layer, void *ws, size_t ws_bytes, int B)
+{
+    if (!layer || !ws) return SATS_EINVAL;
+    if (B < 0) return SATS_EINVAL;
+    if (!aligned16(ws)) return SATS_EINVAL;
+    if (ws_bytes < ws_layout(layer->H, layer->N, B).total) return SATS_ENOSPACE;
+    return SATS_OK;
+}
+
+static sats_status sparse_common(const sats_layer *layer, int x_mode, const void *x, int B, float t_l, float *y,
+                                 int32_t *active_idx, int32_t *active_cnt, void *ws, size_t ws_bytes, void *stream)
+{
+    sats_status s = check_layer(layer, ws, ws_bytes, B);
+    if (s != SATS_OK) return s;
+    if (bad_threshold(t_l)) return SATS_EINVAL;
+    if ((active_idx == nullptr) != (active_cnt == nullptr)) return SATS_EINVAL;
+    if (B == 0) return SATS_OK;
+    if (!x || !y || !aligned16(x) || !aligned16(y)) return SATS_EINVAL;
+    return run_layer(layer, x_mode, x, B, &t_l, nullptr, 0.f, nullptr, kOutY, y, active_idx, active_cnt, nullptr,
+                     ws, static_cast<cudaStream_t>(stream));
+}
+
+}  // namespace sats
+
+using namespace sats;
+
+extern "C" {
+
+int sats_version(void) { return (1 << 16) | 0; }
+
+const char *sats_status_string(sats_status s)
+{
+    switch (s) {
+    case SATS_OK: return "ok";
+    case SATS_EINVAL: return "invalid argument";
+    case SATS_ESHAPE: return "unsupported shape";
+    case SATS_ECUDA: return "CUDA runtime error";
+    case SATS_EDEVICE: return "bad input detected on the device (token id outside the vocabulary)";
+    case SATS_ETIMEOUT: return "a bounded device-side wait gave up";
+    case SATS_ENOSPACE: return "workspace too small";
+    }
+    return "unknown status";
+}
+
+sats_status sats_layer_create(const void *W_gate, const void *W_up, const void *W_down, int H, int N, void *stream,
+                              sats_layer **out)
+{
+    if (!out) return SATS_EINVAL;
+    *out = nullptr;
+    if (!W_gate || !W_up || !W_down) return SATS_EINVAL;
+    if (H < 8 || H > kMaxH || (H % 8) != 0 || N < 1 || N > kMaxN) return SATS_ESHAPE;
+    sats_layer *l = new (std::nothrow) sats_layer();
+    if (!l) return SATS_ECUDA;
+    l->H = H;
+    l->N = N;
+    cudaGetDevice(&l->device);
+    const size_t row_elems = (size_t)N * H;
+    if (cudaMalloc(&l->wg_t, row_elems * 2) != cudaSuccess) { delete l; return SATS_ECUDA; }
+    if (cudaMalloc(&l->w_ud, row_elems * 4) != cudaSuccess) { cudaFree(l->wg_t); delete l; return SATS_ECUDA; }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = launch_pack(static_cast<const uint16_t *>(W_gate), static_cast<const uint16_t *>(W_up),
+                                static_cast<const uint16_t *>(W_down), H, N, l->wg_t, l->w_ud, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) {
+        cudaFree(l->wg_t);
+        cudaFree(l->w_ud);
+        delete l;
+        return SATS_ECUDA;
+    }
+    *out = l;
+    return SATS_OK;
+}
+
+sats_status sats_layer_destroy(sats_layer *layer)
+{
+    if (!layer) return SATS_EINVAL;
+    cudaDeviceSynchronize();
+    cudaError_t e1 = cudaFree(layer->wg_t);
+    cudaError_t e2 = cudaFree(layer->w_ud);
+    delete layer;
+    return (e1 == cudaSuccess && e2 == cudaSuccess) ? SATS_OK : SATS_ECUDA;
+}
+
+sats_status sats_layer_shape(const sats_layer *layer, int *H, int *N)
+{
+    if (!layer) return SATS_EINVAL;
+    if (H) *H = layer->H;
+    if (N) *N = layer->N;
+    return SATS_OK;
+}
+
+size_t sats_workspace_bytes(int H, int N, int B)
+{
+    if (H < 8 || H > kMaxH || (H % 8) != 0 || N < 1 || N > kMaxN || B < 0) return 0;
+    return ws_layout(H, N, B).total;
+}
+
+sats_status sats_workspace_init(void *ws, size_t ws_bytes, void *stream)
+{
+    if (!ws) return SATS_EINVAL;
+    return from_cuda(cudaMemsetAsync(ws, 0, ws_bytes, static_cast<cudaStream_t>(stream)));
+}
+
+sats_status sats_sparse_mlp(const sats_layer *layer, const void *x, int B, float t_l, float *y, int32_t *active_idx,
+                            int32_t *active_cnt, void *ws, size_t ws_bytes, void *stream)
+{
+    return sparse_common(layer, kXBf16, x, B, t_l, y, active_idx, active_cnt, ws, ws_bytes, stream);
+}
+
+sats_status sats_sparse_mlp_f32(const sats_layer *layer, const float *x, int B, float t_l, float *y,
+                                int32_t *active_idx, int32_t *active_cnt, void *ws, size_t ws_bytes, void *stream)
+{
+    return sparse_common(layer, kXF32, x, B, t_l, y, active_idx, active_cnt, ws, ws_bytes, stream);
+}
+
+sats_status sats_dense_mlp(const sats_layer *layer, const void *x, int B, float *y, void *ws, size_t ws_bytes,
+                           void *stream)
+{
+    return sparse_common(layer, kXBf16, x, B, 0.0f, y, nullptr, nullptr, ws, ws_bytes, stream);
+}
+
+sats_status sats_route(const int32_t *token_ids, int B, const uint8_t *lut, int V, int32_t *perm, int32_t *n_dense,
+                       int32_t *dev_status, void *stream)
+{
+    if (B < 0 || V < 1 || !lut || !n_dense) return SATS_EINVAL;
+    if (B > 0 && (!token_ids || !perm)) return SATS_EINVAL;
+    return from_cuda(launch_route(token_ids, B, lut, V, perm, n_dense, nullptr, dev_status,
+                                  static_cast<cudaStream_t>(stream)));
+}
+
+sats_status sats_mlp_stack(const sats_layer *const *layers, const float *const *norm_w, const float *t, int L,
+                           float eps, const int32_t *token_ids, const uint8_t *lut, int V, float *x, int B,
+                           uint8_t *keep_trace, void *ws, size_t ws_bytes, void *stream)
+{
+    if (!layers || !norm_w || !t || L < 0 || B < 0 || !ws) return SATS_EINVAL;
+    if (std::isnan(eps) || eps < 0.0f) return SATS_EINVAL;
+    if (L == 0 || B == 0) return SATS_OK;
+    if (!x || !aligned16(x)) return SATS_EINVAL;
+    if (token_ids && (!lut || V < 1)) return SATS_EINVAL;
+    const int H = layers[0] ? layers[0]->H : 0, N = layers[0] ? layers[0]->N : 0;
+    for (int l = 0; l < L; ++l) {
+        if (!layers[l] || layers[l]->H != H || layers[l]->N != N) return SATS_EINVAL;
+        if (!norm_w[l] || !aligned16(norm_w[l])) return SATS_EINVAL;
+        if (bad_threshold(t[l])) return SATS_EINVAL;
+    }
+    sats_status s = check_layer(layers[0], ws, ws_bytes, B);
+    if (s != SATS_OK) return s;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const WsLayout W = ws_layout(H, N, B);
+    char *base = static_cast<char *>(ws);
+    int *ctl = reinterpret_cast<int *>(base + W.ctl);
+    uint8_t *flags = nullptr;
+    if (token_ids) {
+        flags = reinterpret_cast<uint8_t *>(base + W.route_flags);
+        cudaError_t e = launch_route(token_ids, B, lut, V, reinterpret_cast<int32_t *>(base + W.route_perm),
+                                     ctl + kCtlNDense, flags, ctl + kCtlStatus, st);
+        if (e != cudaSuccess) return SATS_ECUDA;
+    }
+    for (int l = 0; l < L; ++l) {
+        s = run_layer(layers[l], kXResidNorm, x, B, &t[l], norm_w[l], eps, flags, kOutResid, x, nullptr, nullptr,
+                      keep_trace ? keep_trace + (size_t)l * B * N : nullptr, ws, st);
+        if (s != SATS_OK) return s;
+    }
+    return SATS_OK;
+}
+
+sats_status sats_gate_act(const sats_layer *layer, const void *x, int B, float *a, void *ws, size_t ws_bytes,
+                          void *stream)
+{
+    (void)ws;
+    (void)ws_bytes;
+    if (!layer || B < 0) return SATS_EINVAL;
+    if (B == 0) return SATS_OK;
+    if (!x || !a || !aligned16(x)) return SATS_EINVAL;
+    return from_cuda(launch_gate_act(layer, static_cast<const uint16_t *>(x), B, a, static_cast<cudaStream_t>(stream)));
+}
+
+size_t sats_select_workspace_bytes(void) { return select_ws_bytes(); }
+
+sats_status sats_percentile_threshold(const float *a, int64_t n, double k, float *t_out, void *ws, size_t ws_bytes,
+                                      void *stream)
+{
+    if (!t_out || n < 0 || std::isnan(k)) return SATS_EINVAL;
+    if (n == 0 || !(k > 0.0)) { *t_out = 0.0f; return SATS_OK; }
+    if (k > 1.0) { *t_out = INFINITY; return SATS_OK; }
+    if (!a || !ws || ws_bytes < select_ws_bytes() || !aligned16(ws)) return SATS_EINVAL;
+    // m = ceil(k n), with k read as the decimal fraction it stands for
+    int64_t m = (int64_t)std::ceil((k * (double)n) * (1.0 - std::ldexp(1.0, -50)));
+    if (m < 1) m = 1;
+    if (m > n) m = n;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    float *t_dev = reinterpret_cast<float *>(static_cast<char *>(ws) + select_ws_bytes() - 128);
+    cudaError_t e = launch_select(a, n, m, ws, t_dev, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(t_out, t_dev, sizeof(float), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    return from_cuda(e);
+}
+
+static sats_status read_status(int32_t *word, cudaStream_t st)
+{
+    int32_t v = 0;
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) e = cudaMemcpy(&v, word, sizeof v, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && v != 0) e = cudaMemset(word, 0, sizeof v);
+    if (e != cudaSuccess) return SATS_ECUDA;
+    if (v & kStatusTimeout) return SATS_ETIMEOUT;
+    if (v & kStatusBadToken) return SATS_EDEVICE;
+    return SATS_OK;
+}
+
+sats_status sats_get_error(void *ws, size_t ws_bytes, void *stream)
+{
+    if (!ws || ws_bytes < (size_t)kCtlInts * sizeof(int)) return SATS_EINVAL;
+    return read_status(static_cast<int32_t *>(ws) + kCtlStatus, static_cast<cudaStream_t>(stream));
+}
+
+sats_status sats_get_status_word(int32_t *dev_status, void *stream)
+{
+    if (!dev_status) return SATS_EINVAL;
+    return read_status(dev_status, static_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

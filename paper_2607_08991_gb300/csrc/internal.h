@@ -1,0 +1,80 @@
+// internal.h -- declarations shared by the library's translation units.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "sats.h"
+
+struct sats_layer {
+    int H = 0;
+    int N = 0;
+    int device = 0;
+    uint16_t *wg_t = nullptr;   // [N][H]: row j = column j of W_gate
+    uint16_t *w_ud = nullptr;   // [N][2H]: row j = column j of W_up, then row j of W_down
+};
+
+namespace sats {
+
+constexpr int kChunk = 16;              // neurons per scheduling unit of the fused kernel
+constexpr int kMaxTokensPerPass = 4;    // tokens one fused launch carries
+constexpr int kMaxGrid = 256;           // upper bound of the fused grid (partials rows)
+constexpr int kMaxH = 8192;
+constexpr int kMaxN = 1 << 20;
+
+// Control block at the start of the workspace (ints).
+enum {
+    kCtlChunk = 0,      // dynamic chunk counter, reset to 0 by the grid barrier
+    kCtlBarCount = 1,   // grid barrier arrivals, reset to 0 by the last arrival
+    kCtlBarGen = 2,     // grid barrier generation
+    kCtlStatus = 3,     // device status word (kStatus* bits)
+    kCtlNDense = 4,     // route output of the stack driver
+    kCtlInts = 64
+};
+
+struct WsLayout {
+    size_t ctl, partials, chunk_cnt, idx_tmp, route_perm, route_flags, total;
+};
+WsLayout ws_layout(int H, int N, int B);
+
+enum XMode { kXBf16 = 0, kXF32 = 1, kXResidNorm = 2 };
+enum OutMode { kOutY = 0, kOutResid = 1 };
+
+struct FusedParams {
+    const uint16_t *wg_t;
+    const uint16_t *w_ud;
+    int H, N, nchunks;
+    int nb;                       // tokens in this pass, 1..kMaxTokensPerPass
+    int x_mode;
+    const void *x;                // first token of this pass ([nb][H])
+    const float *norm_w;          // kXResidNorm: RMSNorm gain [H]
+    float eps;
+    float t_l;                    // threshold of sparse-path tokens
+    const uint8_t *dense_flags;   // [nb] (1 = base path, threshold 0) or nullptr
+    int out_mode;
+    float *out;                   // kOutY: y [nb][H]; kOutResid: residual [nb][H] (+=)
+    int *ctl;                     // workspace control block
+    float *partials;              // [kMaxGrid][kMaxTokensPerPass][H]
+    int *chunk_cnt;               // [nchunks][kMaxTokensPerPass]
+    int *idx_tmp;                 // [kMaxTokensPerPass][nchunks * kChunk]
+    int32_t *active_idx;          // [nb][N] or nullptr
+    int32_t *active_cnt;          // [nb] or nullptr
+    uint8_t *keep_trace;          // [nb][N] or nullptr
+};
+
+// Number of CTAs the fused kernel runs with on `device` (all co-resident).
+int fused_grid(int nchunks);
+cudaError_t launch_fused(const FusedParams &p, cudaStream_t stream);
+
+cudaError_t launch_pack(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd, int H, int N,
+                        uint16_t *wg_t, uint16_t *w_ud, cudaStream_t stream);
+cudaError_t launch_route(const int32_t *ids, int B, const uint8_t *lut, int V, int32_t *perm,
+                         int32_t *n_dense, uint8_t *flags, int32_t *status, cudaStream_t stream);
+cudaError_t launch_gate_act(const sats_layer *layer, const uint16_t *x, int B, float *a,
+                            cudaStream_t stream);
+size_t select_ws_bytes();
+cudaError_t launch_select(const float *a, int64_t n, int64_t m, void *ws, float *t_dev,
+                          cudaStream_t stream);
+
+}  // namespace sats

@@ -1,0 +1,221 @@
+"""Python binding of libsats.so (include/sats.h): argument marshalling only.
+
+Every function here forwards to the C ABI of the same name (without the
+``sats_`` prefix).  Tensors are torch tensors on the current CUDA device; torch
+provides device memory and streams, the library's kernels do every step of the
+computation.  There is no fallback: if libsats.so is missing or fails to load,
+every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libsats.so")
+
+OK, EINVAL, ESHAPE, ECUDA, EDEVICE, ETIMEOUT, ENOSPACE = range(7)
+
+_lib = None
+
+
+class SatsError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__("%s: %s (status %d)" % (where, status_string(status), status))
+
+
+def lib() -> ctypes.CDLL:
+    """Loads libsats.so (built by paper_2607_08991_gb300.build); raises if absent."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError("libsats.so is not built (run __graft_entry__.build()); "
+                               "this library has no CPU fallback")
+        L = ctypes.CDLL(LIB_PATH)
+        P, I, F, D, Z, I64 = (ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_double,
+                              ctypes.c_size_t, ctypes.c_int64)
+        sig = {
+            "sats_version": (I, []),
+            "sats_status_string": (ctypes.c_char_p, [I]),
+            "sats_layer_create": (I, [P, P, P, I, I, P, ctypes.POINTER(P)]),
+            "sats_layer_destroy": (I, [P]),
+            "sats_layer_shape": (I, [P, ctypes.POINTER(I), ctypes.POINTER(I)]),
+            "sats_workspace_bytes": (Z, [I, I, I]),
+            "sats_workspace_init": (I, [P, Z, P]),
+            "sats_sparse_mlp": (I, [P, P, I, F, P, P, P, P, Z, P]),
+            "sats_sparse_mlp_f32": (I, [P, P, I, F, P, P, P, P, Z, P]),
+            "sats_dense_mlp": (I, [P, P, I, P, P, Z, P]),
+            "sats_route": (I, [P, I, P, I, P, P, P, P]),
+            "sats_mlp_stack": (I, [P, P, P, I, F, P, P, I, P, I, P, P, Z, P]),
+            "sats_gate_act": (I, [P, P, I, P, P, Z, P]),
+            "sats_select_workspace_bytes": (Z, []),
+            "sats_percentile_threshold": (I, [P, I64, D, ctypes.POINTER(F), P, Z, P]),
+            "sats_get_error": (I, [P, Z, P]),
+            "sats_get_status_word": (I, [P, P]),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def exported_symbols() -> Sequence[str]:
+    return [n for n in ("sats_version", "sats_status_string", "sats_layer_create", "sats_layer_destroy",
+                        "sats_layer_shape", "sats_workspace_bytes", "sats_workspace_init", "sats_sparse_mlp",
+                        "sats_sparse_mlp_f32", "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
+                        "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_get_error",
+                        "sats_get_status_word")]
+
+
+def status_string(s: int) -> str:
+    return lib().sats_status_string(int(s)).decode()
+
+
+def _check(s: int, where: str):
+    if s != OK:
+        raise SatsError(s, where)
+
+
+def _stream(stream: Optional[torch.cuda.Stream]):
+    st = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(st.cuda_stream)
+
+
+def _ptr(t: Optional[torch.Tensor], name: str, elem: Optional[int] = None):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("%s must be a CUDA tensor" % name)
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    if elem is not None and t.element_size() != elem:
+        raise ValueError("%s must have %d-byte elements" % (name, elem))
+    return ctypes.c_void_p(t.data_ptr())
+
+
+class Layer:
+    """Handle of one repacked MLP block (sats_layer_create / sats_layer_destroy)."""
+
+    def __init__(self, W_gate: torch.Tensor, W_up: torch.Tensor, W_down: torch.Tensor,
+                 stream: Optional[torch.cuda.Stream] = None):
+        H, N = W_gate.shape
+        if tuple(W_up.shape) != (H, N) or tuple(W_down.shape) != (N, H):
+            raise ValueError("expected W_gate, W_up [H][N] and W_down [N][H]")
+        h = ctypes.c_void_p()
+        _check(lib().sats_layer_create(_ptr(W_gate, "W_gate", 2), _ptr(W_up, "W_up", 2), _ptr(W_down, "W_down", 2),
+                                       H, N, _stream(stream), ctypes.byref(h)), "sats_layer_create")
+        self.handle = h
+        self.H, self.N = H, N
+
+    def close(self):
+        if self.handle is not None and self.handle.value:
+            _check(lib().sats_layer_destroy(self.handle), "sats_layer_destroy")
+        self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def workspace_bytes(H: int, N: int, B: int) -> int:
+    return int(lib().sats_workspace_bytes(H, N, B))
+
+
+class Workspace:
+    """A zero-initialised device workspace (torch memory) for calls up to batch B."""
+
+    def __init__(self, H: int, N: int, B: int, device=None, stream: Optional[torch.cuda.Stream] = None):
+        n = workspace_bytes(H, N, B)
+        if n == 0:
+            raise ValueError("unsupported shape for a workspace: H=%d N=%d B=%d" % (H, N, B))
+        self.buf = torch.empty(n, dtype=torch.uint8, device=device or "cuda")
+        self.nbytes = n
+        _check(lib().sats_workspace_init(_ptr(self.buf, "ws"), n, _stream(stream)), "sats_workspace_init")
+
+    @property
+    def ptr(self):
+        return ctypes.c_void_p(self.buf.data_ptr())
+
+
+def sparse_mlp(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor, ws: Workspace,
+               active_idx: Optional[torch.Tensor] = None, active_cnt: Optional[torch.Tensor] = None,
+               stream: Optional[torch.cuda.Stream] = None):
+    B = x.shape[0]
+    _check(lib().sats_sparse_mlp(layer.handle, _ptr(x, "x", 2), B, float(t_l), _ptr(y, "y", 4),
+                                 _ptr(active_idx, "active_idx", 4), _ptr(active_cnt, "active_cnt", 4),
+                                 ws.ptr, ws.nbytes, _stream(stream)), "sats_sparse_mlp")
+
+
+def sparse_mlp_f32(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor, ws: Workspace,
+                   active_idx: Optional[torch.Tensor] = None, active_cnt: Optional[torch.Tensor] = None,
+                   stream: Optional[torch.cuda.Stream] = None):
+    B = x.shape[0]
+    _check(lib().sats_sparse_mlp_f32(layer.handle, _ptr(x, "x", 4), B, float(t_l), _ptr(y, "y", 4),
+                                     _ptr(active_idx, "active_idx", 4), _ptr(active_cnt, "active_cnt", 4),
+                                     ws.ptr, ws.nbytes, _stream(stream)), "sats_sparse_mlp_f32")
+
+
+def dense_mlp(layer: Layer, x: torch.Tensor, y: torch.Tensor, ws: Workspace,
+              stream: Optional[torch.cuda.Stream] = None):
+    _check(lib().sats_dense_mlp(layer.handle, _ptr(x, "x", 2), x.shape[0], _ptr(y, "y", 4), ws.ptr, ws.nbytes,
+                                _stream(stream)), "sats_dense_mlp")
+
+
+def route(token_ids: torch.Tensor, lut: torch.Tensor, perm: torch.Tensor, n_dense: torch.Tensor,
+          dev_status: Optional[torch.Tensor] = None, stream: Optional[torch.cuda.Stream] = None):
+    _check(lib().sats_route(_ptr(token_ids, "token_ids", 4), token_ids.numel(), _ptr(lut, "lut", 1), lut.numel(),
+                            _ptr(perm, "perm", 4), _ptr(n_dense, "n_dense", 4), _ptr(dev_status, "dev_status", 4),
+                            _stream(stream)), "sats_route")
+
+
+def mlp_stack(layers: Sequence[Layer], norm_w: Sequence[torch.Tensor], t: Sequence[float], eps: float,
+              x: torch.Tensor, ws: Workspace, token_ids: Optional[torch.Tensor] = None,
+              lut: Optional[torch.Tensor] = None, keep_trace: Optional[torch.Tensor] = None,
+              stream: Optional[torch.cuda.Stream] = None):
+    L = len(layers)
+    hs = (ctypes.c_void_p * L)(*[l.handle.value for l in layers])
+    nws = (ctypes.c_void_p * L)(*[w.data_ptr() for w in norm_w])
+    for w in norm_w:
+        _ptr(w, "norm_w", 4)
+    ts = (ctypes.c_float * L)(*[float(v) for v in t])
+    _check(lib().sats_mlp_stack(hs, nws, ts, L, float(eps), _ptr(token_ids, "token_ids", 4), _ptr(lut, "lut", 1),
+                                0 if lut is None else lut.numel(), _ptr(x, "x", 4), x.shape[0],
+                                _ptr(keep_trace, "keep_trace", 1), ws.ptr, ws.nbytes, _stream(stream)),
+           "sats_mlp_stack")
+
+
+def gate_act(layer: Layer, x: torch.Tensor, a: torch.Tensor, ws: Optional[Workspace] = None,
+             stream: Optional[torch.cuda.Stream] = None):
+    _check(lib().sats_gate_act(layer.handle, _ptr(x, "x", 2), x.shape[0], _ptr(a, "a", 4),
+                               None if ws is None else ws.ptr, 0 if ws is None else ws.nbytes, _stream(stream)),
+           "sats_gate_act")
+
+
+def select_workspace_bytes() -> int:
+    return int(lib().sats_select_workspace_bytes())
+
+
+def percentile_threshold(a: torch.Tensor, k: float, sel_ws: torch.Tensor,
+                         stream: Optional[torch.cuda.Stream] = None) -> float:
+    out = ctypes.c_float()
+    _check(lib().sats_percentile_threshold(_ptr(a, "a", 4), a.numel(), float(k), ctypes.byref(out),
+                                           _ptr(sel_ws, "sel_ws"), sel_ws.numel() * sel_ws.element_size(),
+                                           _stream(stream)), "sats_percentile_threshold")
+    return float(out.value)
+
+
+def get_error(ws: Workspace, stream: Optional[torch.cuda.Stream] = None) -> int:
+    """Returns the device status of the workspace (OK, EDEVICE or ETIMEOUT) and clears it."""
+    return int(lib().sats_get_error(ws.ptr, ws.nbytes, _stream(stream)))
+
+
+def get_status_word(dev_status: torch.Tensor, stream: Optional[torch.cuda.Stream] = None) -> int:
+    return int(lib().sats_get_status_word(_ptr(dev_status, "dev_status", 4), _stream(stream)))

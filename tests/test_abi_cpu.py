@@ -1,0 +1,63 @@
+"""The C-ABI library builds, loads and exports every symbol include/sats.h
+declares; host-side argument checks answer without touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def libsats():
+    from paper_2607_08991_gb300 import build
+    path = build.build_library()
+    return ctypes.CDLL(path)
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "sats.h")).read()
+    return sorted(set(re.findall(r"SATS_API[^;(]*?\b(sats_\w+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for required in ("sats_sparse_mlp", "sats_route", "sats_mlp_stack", "sats_dense_mlp", "sats_layer_create"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(libsats):
+    for name in _declared():
+        assert hasattr(libsats, name), name
+
+
+def test_binding_covers_every_symbol():
+    from paper_2607_08991_gb300 import sats
+    assert sorted(sats.exported_symbols()) == _declared()
+
+
+def test_host_side_checks(libsats):
+    from paper_2607_08991_gb300 import sats
+    L = sats.lib()
+    assert L.sats_version() >> 16 == 1
+    assert sats.status_string(sats.ESHAPE) == "unsupported shape"
+    assert L.sats_workspace_bytes(12, 10, 1) == 0          # H not a multiple of 8
+    assert L.sats_workspace_bytes(8, 0, 1) == 0            # N < 1
+    assert L.sats_workspace_bytes(16384, 10, 1) == 0       # H too large
+    ws = L.sats_workspace_bytes(4096, 14336, 1)
+    assert ws >= 256 * 4 * 4096 * 4                       # partial sums of every CTA
+    assert L.sats_workspace_bytes(4096, 14336, 64) >= ws
+    out = ctypes.c_void_p()
+    # argument errors come back before any CUDA call
+    assert L.sats_layer_create(None, None, None, 64, 64, None, ctypes.byref(out)) == sats.EINVAL
+    assert L.sats_layer_create(1, 1, 1, 60, 64, None, ctypes.byref(out)) == sats.ESHAPE
+    assert L.sats_layer_create(1, 1, 1, 64, 0, None, None) == sats.EINVAL
+    assert L.sats_sparse_mlp(None, None, 1, 0.5, None, None, None, None, 0, None) == sats.EINVAL
+    assert L.sats_route(None, 4, None, 10, None, None, None, None) == sats.EINVAL
+    assert L.sats_mlp_stack(None, None, None, 1, 1e-5, None, None, 0, None, 1, None, None, 0, None) == sats.EINVAL
+    t = ctypes.c_float(-1.0)
+    assert L.sats_percentile_threshold(None, 0, 0.5, ctypes.byref(t), None, 0, None) == sats.OK and t.value == 0.0
+    assert L.sats_percentile_threshold(None, 10, 0.0, ctypes.byref(t), None, 0, None) == sats.OK and t.value == 0.0
+    assert L.sats_percentile_threshold(None, 10, 1.5, ctypes.byref(t), None, 0, None) == sats.OK
+    assert t.value == float("inf")
