@@ -211,9 +211,10 @@ def run_gpu(args):
     H, N = inputs.LLAMA_H, inputs.LLAMA_N
     stream = torch.cuda.Stream(device=dev)
     w = inputs.mlp_weights(H, N)
+    copies = 1 if args.profile else LAYER_COPIES
     with torch.cuda.stream(stream):
         src = [torch.from_numpy(m.view(np.int16)).to(dev) for m in (w.Wg, w.Wu, w.Wd)]
-        layers = [sats.Layer(*src, stream=stream) for _ in range(LAYER_COPIES)]
+        layers = [sats.Layer(*src, stream=stream) for _ in range(copies)]
         del src
         ws = sats.Workspace(H, N, 1, device=dev, stream=stream)
         # thresholds: Eq. 3 on the post-gate activations of 256 calibration vectors
@@ -233,7 +234,7 @@ def run_gpu(args):
     copy = [0]
 
     def one_call(si, t, ev0=None, ev1=None):
-        layer = layers[copy[0] % LAYER_COPIES]
+        layer = layers[copy[0] % len(layers)]
         copy[0] += 1
         if ev0 is not None:
             ev0.record(stream)
@@ -279,10 +280,17 @@ def run_gpu(args):
     per_call_us = [[1e3 * evs[k][i][0].elapsed_time(evs[k][i][1]) for k in range(K)] for i in range(len(calls))]
     mean_us = [sum(v) / len(v) for v in per_call_us]
 
+    if args.profile:
+        if rank == 0:
+            print(json.dumps({"profile_case": WORKLOAD, "per_call_us": mean_us, "realised": realised}))
+        for l in layers:
+            l.close()
+        return
+
     # dense path on the same copies, for the speedup
     dense_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     for i in range(3 + K):
-        layer = layers[i % LAYER_COPIES]
+        layer = layers[i % len(layers)]
         if i >= 3:
             dense_ev[i - 3][0].record(stream)
         sats.dense_mlp(layer, x, y, ws, stream=stream)
@@ -374,7 +382,11 @@ def main():
     ap.add_argument("--impl", default="sats", choices=["sats", "reference"])
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile", action="store_true",
+                    help="small capture case for ncu: one layer copy, timed calls only, no CPU baseline")
     args = ap.parse_args()
+    if args.profile:
+        args.no_cpu_baseline = True
     if args.impl == "reference":
         run_reference(args)
     else:

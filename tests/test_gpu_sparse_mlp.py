@@ -130,22 +130,29 @@ def test_skipped_rows_are_not_read(sats, oracle):
         sats.sparse_mlp(layer, P.dev_u16(xb), t, y, ws)
         ys.append(y.cpu().numpy())
         layer.close()
+    # chunks are claimed dynamically, so the fp32 grouping of the sum over kept
+    # neurons (and its last bits) may differ between calls; nothing else may
     assert np.all(np.isfinite(ys[1]))
-    assert np.array_equal(ys[0], ys[1])
+    np.testing.assert_allclose(ys[1], ys[0], rtol=1e-5, atol=1e-6)
 
 
-def test_repeat_calls_are_deterministic(sats):
+def test_repeat_calls_agree(sats):
     H, N, B = 512, 1408, 3
     w = inputs.mlp_weights(H, N)
     xb = P.dev_u16(inputs.activations_bf16(B, H))
     layer = sats.Layer(P.dev_u16(w.Wg), P.dev_u16(w.Wu), P.dev_u16(w.Wd))
     ws = sats.Workspace(H, N, B)
-    outs = []
+    outs, lists = [], []
     for _ in range(3):
         y = torch.empty(B, H, dtype=torch.float32, device="cuda")
-        sats.sparse_mlp(layer, xb, 0.2, y, ws)
+        idx = torch.full((B, N), -1, dtype=torch.int32, device="cuda")
+        cnt = torch.empty(B, dtype=torch.int32, device="cuda")
+        sats.sparse_mlp(layer, xb, 0.2, y, ws, idx, cnt)
         outs.append(y.cpu().numpy())
-    assert np.array_equal(outs[0], outs[1]) and np.array_equal(outs[1], outs[2])
+        lists.append(P.keep_from_lists(idx, cnt, N))
+    for i in (1, 2):
+        assert np.array_equal(lists[0], lists[i])          # the kept sets are exactly reproducible
+        np.testing.assert_allclose(outs[i], outs[0], rtol=1e-5, atol=1e-6)
 
 
 def test_argument_errors(sats):
