@@ -50,7 +50,7 @@ static sats_status run_layer(const sats_layer *layer, int x_mode, const void *x,
     const int H = layer->H, N = layer->N;
     const WsLayout L = ws_layout(H, N, B);
     char *base = static_cast<char *>(ws);
-    const int per_pass = H > 4096 ? 2 : kMaxTokensPerPass;
+    const int per_pass = fused_tokens_per_pass(H);
     const size_t x_elem = (x_mode == kXBf16) ? 2 : 4;
     for (int b0 = 0; b0 < B; b0 += per_pass) {
         FusedParams p{};

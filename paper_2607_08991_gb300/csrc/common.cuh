@@ -130,6 +130,97 @@ __device__ __forceinline__ void unpack8(const uint4 &v, float (&f)[8])
     f[6] = bf16_lo(v.w); f[7] = bf16_hi(v.w);
 }
 
+// Packed pair of floats in one 64-bit register (low half = even element), the
+// operand type of the sm_100-family paired FP32 instructions.
+typedef unsigned long long f32x2;
+
+__device__ __forceinline__ f32x2 pack2(float lo, float hi)
+{
+    f32x2 r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+__device__ __forceinline__ float2 unpack2(f32x2 v)
+{
+    float lo, hi;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+    return make_float2(lo, hi);
+}
+
+// d = a * b + c on both halves, each rounded once (fma.rn per element).
+__device__ __forceinline__ f32x2 ffma2(f32x2 a, f32x2 b, f32x2 c)
+{
+    f32x2 d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+
+// One 32-bit word holding two bf16 (element 2i low) -> their exact float pair.
+__device__ __forceinline__ f32x2 bf16x2_to_f32x2(uint32_t w)
+{
+    return pack2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+}
+
+// acc += w[0..7] * x[0..7] on pairs (w: 8 bf16 in a uint4, x: 4 float pairs).
+__device__ __forceinline__ f32x2 dot8_acc(const uint4 &w, const f32x2 (&x)[4], f32x2 acc)
+{
+    acc = ffma2(bf16x2_to_f32x2(w.x), x[0], acc);
+    acc = ffma2(bf16x2_to_f32x2(w.y), x[1], acc);
+    acc = ffma2(bf16x2_to_f32x2(w.z), x[2], acc);
+    acc = ffma2(bf16x2_to_f32x2(w.w), x[3], acc);
+    return acc;
+}
+
+// y[0..7] += h * w[0..7] on pairs.
+__device__ __forceinline__ void axpy8(const uint4 &w, f32x2 hh, f32x2 (&y)[4])
+{
+    y[0] = ffma2(bf16x2_to_f32x2(w.x), hh, y[0]);
+    y[1] = ffma2(bf16x2_to_f32x2(w.y), hh, y[1]);
+    y[2] = ffma2(bf16x2_to_f32x2(w.z), hh, y[2]);
+    y[3] = ffma2(bf16x2_to_f32x2(w.w), hh, y[3]);
+}
+
+__device__ __forceinline__ float hsum2(f32x2 v)
+{
+    const float2 f = unpack2(v);
+    return f.x + f.y;
+}
+
+// Sums four per-lane values p[0..3] over the warp with 6 shuffles: on return,
+// lane L holds the warp total of p[(L >> 3) & 3] (lanes 0, 8, 16, 24 hold
+// rows 0, 1, 2, 3).
+__device__ __forceinline__ float warp_sum4_transposed(float p0, float p1, float p2, float p3, int lane)
+{
+    const bool up = (lane & 16) != 0;
+    float a0 = up ? p2 : p0, a1 = up ? p3 : p1;
+    const float s0 = up ? p0 : p2, s1 = up ? p1 : p3;
+    a0 += __shfl_xor_sync(0xffffffffu, s0, 16);
+    a1 += __shfl_xor_sync(0xffffffffu, s1, 16);
+    const bool b3 = (lane & 8) != 0;
+    float b = b3 ? a1 : a0;
+    const float s = b3 ? a0 : a1;
+    b += __shfl_xor_sync(0xffffffffu, s, 8);
+    b += __shfl_xor_sync(0xffffffffu, b, 4);
+    b += __shfl_xor_sync(0xffffffffu, b, 2);
+    b += __shfl_xor_sync(0xffffffffu, b, 1);
+    return b;
+}
+
+// Same for two values: lanes 0-15 hold the total of p0, lanes 16-31 of p1.
+__device__ __forceinline__ float warp_sum2_transposed(float p0, float p1, int lane)
+{
+    const bool up = (lane & 16) != 0;
+    float a = up ? p1 : p0;
+    const float s = up ? p0 : p1;
+    a += __shfl_xor_sync(0xffffffffu, s, 16);
+    a += __shfl_xor_sync(0xffffffffu, a, 8);
+    a += __shfl_xor_sync(0xffffffffu, a, 4);
+    a += __shfl_xor_sync(0xffffffffu, a, 2);
+    a += __shfl_xor_sync(0xffffffffu, a, 1);
+    return a;
+}
+
 __device__ __forceinline__ float warp_sum(float v)
 {
 #pragma unroll

@@ -1,7 +1,7 @@
 // fused_mlp.cu -- the CATS-thresholded gated MLP (Sec. 2, Eqs. 1-5 of
 // arXiv 2607.08991) as one persistent, warp-specialised kernel for sm_103a.
 //
-// Per call, for nb <= 4 tokens with per-token threshold t_b:
+// Per call, for nb tokens with per-token threshold t_b:
 //   a_j = SiLU(x . W_gate[:, j]);  keep_bj = |a_bj| >= t_b
 //   y_b = sum_j keep_bj * a_bj * (x_b . W_up[:, j]) * W_down[j, :]
 //
@@ -10,24 +10,30 @@
 // contiguous bytes.  A neuron no token keeps costs no HBM traffic beyond its
 // gate row.
 //
-// One CTA per SM (288 threads, ~205 KB shared memory):
-//   * producer warp, one thread: claims chunks of 16 neurons from a global
-//     counter and streams, through a ring of 6 x 32 KB shared-memory stages,
-//     first the chunk's gate rows, then -- once the consumers have published
-//     which neurons of the previous chunk are kept -- that chunk's W_ud rows.
-//     Every copy is one cp.async.bulk that completes on the stage's mbarrier.
-//   * 8 consumer warps: thread t owns 16-byte vectors t, t + 256, ... of every
-//     row, holds the matching x values and y accumulators in registers, forms
-//     dot-product partials, reduces them per warp and across warps through
-//     shared memory, applies SiLU and the mask, compacts the kept neurons with
-//     warp ballots, and accumulates h_j * W_down[j, :] into its y registers.
-//   * after the stream: each CTA writes its y partial, a bounded grid barrier,
-//     then every CTA reduces a slice of y across the partials in a fixed order
-//     (deterministic), and the per-chunk index lists are compacted into the
-//     ascending per-token active-index list.
+// One CTA per SM (544 threads, ~210 KB shared memory):
+//   * producer warp: claims chunks of 8 neurons from a global counter and
+//     streams them through a ring of 6 x 32 KB shared-memory stages with
+//     cp.async.bulk copies that complete on per-stage mbarriers.  Stream
+//     order: gate rows of chunks c0 .. cD (D = gate lookahead), then W_ud rows
+//     of the kept neurons of c0, gate rows of c(D+1), W_ud rows of c1, ...
+//     Once the consumers' gate partials of a chunk are in, the producer warp
+//     forms its kept list itself (lane = row: SiLU, mask, ballots) and issues
+//     the W_ud rows; the D chunks of gate rows in between keep the ring full
+//     meanwhile.
+//   * 16 consumer warps: thread t owns the 16-byte vectors t, t + 512 of
+//     every row, keeps the matching activations and its y accumulators in
+//     registers as float pairs, and computes with paired FP32 FMAs
+//     (fma.rn.f32x2).  Gate rows are reduced four at a time with a transposed
+//     warp reduction, then across warps through shared memory, and each warp
+//     arrives on the chunk's barrier without waiting.  For a W_ud stage
+//     the up dot products are reduced across warps through a split barrier:
+//     each warp arrives, performs the down projection of the previous W_ud
+//     stage (h_j * W_down[j, :] into its y columns), then waits.
+//   * after the stream: each CTA writes its y partial; a bounded grid barrier;
+//     every CTA sums a slice of y over the partials in a fixed order; the
+//     per-chunk index lists are compacted into the ascending per-token list.
 // Every wait is bounded in time; a wait that gives up sets the status word.
 #include <cmath>
-#include <cstdio>
 
 #include "common.cuh"
 #include "internal.h"
@@ -35,34 +41,35 @@
 namespace sats {
 namespace {
 
-constexpr int kConsumerWarps = 8;
-constexpr int kConsumers = kConsumerWarps * 32;   // 256
+constexpr int kConsumerWarps = 16;
+constexpr int kConsumers = kConsumerWarps * 32;   // 512
 constexpr int kThreads = kConsumers + 32;         // + producer warp
 constexpr int kStageBytes = 32768;
 constexpr int kStages = 6;
+constexpr int kMaxLook = 4;                       // gate lookahead, chunks
+constexpr int kBufs = kMaxLook + 1;
+constexpr int kMaxRowsPerStage = 16;
 
 enum StageKind { kGate = 0, kUpDown = 1, kEnd = 2 };
 
 template <int BT>
 struct StageDesc {
     int kind, nrows, chunk_pos, last, buf, chunk, pad0, pad1;
-    int neuron[kChunk];
-    float am[kChunk][BT];   // keep ? a : 0, per row and token
+    int neuron[kMaxRowsPerStage];
+    float am[kMaxRowsPerStage][BT];   // keep ? a : 0, per row and token
 };
 
 template <int BT>
 struct Shared {
     uint64_t full[kStages];
     uint64_t empty[kStages];
-    uint64_t listready[2];
-    uint64_t csync;                                  // consumer-wide barrier
+    uint64_t csync;                                     // consumer-wide barrier (prologue, W_ud stages)
+    uint64_t gsync[kBufs];                              // per chunk buffer: gate partials written
     StageDesc<BT> desc[kStages];
-    float gpart[2][kChunk][BT][kConsumerWarps];      // gate partials per chunk buffer
-    float upart[2][kChunk][BT][kConsumerWarps];      // up partials per UD stage parity
-    int ulist[2][kChunk];                            // kept-by-any-token rows of a chunk
-    float uam[2][kChunk][BT];
-    int ucnt[2];
-    int issued[kStages];                             // producer: parity+1 of last fill
+    float gpart[kBufs][kChunk][BT][kConsumerWarps];     // gate partials per chunk buffer
+    float upart[3][kMaxRowsPerStage][BT][kConsumerWarps];   // by W_ud stage, mod 3
+    int bufchunk[kBufs];
+    int issued[kStages];                                // producer: parity+1 of last fill
     float thr[BT];
     float red[kConsumerWarps][BT];
     int warp_sums[kThreads / 32];
@@ -74,106 +81,178 @@ constexpr size_t smem_bytes() { return (size_t)kStages * kStageBytes + sizeof(Sh
 
 __device__ __forceinline__ void flag_status(int *ctl, int bits) { atomicOr(ctl + kCtlStatus, bits); }
 
-// Consumer-wide barrier on an mbarrier (one arrival per consumer warp), bounded in time.
+// Consumer-wide barrier on an mbarrier (one arrival per consumer warp), bounded
+// in time; arrive() and wait() may be separated by independent work.
 struct ConsumerSync {
     uint64_t *bar;
     uint32_t parity;
-    __device__ bool operator()(int lane, volatile int *abort)
+    __device__ void arrive(int lane)
     {
         __syncwarp();
         if (lane == 0) mbar_arrive(bar);
+    }
+    __device__ bool wait(volatile int *abort)
+    {
         const bool ok = mbar_wait(bar, parity, abort);
         parity ^= 1u;
         return ok;
     }
+    __device__ bool operator()(int lane, volatile int *abort)
+    {
+        arrive(lane);
+        return wait(abort);
+    }
 };
 
 // ------------------------------------------------------------------ producer
+// The kept list of one chunk, formed by the producer warp (lane r = row r):
+// sums the consumers' gate partials across warps, applies SiLU (Eq. 2) and the
+// CATS mask (Eqs. 4-5) per token, writes the optional index outputs, and
+// returns the union of the rows kept by any token (a ballot mask) together
+// with each lane's a values and keep bits.
 template <int BT>
-__device__ void producer(const FusedParams &p, Shared<BT> &S, uint8_t *stages)
+__device__ uint32_t chunk_keep(const FusedParams &p, Shared<BT> &S, int buf, int chunk, int lane, float (&a)[BT],
+                               uint32_t (&bal)[BT])
+{
+    const int n0 = chunk * kChunk;
+    const int rows = min(kChunk, p.N - n0);
+    const bool in = lane < rows;
+    uint32_t uni = 0;
+#pragma unroll
+    for (int b = 0; b < BT; ++b) {
+        float g = 0.f;
+        if (in) {
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w) g += S.gpart[buf][lane][b][w];
+        }
+        a[b] = g / (1.0f + expf(-g));                                   // SiLU, Eq. 2
+        const bool keep = in && b < p.nb && fabsf(a[b]) >= S.thr[b];    // Eqs. 4-5
+        bal[b] = __ballot_sync(0xffffffffu, keep);
+        uni |= bal[b];
+    }
+    const uint32_t lt = (1u << lane) - 1u;
+    if (p.active_idx) {
+        const int stride = p.nchunks * kChunk;
+#pragma unroll
+        for (int b = 0; b < BT; ++b) {
+            if (b >= p.nb) break;
+            if ((bal[b] >> lane) & 1u) p.idx_tmp[b * stride + n0 + __popc(bal[b] & lt)] = n0 + lane;
+            if (lane == 0) p.chunk_cnt[chunk * kMaxTokensPerPass + b] = __popc(bal[b]);
+        }
+    }
+    if (p.keep_trace && in) {
+#pragma unroll
+        for (int b = 0; b < BT; ++b)
+            if (b < p.nb) p.keep_trace[(size_t)b * p.N + n0 + lane] = (uint8_t)((bal[b] >> lane) & 1u);
+    }
+    return uni;
+}
+
+// Runs on the whole producer warp with uniform control flow; lane 0 claims
+// chunks and posts gate stages, every lane whose row is kept issues that row's
+// W_ud copy.
+template <int BT>
+__device__ void producer(const FusedParams &p, Shared<BT> &S, uint8_t *stages, int look, int lane)
 {
     const uint64_t pol = l2_policy_evict_first();
     const int H = p.H, N = p.N;
     const uint32_t gate_row_bytes = (uint32_t)H * 2u;
     const uint32_t ud_row_bytes = (uint32_t)H * 4u;
     const int rows_per_gate_stage = min(kChunk, kStageBytes / (int)gate_row_bytes);
-    const int rows_per_ud_stage = min(kChunk, kStageBytes / (int)ud_row_bytes);
+    const int rows_per_ud_stage = min(kMaxRowsPerStage, kStageBytes / (int)ud_row_bytes);
+    const int nbufs = look + 1;
     int *counter = p.ctl + kCtlChunk;
+    const uint32_t lt = (1u << lane) - 1u;
 
     uint32_t stage = 0, phase = 0;
-    uint32_t lr_uses[2] = {0u, 0u};
-    int seq = 0, prev = -1, prev_buf = 0;
-    bool ok = true;
-    int next = atomicAdd(counter, 1);
-
-    auto advance = [&]() {
-        if (++stage == kStages) { stage = 0; phase ^= 1u; }
-    };
+    int seq_gate = 0, seq_ud = 0;     // chunks whose gate / W_ud rows have been issued
+    bool more = true, ok = true;
+    int next = 0;
+    if (lane == 0) next = atomicAdd(counter, 1);
+    next = __shfl_sync(0xffffffffu, next, 0);
 
     for (;;) {
-        const int c = next;
-        const bool have = c < p.nchunks;
-        const int buf = seq & 1;
-        if (have) {
-            next = atomicAdd(counter, 1);
+        // gate rows, up to `look` chunks ahead of the W_ud rows
+        while (ok && more && seq_gate - seq_ud <= look) {
+            const int c = next;
+            if (c >= p.nchunks) { more = false; break; }
+            if (lane == 0) next = atomicAdd(counter, 1);
+            next = __shfl_sync(0xffffffffu, next, 0);
+            const int buf = seq_gate % nbufs;
             const int n0 = c * kChunk;
             const int rows = min(kChunk, N - n0);
             for (int r0 = 0; r0 < rows; r0 += rows_per_gate_stage) {
                 const int nr = min(rows_per_gate_stage, rows - r0);
                 if (!mbar_wait(&S.empty[stage], phase ^ 1u, &S.abort)) { ok = false; break; }
-                StageDesc<BT> &d = S.desc[stage];
-                d.kind = kGate;
-                d.nrows = nr;
-                d.chunk_pos = r0;
-                d.last = (r0 + nr >= rows) ? 1 : 0;
-                d.buf = buf;
-                d.chunk = c;
-                S.issued[stage] = (int)phase + 1;
-                mbar_arrive_expect_tx(&S.full[stage], (uint32_t)nr * gate_row_bytes);
-                bulk_load(stages + (size_t)stage * kStageBytes, p.wg_t + (size_t)(n0 + r0) * H,
-                          (uint32_t)nr * gate_row_bytes, &S.full[stage], pol);
-                advance();
+                if (lane == 0) {
+                    StageDesc<BT> &d = S.desc[stage];
+                    d.kind = kGate;
+                    d.nrows = nr;
+                    d.chunk_pos = r0;
+                    d.last = (r0 + nr >= rows) ? 1 : 0;
+                    d.buf = buf;
+                    d.chunk = c;
+                    S.issued[stage] = (int)phase + 1;
+                    mbar_arrive_expect_tx(&S.full[stage], (uint32_t)nr * gate_row_bytes);
+                    bulk_load(stages + (size_t)stage * kStageBytes, p.wg_t + (size_t)(n0 + r0) * H,
+                              (uint32_t)nr * gate_row_bytes, &S.full[stage], pol);
+                }
+                __syncwarp();
+                if (++stage == kStages) { stage = 0; phase ^= 1u; }
             }
-            if (!ok) break;
+            if (lane == 0) S.bufchunk[buf] = c;
+            ++seq_gate;
         }
-        if (prev >= 0) {
-            if (!mbar_wait(&S.listready[prev_buf], lr_uses[prev_buf] & 1u, &S.abort)) { ok = false; break; }
-            ++lr_uses[prev_buf];
-            const int cnt = S.ucnt[prev_buf];
-            const int n0 = prev * kChunk;
-            for (int k0 = 0; k0 < cnt; k0 += rows_per_ud_stage) {
-                const int nr = min(rows_per_ud_stage, cnt - k0);
-                if (!mbar_wait(&S.empty[stage], phase ^ 1u, &S.abort)) { ok = false; break; }
-                StageDesc<BT> &d = S.desc[stage];
+        if (!ok || seq_ud == seq_gate) break;
+        // kept list of the oldest chunk whose gate rows were issued, then its W_ud rows
+        const int buf = seq_ud % nbufs;
+        if (!mbar_wait(&S.gsync[buf], (uint32_t)(seq_ud / nbufs) & 1u, &S.abort)) { ok = false; break; }
+        __syncwarp();
+        const int chunk = S.bufchunk[buf];
+        float a[BT];
+        uint32_t bal[BT];
+        const uint32_t uni = chunk_keep<BT>(p, S, buf, chunk, lane, a, bal);
+        const int cnt = __popc(uni);
+        const int pos = __popc(uni & lt);
+        const bool mine = (uni >> lane) & 1u;
+        const int nid = chunk * kChunk + lane;
+        for (int k0 = 0; k0 < cnt; k0 += rows_per_ud_stage) {
+            const int nr = min(rows_per_ud_stage, cnt - k0);
+            if (!mbar_wait(&S.empty[stage], phase ^ 1u, &S.abort)) { ok = false; break; }
+            StageDesc<BT> &d = S.desc[stage];
+            const bool in_stage = mine && pos >= k0 && pos < k0 + nr;
+            if (in_stage) {
+                const int k = pos - k0;
+                d.neuron[k] = nid;
+#pragma unroll
+                for (int b = 0; b < BT; ++b) d.am[k][b] = ((bal[b] >> lane) & 1u) ? a[b] : 0.f;
+            }
+            __syncwarp();     // descriptor entries written before lane 0's release below
+            if (lane == 0) {
                 d.kind = kUpDown;
                 d.nrows = nr;
-                for (int k = 0; k < nr; ++k) {
-                    d.neuron[k] = n0 + S.ulist[prev_buf][k0 + k];
-#pragma unroll
-                    for (int b = 0; b < BT; ++b) d.am[k][b] = S.uam[prev_buf][k0 + k][b];
-                }
                 S.issued[stage] = (int)phase + 1;
                 mbar_arrive_expect_tx(&S.full[stage], (uint32_t)nr * ud_row_bytes);
-                uint8_t *dst = stages + (size_t)stage * kStageBytes;
-                for (int k = 0; k < nr; ++k)
-                    bulk_load(dst + (size_t)k * ud_row_bytes, p.w_ud + (size_t)d.neuron[k] * 2 * H, ud_row_bytes,
-                              &S.full[stage], pol);
-                advance();
             }
-            if (!ok) break;
+            __syncwarp();
+            if (in_stage)
+                bulk_load(stages + (size_t)stage * kStageBytes + (size_t)(pos - k0) * ud_row_bytes,
+                          p.w_ud + (size_t)nid * 2 * H, ud_row_bytes, &S.full[stage], pol);
+            __syncwarp();
+            if (++stage == kStages) { stage = 0; phase ^= 1u; }
         }
-        if (!have) break;
-        prev = c;
-        prev_buf = buf;
-        ++seq;
+        ++seq_ud;
     }
     if (ok && mbar_wait(&S.empty[stage], phase ^ 1u, &S.abort)) {
-        S.desc[stage].kind = kEnd;
-        mbar_arrive(&S.full[stage]);
-    } else {
+        if (lane == 0) {
+            S.desc[stage].kind = kEnd;
+            mbar_arrive(&S.full[stage]);
+        }
+    } else if (lane == 0) {
         S.abort = 1;
         flag_status(p.ctl, kStatusTimeout);
     }
+    __syncwarp();
 }
 
 // Bounded wait for every bulk copy still in flight (only on the error path).
@@ -187,63 +266,11 @@ __device__ void drain_copies(Shared<BT> &S)
 
 // ------------------------------------------------------------------ consumers
 template <int BT, int VPT>
-__device__ void chunk_lists(const FusedParams &p, Shared<BT> &S, int buf, int chunk, int lane)
+__device__ void load_activations(const FusedParams &p, Shared<BT> &S, ConsumerSync &csync, int tid,
+                                 f32x2 (&xp)[BT][VPT][4], bool &ok)
 {
-    const int n0 = chunk * kChunk;
-    const int rows = min(kChunk, p.N - n0);
-    const int r = lane;
-    const bool in = r < rows;
-    float a[BT];
-    uint32_t bal[BT];
-    uint32_t uni = 0;
-#pragma unroll
-    for (int b = 0; b < BT; ++b) {
-        float g = 0.f;
-        if (in) {
-#pragma unroll
-            for (int w = 0; w < kConsumerWarps; ++w) g += S.gpart[buf][r][b][w];
-        }
-        a[b] = g / (1.0f + expf(-g));                 // SiLU, Eq. 2
-        const bool keep = in && b < p.nb && fabsf(a[b]) >= S.thr[b];   // Eqs. 4-5
-        bal[b] = __ballot_sync(0xffffffffu, keep);
-        uni |= bal[b];
-    }
-    const uint32_t lt = (1u << lane) - 1u;
-    if ((uni >> lane) & 1u) {
-        const int pos = __popc(uni & lt);
-        S.ulist[buf][pos] = r;
-#pragma unroll
-        for (int b = 0; b < BT; ++b) S.uam[buf][pos][b] = ((bal[b] >> lane) & 1u) ? a[b] : 0.f;
-    }
-    if (lane == 0) S.ucnt[buf] = __popc(uni);
-    if (p.active_idx) {
-        const int stride = p.nchunks * kChunk;
-#pragma unroll
-        for (int b = 0; b < BT; ++b) {
-            if (b >= p.nb) break;
-            if ((bal[b] >> lane) & 1u) p.idx_tmp[b * stride + n0 + __popc(bal[b] & lt)] = n0 + r;
-            if (lane == 0) p.chunk_cnt[chunk * kMaxTokensPerPass + b] = __popc(bal[b]);
-        }
-    }
-    if (p.keep_trace && in) {
-#pragma unroll
-        for (int b = 0; b < BT; ++b)
-            if (b < p.nb) p.keep_trace[(size_t)b * p.N + n0 + r] = (uint8_t)((bal[b] >> lane) & 1u);
-    }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&S.listready[buf]);
-}
-
-template <int BT, int VPT>
-__device__ void consumer(const FusedParams &p, Shared<BT> &S, const uint8_t *stages, float (&yv)[BT][VPT][8])
-{
-    const int tid = threadIdx.x;
-    const int warp = tid >> 5, lane = tid & 31;
+    const int lane = tid & 31, warp = tid >> 5;
     const int H = p.H, HV = H >> 3;
-    const size_t gate_row_bytes = (size_t)H * 2, ud_row_bytes = (size_t)H * 4;
-    ConsumerSync csync{&S.csync, 0u};
-
-    // ---- activations of this pass, in registers
     float xv[BT][VPT][8];
 #pragma unroll
     for (int b = 0; b < BT; ++b)
@@ -251,7 +278,7 @@ __device__ void consumer(const FusedParams &p, Shared<BT> &S, const uint8_t *sta
         for (int i = 0; i < VPT; ++i) {
             const int v = tid + i * kConsumers;
 #pragma unroll
-            for (int e = 0; e < 8; ++e) { xv[b][i][e] = 0.f; yv[b][i][e] = 0.f; }
+            for (int e = 0; e < 8; ++e) xv[b][i][e] = 0.f;
             if (v < HV && b < p.nb) {
                 if (p.x_mode == kXBf16) {
                     const uint4 w = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(p.x) + (size_t)b * H)[v];
@@ -280,7 +307,7 @@ __device__ void consumer(const FusedParams &p, Shared<BT> &S, const uint8_t *sta
 #pragma unroll
             for (int b = 0; b < BT; ++b) S.red[warp][b] = ss[b];
         }
-        if (!csync(lane, &S.abort)) { S.abort = 1; flag_status(p.ctl, kStatusTimeout); return; }
+        if (!csync(lane, &S.abort)) { ok = false; return; }
 #pragma unroll
         for (int b = 0; b < BT; ++b) {
             float tot = 0.f;
@@ -299,9 +326,76 @@ __device__ void consumer(const FusedParams &p, Shared<BT> &S, const uint8_t *sta
             }
         }
     }
+#pragma unroll
+    for (int b = 0; b < BT; ++b)
+#pragma unroll
+        for (int i = 0; i < VPT; ++i)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) xp[b][i][e] = pack2(xv[b][i][2 * e], xv[b][i][2 * e + 1]);
+}
+
+// Down projection of one W_ud stage: y[cols] += h_j * W_down[j, cols] for the
+// stage's rows, with h_j = am_j * u_j and u_j the cross-warp sum of the stage's
+// up partials.  Then releases the stage to the producer.
+template <int BT, int VPT>
+__device__ __forceinline__ void down_stage(const FusedParams &p, Shared<BT> &S, const uint8_t *sbase,
+                                           const StageDesc<BT> &d, int nr, int ub, uint32_t stage, int tid, int lane,
+                                           f32x2 (&yp)[BT][VPT][4])
+{
+    const int H = p.H, HV = H >> 3;
+    const size_t ud_row_bytes = (size_t)H * 4;
+    for (int k = 0; k < nr; ++k) {
+        f32x2 hh[BT];
+#pragma unroll
+        for (int b = 0; b < BT; ++b) {
+            float u = S.upart[ub][k][b][lane & (kConsumerWarps - 1)];
+#pragma unroll
+            for (int o = kConsumerWarps / 2; o > 0; o >>= 1) u += __shfl_xor_sync(0xffffffffu, u, o);
+            const float h = d.am[k][b] * u;     // CATS_t(a) * (x W_up), Eqs. 1 and 5
+            hh[b] = pack2(h, h);
+        }
+        const uint4 *down = reinterpret_cast<const uint4 *>(sbase + (size_t)k * ud_row_bytes + (size_t)H * 2);
+#pragma unroll
+        for (int i = 0; i < VPT; ++i) {
+            const int v = tid + i * kConsumers;
+            if (v < HV) {
+                const uint4 w = down[v];
+#pragma unroll
+                for (int b = 0; b < BT; ++b) axpy8(w, hh[b], yp[b][i]);
+            }
+        }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&S.empty[stage]);
+}
+
+template <int BT, int VPT>
+__device__ void consumer(const FusedParams &p, Shared<BT> &S, const uint8_t *stages, f32x2 (&yp)[BT][VPT][4])
+{
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    const int H = p.H, HV = H >> 3;
+    const size_t gate_row_bytes = (size_t)H * 2, ud_row_bytes = (size_t)H * 4;
+    ConsumerSync csync{&S.csync, 0u};
+    const uint4 zero4 = make_uint4(0u, 0u, 0u, 0u);
+
+#pragma unroll
+    for (int b = 0; b < BT; ++b)
+#pragma unroll
+        for (int i = 0; i < VPT; ++i)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) yp[b][i][e] = 0ull;
+
+    f32x2 xp[BT][VPT][4];
+    bool ok = true;
+    load_activations<BT, VPT>(p, S, csync, tid, xp, ok);
+    if (!ok) { S.abort = 1; flag_status(p.ctl, kStatusTimeout); return; }
 
     uint32_t stage = 0, phase = 0;
     int ud_seq = 0;
+    // a W_ud stage whose up sums are complete but whose down projection is
+    // still to do (it is done while waiting on the next W_ud stage's barrier)
+    int pend_stage = -1, pend_nr = 0, pend_ub = 0;
     for (;;) {
         if (!mbar_wait(&S.full[stage], phase, &S.abort)) {
             S.abort = 1;
@@ -310,96 +404,92 @@ __device__ void consumer(const FusedParams &p, Shared<BT> &S, const uint8_t *sta
         }
         const StageDesc<BT> &d = S.desc[stage];
         const int kind = d.kind;
+        if (kind != kUpDown && pend_stage >= 0) {
+            down_stage<BT, VPT>(p, S, stages + (size_t)pend_stage * kStageBytes, S.desc[pend_stage], pend_nr,
+                                pend_ub, (uint32_t)pend_stage, tid, lane, yp);
+            pend_stage = -1;
+        }
         if (kind == kEnd) break;
         const uint8_t *sbase = stages + (size_t)stage * kStageBytes;
         const int nr = d.nrows;
         if (kind == kGate) {
-            const int r0 = d.chunk_pos, buf = d.buf, last = d.last, chunk = d.chunk;
-#pragma unroll 4
-            for (int r = 0; r < nr; ++r) {
-                const uint4 *row = reinterpret_cast<const uint4 *>(sbase + (size_t)r * gate_row_bytes);
-                float acc[BT];
+            const int r0 = d.chunk_pos, buf = d.buf, last = d.last;
+            for (int q = 0; q < nr; q += 4) {
+                // four rows at once: independent FMA chains, one transposed reduction
+                f32x2 acc[4][BT];
 #pragma unroll
-                for (int b = 0; b < BT; ++b) acc[b] = 0.f;
+                for (int r = 0; r < 4; ++r)
 #pragma unroll
-                for (int i = 0; i < VPT; ++i) {
-                    const int v = tid + i * kConsumers;
-                    if (v < HV) {
-                        float f[8];
-                        unpack8(row[v], f);
-#pragma unroll
-                        for (int b = 0; b < BT; ++b)
-#pragma unroll
-                            for (int e = 0; e < 8; ++e) acc[b] = fmaf(f[e], xv[b][i][e], acc[b]);
-                    }
-                }
-#pragma unroll
-                for (int b = 0; b < BT; ++b) acc[b] = warp_sum(acc[b]);
-                if (lane == 0) {
-#pragma unroll
-                    for (int b = 0; b < BT; ++b) S.gpart[buf][r0 + r][b][warp] = acc[b];
-                }
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&S.empty[stage]);
-            if (last) {
-                if (!csync(lane, &S.abort)) { S.abort = 1; flag_status(p.ctl, kStatusTimeout); return; }
-                if (warp == 0) chunk_lists<BT, VPT>(p, S, buf, chunk, lane);
-            }
-        } else {
-            const int ub = ud_seq & 1;
-#pragma unroll 2
-            for (int k = 0; k < nr; ++k) {
-                const uint4 *up = reinterpret_cast<const uint4 *>(sbase + (size_t)k * ud_row_bytes);
-                float acc[BT];
-#pragma unroll
-                for (int b = 0; b < BT; ++b) acc[b] = 0.f;
+                    for (int b = 0; b < BT; ++b) acc[r][b] = 0ull;
 #pragma unroll
                 for (int i = 0; i < VPT; ++i) {
                     const int v = tid + i * kConsumers;
                     if (v < HV) {
-                        float f[8];
-                        unpack8(up[v], f);
+                        uint4 w[4];
 #pragma unroll
-                        for (int b = 0; b < BT; ++b)
+                        for (int r = 0; r < 4; ++r)
+                            w[r] = (q + r < nr)
+                                       ? reinterpret_cast<const uint4 *>(sbase + (size_t)(q + r) * gate_row_bytes)[v]
+                                       : zero4;
 #pragma unroll
-                            for (int e = 0; e < 8; ++e) acc[b] = fmaf(f[e], xv[b][i][e], acc[b]);
+                        for (int r = 0; r < 4; ++r)
+#pragma unroll
+                            for (int b = 0; b < BT; ++b) acc[r][b] = dot8_acc(w[r], xp[b][i], acc[r][b]);
                     }
                 }
-#pragma unroll
-                for (int b = 0; b < BT; ++b) acc[b] = warp_sum(acc[b]);
-                if (lane == 0) {
-#pragma unroll
-                    for (int b = 0; b < BT; ++b) S.upart[ub][k][b][warp] = acc[b];
-                }
-            }
-            if (!csync(lane, &S.abort)) { S.abort = 1; flag_status(p.ctl, kStatusTimeout); return; }
-            for (int k = 0; k < nr; ++k) {
-                float h[BT];
 #pragma unroll
                 for (int b = 0; b < BT; ++b) {
-                    float u = S.upart[ub][k][b][lane & (kConsumerWarps - 1)];
-                    u += __shfl_xor_sync(0xffffffffu, u, 4);
-                    u += __shfl_xor_sync(0xffffffffu, u, 2);
-                    u += __shfl_xor_sync(0xffffffffu, u, 1);
-                    h[b] = d.am[k][b] * u;     // CATS_t(a) * (x W_up), Eqs. 1 and 5
+                    const float tot = warp_sum4_transposed(hsum2(acc[0][b]), hsum2(acc[1][b]), hsum2(acc[2][b]),
+                                                           hsum2(acc[3][b]), lane);
+                    const int r = (lane >> 3) & 3;
+                    if ((lane & 7) == 0 && q + r < nr) S.gpart[buf][r0 + q + r][b][warp] = tot;
                 }
-                const uint4 *down = reinterpret_cast<const uint4 *>(sbase + (size_t)k * ud_row_bytes + (size_t)H * 2);
+            }
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(&S.empty[stage]);
+                if (last) mbar_arrive(&S.gsync[buf]);   // this warp's partials of the chunk are written
+            }
+        } else {
+            const int ub = ud_seq % 3;
+            // up dot products, two rows at a time
+            for (int q = 0; q < nr; q += 2) {
+                f32x2 acc[2][BT];
+#pragma unroll
+                for (int r = 0; r < 2; ++r)
+#pragma unroll
+                    for (int b = 0; b < BT; ++b) acc[r][b] = 0ull;
 #pragma unroll
                 for (int i = 0; i < VPT; ++i) {
                     const int v = tid + i * kConsumers;
                     if (v < HV) {
-                        float f[8];
-                        unpack8(down[v], f);
+                        uint4 w[2];
 #pragma unroll
-                        for (int b = 0; b < BT; ++b)
+                        for (int r = 0; r < 2; ++r)
+                            w[r] = (q + r < nr) ? reinterpret_cast<const uint4 *>(sbase + (size_t)(q + r) * ud_row_bytes)[v]
+                                                : zero4;
 #pragma unroll
-                            for (int e = 0; e < 8; ++e) yv[b][i][e] = fmaf(h[b], f[e], yv[b][i][e]);
+                        for (int r = 0; r < 2; ++r)
+#pragma unroll
+                            for (int b = 0; b < BT; ++b) acc[r][b] = dot8_acc(w[r], xp[b][i], acc[r][b]);
                     }
                 }
+#pragma unroll
+                for (int b = 0; b < BT; ++b) {
+                    const float tot = warp_sum2_transposed(hsum2(acc[0][b]), hsum2(acc[1][b]), lane);
+                    const int r = lane >> 4;
+                    if ((lane & 15) == 0 && q + r < nr) S.upart[ub][q + r][b][warp] = tot;
+                }
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&S.empty[stage]);
+            csync.arrive(lane);
+            if (pend_stage >= 0) {
+                down_stage<BT, VPT>(p, S, stages + (size_t)pend_stage * kStageBytes, S.desc[pend_stage], pend_nr,
+                                    pend_ub, (uint32_t)pend_stage, tid, lane, yp);
+            }
+            if (!csync.wait(&S.abort)) { S.abort = 1; flag_status(p.ctl, kStatusTimeout); return; }
+            pend_stage = (int)stage;
+            pend_nr = nr;
+            pend_ub = ub;
             ++ud_seq;
         }
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
@@ -429,7 +519,7 @@ __device__ bool grid_barrier(int *ctl)
                     ok = 0;
                     break;
                 }
-                __nanosleep(64);
+                __nanosleep(32);
             }
         }
         __threadfence();
@@ -439,7 +529,6 @@ __device__ bool grid_barrier(int *ctl)
     return ok_s != 0;
 }
 
-template <int BT>
 __device__ void reduce_partials(const FusedParams &p)
 {
     const int H4 = p.H >> 2;
@@ -504,12 +593,11 @@ __device__ void compact_indices(const FusedParams &p, Shared<BT> &S, int *prefix
             if (p.active_cnt) p.active_cnt[b] = tot;
         }
         __syncthreads();
-        // copy this CTA's chunks (c = blockIdx.x + k * gridDim.x), 16 entries each
+        // copy this CTA's chunks (c = blockIdx.x + k * gridDim.x)
         const int slots = kThreads / kChunk;   // chunks per sweep
         for (int s0 = 0;; s0 += slots) {
-            const int ci = s0 + tid / kChunk;
-            const int c = blockIdx.x + ci * gridDim.x;
             if (blockIdx.x + s0 * gridDim.x >= nc) break;
+            const int c = blockIdx.x + (s0 + tid / kChunk) * gridDim.x;
             const int k = tid % kChunk;
             if (c < nc && tid < slots * kChunk) {
                 const int cnt = __ldcg(p.chunk_cnt + c * kMaxTokensPerPass + b);
@@ -522,7 +610,7 @@ __device__ void compact_indices(const FusedParams &p, Shared<BT> &S, int *prefix
 }
 
 template <int BT, int VPT>
-__global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParams p)
+__global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParams p, int look)
 {
     extern __shared__ __align__(128) uint8_t smem[];
     uint8_t *stages = smem;
@@ -536,8 +624,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
             mbar_init(&S.empty[s], kConsumerWarps);
             S.issued[s] = 0;
         }
-        mbar_init(&S.listready[0], 1);
-        mbar_init(&S.listready[1], 1);
+        for (int b = 0; b < kBufs; ++b) mbar_init(&S.gsync[b], kConsumerWarps);
         mbar_init(&S.csync, kConsumerWarps);
         S.abort = 0;
         mbar_init_fence();
@@ -549,15 +636,13 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
     }
     __syncthreads();
 
-    float yv[BT][VPT][8];
+    f32x2 yp[BT][VPT][4];
     if (warp == kConsumerWarps) {
-        if (lane == 0) {
-            producer<BT>(p, S, stages);
-            if (S.abort) drain_copies<BT>(S);
-        }
+        producer<BT>(p, S, stages, look, lane);
+        if (lane == 0 && S.abort) drain_copies<BT>(S);
         __syncwarp();
     } else {
-        consumer<BT, VPT>(p, S, stages, yv);
+        consumer<BT, VPT>(p, S, stages, yp);
         // y partial of this CTA: partials[blockIdx.x][b][:]
         const int HV = p.H >> 3;
 #pragma unroll
@@ -569,19 +654,21 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
                 if (v < HV) {
                     float4 *dst = reinterpret_cast<float4 *>(
                         p.partials + ((size_t)blockIdx.x * kMaxTokensPerPass + b) * p.H + (size_t)v * 8);
-                    dst[0] = make_float4(yv[b][i][0], yv[b][i][1], yv[b][i][2], yv[b][i][3]);
-                    dst[1] = make_float4(yv[b][i][4], yv[b][i][5], yv[b][i][6], yv[b][i][7]);
+                    const float2 y0 = unpack2(yp[b][i][0]), y1 = unpack2(yp[b][i][1]);
+                    const float2 y2 = unpack2(yp[b][i][2]), y3 = unpack2(yp[b][i][3]);
+                    dst[0] = make_float4(y0.x, y0.y, y1.x, y1.y);
+                    dst[1] = make_float4(y2.x, y2.y, y3.x, y3.y);
                 }
             }
         }
     }
     if (!grid_barrier(p.ctl)) return;
-    reduce_partials<BT>(p);
+    reduce_partials(p);
     if (p.active_idx && !S.abort) compact_indices<BT>(p, S, reinterpret_cast<int *>(stages));
 }
 
 template <int BT, int VPT>
-cudaError_t launch_t(const FusedParams &p, int grid, cudaStream_t stream)
+cudaError_t launch_t(const FusedParams &p, int grid, int look, cudaStream_t stream)
 {
     static unsigned long long configured = 0;   // one bit per device ordinal
     const size_t smem = smem_bytes<BT>();
@@ -604,39 +691,41 @@ cudaError_t launch_t(const FusedParams &p, int grid, cudaStream_t stream)
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, fused_mlp_kernel<BT, VPT>, p);
+    return cudaLaunchKernelEx(&cfg, fused_mlp_kernel<BT, VPT>, p, look);
 }
 
 }  // namespace
 
 int fused_grid(int nchunks)
 {
-    int dev = 0, sms = 0;
+    static int sms_by_dev[64] = {0};
+    int dev = 0;
     cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    int &sms = sms_by_dev[dev & 63];
+    if (sms == 0) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     int g = sms < kMaxGrid ? sms : kMaxGrid;
     if (nchunks < g) g = nchunks;
     return g < 1 ? 1 : g;
 }
 
+// 16-byte vectors per consumer thread and row: ceil(H / 8 / 512).
+static int fused_vectors_per_thread(int H) { return H <= 4096 ? 1 : 2; }
+
+int fused_tokens_per_pass(int H) { return fused_vectors_per_thread(H) == 1 ? 2 : 1; }
+
 cudaError_t launch_fused(const FusedParams &p, cudaStream_t stream)
 {
     const int grid = fused_grid(p.nchunks);
-    // vectors of 8 bf16 per consumer thread and row: VPT = ceil(H / 8 / 256)
-    const int vpt = p.H <= 2048 ? 1 : (p.H <= 4096 ? 2 : 4);
+    // chunks of gate rows kept in flight ahead of the W_ud rows: about 128 KB
+    int look = (128 * 1024) / (kChunk * 2 * p.H);
+    look = look < 1 ? 1 : (look > kMaxLook ? kMaxLook : look);
+    const int vpt = fused_vectors_per_thread(p.H);
+    if (p.nb < 1 || p.nb > fused_tokens_per_pass(p.H)) return cudaErrorInvalidValue;
     if (vpt == 1) {
-        if (p.nb <= 1) return launch_t<1, 1>(p, grid, stream);
-        if (p.nb <= 2) return launch_t<2, 1>(p, grid, stream);
-        return launch_t<4, 1>(p, grid, stream);
+        if (p.nb <= 1) return launch_t<1, 1>(p, grid, look, stream);
+        return launch_t<2, 1>(p, grid, look, stream);
     }
-    if (vpt == 2) {
-        if (p.nb <= 1) return launch_t<1, 2>(p, grid, stream);
-        if (p.nb <= 2) return launch_t<2, 2>(p, grid, stream);
-        return launch_t<4, 2>(p, grid, stream);
-    }
-    if (p.nb <= 1) return launch_t<1, 4>(p, grid, stream);
-    if (p.nb <= 2) return launch_t<2, 4>(p, grid, stream);
-    return cudaErrorInvalidValue;   // callers split H > 4096 into passes of <= 2 tokens
+    return launch_t<1, 2>(p, grid, look, stream);
 }
 
 }  // namespace sats

@@ -17,7 +17,7 @@ struct sats_layer {
 
 namespace sats {
 
-constexpr int kChunk = 16;              // neurons per scheduling unit of the fused kernel
+constexpr int kChunk = 8;               // neurons per scheduling unit of the fused kernel
 constexpr int kMaxTokensPerPass = 4;    // tokens one fused launch carries
 constexpr int kMaxGrid = 256;           // upper bound of the fused grid (partials rows)
 constexpr int kMaxH = 8192;
@@ -65,6 +65,7 @@ struct FusedParams {
 
 // Number of CTAs the fused kernel runs with on `device` (all co-resident).
 int fused_grid(int nchunks);
+int fused_tokens_per_pass(int H);
 cudaError_t launch_fused(const FusedParams &p, cudaStream_t stream);
 
 cudaError_t launch_pack(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd, int H, int N,
