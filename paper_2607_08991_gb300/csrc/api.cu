@@ -23,8 +23,8 @@ WsLayout ws_layout(int H, int N, int B)
     off += align256(kCtlInts * sizeof(int));
     L.partials = off;
     off += align256((size_t)kMaxGrid * kMaxTokensPerPass * H * sizeof(float));
-    L.chunk_cnt = off;
-    off += align256(nc * kMaxTokensPerPass * sizeof(int));
+    L.chunk_cnt = off;   // per-CTA kept counts
+    off += align256((size_t)kMaxGrid * kMaxTokensPerPass * sizeof(int));
     L.idx_tmp = off;
     off += align256((size_t)kMaxTokensPerPass * nc * kChunk * sizeof(int));
     L.route_perm = off;
@@ -71,7 +71,7 @@ static sats_status run_layer(const sats_layer *layer, int x_mode, const void *x,
         p.ctl = reinterpret_cast<int *>(base + L.ctl);
         p.partials = reinterpret_cast<float *>(base + L.partials);
         p.chunk_cnt = reinterpret_cast<int *>(base + L.chunk_cnt);
-        p.idx_tmp = reinterpret_cast<int *>(base + L.idx_tmp);
+        p.keep_tmp = reinterpret_cast<uint8_t *>(base + L.idx_tmp);
         p.active_idx = active_idx ? active_idx + (size_t)b0 * N : nullptr;
         p.active_cnt = active_cnt ? active_cnt + b0 : nullptr;
         p.keep_trace = keep_trace ? keep_trace + (size_t)b0 * N : nullptr;

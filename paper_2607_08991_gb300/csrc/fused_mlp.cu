@@ -10,28 +10,35 @@
 // contiguous bytes.  A neuron no token keeps costs no HBM traffic beyond its
 // gate row.
 //
-// One CTA per SM (544 threads, ~210 KB shared memory):
-//   * producer warp: claims chunks of 8 neurons from a global counter and
-//     streams them through a ring of 6 x 32 KB shared-memory stages with
-//     cp.async.bulk copies that complete on per-stage mbarriers.  Stream
-//     order: gate rows of chunks c0 .. cD (D = gate lookahead), then W_ud rows
-//     of the kept neurons of c0, gate rows of c(D+1), W_ud rows of c1, ...
-//     Once the consumers' gate partials of a chunk are in, the producer warp
-//     forms its kept list itself (lane = row: SiLU, mask, ballots) and issues
-//     the W_ud rows; the D chunks of gate rows in between keep the ring full
-//     meanwhile.
-//   * 16 consumer warps: thread t owns the 16-byte vectors t, t + 512 of
-//     every row, keeps the matching activations and its y accumulators in
-//     registers as float pairs, and computes with paired FP32 FMAs
-//     (fma.rn.f32x2).  Gate rows are reduced four at a time with a transposed
-//     warp reduction, then across warps through shared memory, and each warp
-//     arrives on the chunk's barrier without waiting.  For a W_ud stage
-//     the up dot products are reduced across warps through a split barrier:
-//     each warp arrives, performs the down projection of the previous W_ud
-//     stage (h_j * W_down[j, :] into its y columns), then waits.
-//   * after the stream: each CTA writes its y partial; a bounded grid barrier;
-//     every CTA sums a slice of y over the partials in a fixed order; the
-//     per-chunk index lists are compacted into the ascending per-token list.
+// One CTA per SM, 576 threads in four roles, two shared-memory rings fed by
+// cp.async.bulk copies that complete on per-stage mbarriers:
+//   * gate producer (one thread): walks the first part of the CTA's contiguous
+//     range of N / G neurons in chunks of 8, then claims chunks from a shared
+//     pool (the last few chunks of every CTA's range) until it is empty, so
+//     that faster SMs take more of the tail; a chunk is started only when one
+//     of four list buffers is free.  Streams gate rows into the gate ring
+//     (5 x 16 KB).
+//   * 8 gate warps: thread t owns the 16-byte vectors t, t + 256, ... of every
+//     gate row and keeps the matching activations in registers as float pairs;
+//     dot products use paired FP32 FMAs (fma.rn.f32x2), two rows at a time
+//     with a transposed warp reduction; per-warp partials go to the chunk's
+//     list buffer, then each warp arrives on the buffer's barrier.
+//   * list producer (one warp, lane = row): sums the partials of a chunk,
+//     applies SiLU (Eq. 2) and the mask (Eqs. 4-5) per token, writes the
+//     optional index outputs, frees the buffer, and streams the W_ud rows of
+//     the kept neurons into the W_ud ring (4 slots of 32 KB).
+//   * 8 up/down warps: thread t owns vectors t, t + 256, ... of the up and
+//     down halves of each W_ud row and keeps its y columns in registers.  The
+//     up dot products of a stage are reduced across these warps through a
+//     split barrier: each warp arrives, performs the down projection of the
+//     previous stage (h_j * W_down[j, :] into its y columns), then waits.
+// The two groups run concurrently, so neither kind of row waits behind the
+// other.  After its stream each CTA adds its y partial into the output with
+// vector reductions in L2 (red.global.add.v4.f32); a counter guarantees that
+// every CTA has read its activations (the residual stream, which the output
+// may alias) and zeroed its slice of y before any CTA adds.  When the
+// kept-index lists are requested, every chunk writes one keep byte per neuron
+// and token, and the last CTA to finish turns them into the ascending lists.
 // Every wait is bounded in time; a wait that gives up sets the status word.
 #include <cmath>
 
@@ -41,49 +48,81 @@
 namespace sats {
 namespace {
 
-constexpr int kConsumerWarps = 16;
-constexpr int kConsumers = kConsumerWarps * 32;   // 512
-constexpr int kThreads = kConsumers + 32;         // + producer warp
-constexpr int kStageBytes = 32768;
-constexpr int kStages = 6;
-constexpr int kMaxLook = 4;                       // gate lookahead, chunks
-constexpr int kBufs = kMaxLook + 1;
-constexpr int kMaxRowsPerStage = 16;
+constexpr int kGateWarps = 8;
+constexpr int kUdWarps = 8;
+constexpr int kGateThreads = kGateWarps * 32;        // 256
+constexpr int kUdThreads = kUdWarps * 32;            // 256
+constexpr int kGateProducerWarp = kGateWarps + kUdWarps;   // 16
+constexpr int kListWarp = kGateProducerWarp + 1;           // 17
+constexpr int kThreads = (kListWarp + 1) * 32;             // 576
+constexpr int kGateStageBytes = 16384;
+constexpr int kGateStages = 5;
+constexpr int kUdRingBytes = 131072;
+constexpr int kUdSlots = 4;
+constexpr int kUdSlotBytes = kUdRingBytes / kUdSlots;      // 32 KB
+constexpr int kBufs = 4;                                   // list buffers (gate lookahead, chunks)
+constexpr int kPoolChunksPerCta = 3;                       // chunks of each range left to the shared pool
+constexpr int kMaxUdRows = 8;                              // W_ud rows per stage (small H)
 
-enum StageKind { kGate = 0, kUpDown = 1, kEnd = 2 };
+enum StageKind { kRows = 0, kEnd = 1 };
+
+struct GateDesc {
+    int kind, nrows, chunk_pos, last, buf, pad0, pad1, pad2;
+};
 
 template <int BT>
-struct StageDesc {
-    int kind, nrows, chunk_pos, last, buf, chunk, pad0, pad1;
-    int neuron[kMaxRowsPerStage];
-    float am[kMaxRowsPerStage][BT];   // keep ? a : 0, per row and token
+struct UdDesc {
+    int kind, nrows, pad0, pad1;
+    float am[kMaxUdRows][BT];   // keep ? a : 0, per row and token
 };
 
 template <int BT>
 struct Shared {
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
-    uint64_t csync;                                     // consumer-wide barrier (prologue, W_ud stages)
-    uint64_t gsync[kBufs];                              // per chunk buffer: gate partials written
-    StageDesc<BT> desc[kStages];
-    float gpart[kBufs][kChunk][BT][kConsumerWarps];     // gate partials per chunk buffer
-    float upart[3][kMaxRowsPerStage][BT][kConsumerWarps];   // by W_ud stage, mod 3
-    int bufchunk[kBufs];
-    int issued[kStages];                                // producer: parity+1 of last fill
+    uint64_t gfull[kGateStages], gempty[kGateStages];
+    uint64_t ufull[kUdSlots], uempty[kUdSlots];
+    uint64_t gsync[kBufs];      // gate partials of a buffer written (one arrival per gate warp)
+    uint64_t bfree[kBufs];      // buffer's list formed (one arrival by the list producer)
+    uint64_t xloaded;           // every consumer warp holds its activations
+    uint64_t gbar;              // gate-warp barrier
+    uint64_t ubar;              // up/down-warp barrier
+    GateDesc gdesc[kGateStages];
+    UdDesc<BT> udesc[kUdSlots];
+    float gpart[kBufs][kChunk][BT][kGateWarps];
+    float upart[3][kMaxUdRows][BT][kUdWarps];   // by W_ud stage, mod 3
+    int chunkq[kBufs];          // first neuron of the chunk in a buffer (-1: no more work)
+    int chunkrows[kBufs];
+    int gissued[kGateStages], uissued[kUdSlots];
     float thr[BT];
-    float red[kConsumerWarps][BT];
+    float red[kGateWarps + kUdWarps][BT];
     int warp_sums[kThreads / 32];
     int abort;
 };
 
 template <int BT>
-constexpr size_t smem_bytes() { return (size_t)kStages * kStageBytes + sizeof(Shared<BT>); }
+constexpr size_t smem_bytes()
+{
+    return (size_t)kGateStages * kGateStageBytes + kUdRingBytes + sizeof(Shared<BT>);
+}
 
 __device__ __forceinline__ void flag_status(int *ctl, int bits) { atomicOr(ctl + kCtlStatus, bits); }
 
-// Consumer-wide barrier on an mbarrier (one arrival per consumer warp), bounded
-// in time; arrive() and wait() may be separated by independent work.
-struct ConsumerSync {
+// Geometry of the W_ud ring for a hidden size: rows per stage and slots per stage.
+struct UdGeometry {
+    int rows, slots, stages;
+    size_t stage_bytes;
+    __device__ explicit UdGeometry(int H)
+    {
+        const int row_bytes = 4 * H;
+        rows = max(1, min(kMaxUdRows, kUdSlotBytes / row_bytes));
+        slots = (rows * row_bytes + kUdSlotBytes - 1) / kUdSlotBytes;
+        stages = kUdSlots / slots;
+        stage_bytes = (size_t)slots * kUdSlotBytes;
+    }
+};
+
+// Barrier over one warp group on an mbarrier (one arrival per warp), bounded in
+// time; arrive() and wait() may be separated by independent work.
+struct GroupSync {
     uint64_t *bar;
     uint32_t parity;
     __device__ void arrive(int lane)
@@ -104,179 +143,21 @@ struct ConsumerSync {
     }
 };
 
-// ------------------------------------------------------------------ producer
-// The kept list of one chunk, formed by the producer warp (lane r = row r):
-// sums the consumers' gate partials across warps, applies SiLU (Eq. 2) and the
-// CATS mask (Eqs. 4-5) per token, writes the optional index outputs, and
-// returns the union of the rows kept by any token (a ballot mask) together
-// with each lane's a values and keep bits.
-template <int BT>
-__device__ uint32_t chunk_keep(const FusedParams &p, Shared<BT> &S, int buf, int chunk, int lane, float (&a)[BT],
-                               uint32_t (&bal)[BT])
-{
-    const int n0 = chunk * kChunk;
-    const int rows = min(kChunk, p.N - n0);
-    const bool in = lane < rows;
-    uint32_t uni = 0;
-#pragma unroll
-    for (int b = 0; b < BT; ++b) {
-        float g = 0.f;
-        if (in) {
-#pragma unroll
-            for (int w = 0; w < kConsumerWarps; ++w) g += S.gpart[buf][lane][b][w];
-        }
-        a[b] = g / (1.0f + expf(-g));                                   // SiLU, Eq. 2
-        const bool keep = in && b < p.nb && fabsf(a[b]) >= S.thr[b];    // Eqs. 4-5
-        bal[b] = __ballot_sync(0xffffffffu, keep);
-        uni |= bal[b];
-    }
-    const uint32_t lt = (1u << lane) - 1u;
-    if (p.active_idx) {
-        const int stride = p.nchunks * kChunk;
-#pragma unroll
-        for (int b = 0; b < BT; ++b) {
-            if (b >= p.nb) break;
-            if ((bal[b] >> lane) & 1u) p.idx_tmp[b * stride + n0 + __popc(bal[b] & lt)] = n0 + lane;
-            if (lane == 0) p.chunk_cnt[chunk * kMaxTokensPerPass + b] = __popc(bal[b]);
-        }
-    }
-    if (p.keep_trace && in) {
-#pragma unroll
-        for (int b = 0; b < BT; ++b)
-            if (b < p.nb) p.keep_trace[(size_t)b * p.N + n0 + lane] = (uint8_t)((bal[b] >> lane) & 1u);
-    }
-    return uni;
-}
-
-// Runs on the whole producer warp with uniform control flow; lane 0 claims
-// chunks and posts gate stages, every lane whose row is kept issues that row's
-// W_ud copy.
-template <int BT>
-__device__ void producer(const FusedParams &p, Shared<BT> &S, uint8_t *stages, int look, int lane)
-{
-    const uint64_t pol = l2_policy_evict_first();
-    const int H = p.H, N = p.N;
-    const uint32_t gate_row_bytes = (uint32_t)H * 2u;
-    const uint32_t ud_row_bytes = (uint32_t)H * 4u;
-    const int rows_per_gate_stage = min(kChunk, kStageBytes / (int)gate_row_bytes);
-    const int rows_per_ud_stage = min(kMaxRowsPerStage, kStageBytes / (int)ud_row_bytes);
-    const int nbufs = look + 1;
-    int *counter = p.ctl + kCtlChunk;
-    const uint32_t lt = (1u << lane) - 1u;
-
-    uint32_t stage = 0, phase = 0;
-    int seq_gate = 0, seq_ud = 0;     // chunks whose gate / W_ud rows have been issued
-    bool more = true, ok = true;
-    int next = 0;
-    if (lane == 0) next = atomicAdd(counter, 1);
-    next = __shfl_sync(0xffffffffu, next, 0);
-
-    for (;;) {
-        // gate rows, up to `look` chunks ahead of the W_ud rows
-        while (ok && more && seq_gate - seq_ud <= look) {
-            const int c = next;
-            if (c >= p.nchunks) { more = false; break; }
-            if (lane == 0) next = atomicAdd(counter, 1);
-            next = __shfl_sync(0xffffffffu, next, 0);
-            const int buf = seq_gate % nbufs;
-            const int n0 = c * kChunk;
-            const int rows = min(kChunk, N - n0);
-            for (int r0 = 0; r0 < rows; r0 += rows_per_gate_stage) {
-                const int nr = min(rows_per_gate_stage, rows - r0);
-                if (!mbar_wait(&S.empty[stage], phase ^ 1u, &S.abort)) { ok = false; break; }
-                if (lane == 0) {
-                    StageDesc<BT> &d = S.desc[stage];
-                    d.kind = kGate;
-                    d.nrows = nr;
-                    d.chunk_pos = r0;
-                    d.last = (r0 + nr >= rows) ? 1 : 0;
-                    d.buf = buf;
-                    d.chunk = c;
-                    S.issued[stage] = (int)phase + 1;
-                    mbar_arrive_expect_tx(&S.full[stage], (uint32_t)nr * gate_row_bytes);
-                    bulk_load(stages + (size_t)stage * kStageBytes, p.wg_t + (size_t)(n0 + r0) * H,
-                              (uint32_t)nr * gate_row_bytes, &S.full[stage], pol);
-                }
-                __syncwarp();
-                if (++stage == kStages) { stage = 0; phase ^= 1u; }
-            }
-            if (lane == 0) S.bufchunk[buf] = c;
-            ++seq_gate;
-        }
-        if (!ok || seq_ud == seq_gate) break;
-        // kept list of the oldest chunk whose gate rows were issued, then its W_ud rows
-        const int buf = seq_ud % nbufs;
-        if (!mbar_wait(&S.gsync[buf], (uint32_t)(seq_ud / nbufs) & 1u, &S.abort)) { ok = false; break; }
-        __syncwarp();
-        const int chunk = S.bufchunk[buf];
-        float a[BT];
-        uint32_t bal[BT];
-        const uint32_t uni = chunk_keep<BT>(p, S, buf, chunk, lane, a, bal);
-        const int cnt = __popc(uni);
-        const int pos = __popc(uni & lt);
-        const bool mine = (uni >> lane) & 1u;
-        const int nid = chunk * kChunk + lane;
-        for (int k0 = 0; k0 < cnt; k0 += rows_per_ud_stage) {
-            const int nr = min(rows_per_ud_stage, cnt - k0);
-            if (!mbar_wait(&S.empty[stage], phase ^ 1u, &S.abort)) { ok = false; break; }
-            StageDesc<BT> &d = S.desc[stage];
-            const bool in_stage = mine && pos >= k0 && pos < k0 + nr;
-            if (in_stage) {
-                const int k = pos - k0;
-                d.neuron[k] = nid;
-#pragma unroll
-                for (int b = 0; b < BT; ++b) d.am[k][b] = ((bal[b] >> lane) & 1u) ? a[b] : 0.f;
-            }
-            __syncwarp();     // descriptor entries written before lane 0's release below
-            if (lane == 0) {
-                d.kind = kUpDown;
-                d.nrows = nr;
-                S.issued[stage] = (int)phase + 1;
-                mbar_arrive_expect_tx(&S.full[stage], (uint32_t)nr * ud_row_bytes);
-            }
-            __syncwarp();
-            if (in_stage)
-                bulk_load(stages + (size_t)stage * kStageBytes + (size_t)(pos - k0) * ud_row_bytes,
-                          p.w_ud + (size_t)nid * 2 * H, ud_row_bytes, &S.full[stage], pol);
-            __syncwarp();
-            if (++stage == kStages) { stage = 0; phase ^= 1u; }
-        }
-        ++seq_ud;
-    }
-    if (ok && mbar_wait(&S.empty[stage], phase ^ 1u, &S.abort)) {
-        if (lane == 0) {
-            S.desc[stage].kind = kEnd;
-            mbar_arrive(&S.full[stage]);
-        }
-    } else if (lane == 0) {
-        S.abort = 1;
-        flag_status(p.ctl, kStatusTimeout);
-    }
-    __syncwarp();
-}
-
-// Bounded wait for every bulk copy still in flight (only on the error path).
-template <int BT>
-__device__ void drain_copies(Shared<BT> &S)
-{
-    int never = 0;
-    for (int s = 0; s < kStages; ++s)
-        if (S.issued[s] > 0) (void)mbar_wait(&S.full[s], (uint32_t)(S.issued[s] - 1), &never);
-}
-
-// ------------------------------------------------------------------ consumers
+// Activations of this pass for one warp group: thread `t` of `nthreads` owns
+// the vectors t + nthreads * i (i < VPT).  RMSNorm (kXResidNorm) reduces over
+// the group through `gs`, using red[red0 + warp-in-group].
 template <int BT, int VPT>
-__device__ void load_activations(const FusedParams &p, Shared<BT> &S, ConsumerSync &csync, int tid,
-                                 f32x2 (&xp)[BT][VPT][4], bool &ok)
+__device__ bool load_activations(const FusedParams &p, Shared<BT> &S, GroupSync &gs, int t, int nthreads,
+                                 int red0, f32x2 (&xp)[BT][VPT][4])
 {
-    const int lane = tid & 31, warp = tid >> 5;
+    const int lane = t & 31, gw = t >> 5, nw = nthreads >> 5;
     const int H = p.H, HV = H >> 3;
     float xv[BT][VPT][8];
 #pragma unroll
     for (int b = 0; b < BT; ++b)
 #pragma unroll
         for (int i = 0; i < VPT; ++i) {
-            const int v = tid + i * kConsumers;
+            const int v = t + i * nthreads;
 #pragma unroll
             for (int e = 0; e < 8; ++e) xv[b][i][e] = 0.f;
             if (v < HV && b < p.nb) {
@@ -305,20 +186,20 @@ __device__ void load_activations(const FusedParams &p, Shared<BT> &S, ConsumerSy
         }
         if (lane == 0) {
 #pragma unroll
-            for (int b = 0; b < BT; ++b) S.red[warp][b] = ss[b];
+            for (int b = 0; b < BT; ++b) S.red[red0 + gw][b] = ss[b];
         }
-        if (!csync(lane, &S.abort)) { ok = false; return; }
+        if (!gs(lane, &S.abort)) return false;
 #pragma unroll
         for (int b = 0; b < BT; ++b) {
             float tot = 0.f;
-            for (int w = 0; w < kConsumerWarps; ++w) tot += S.red[w][b];
+            for (int w = 0; w < nw; ++w) tot += S.red[red0 + w][b];
             const float inv = 1.0f / sqrtf(tot / (float)H + p.eps);
 #pragma unroll
             for (int i = 0; i < VPT; ++i) {
-                const int v = tid + i * kConsumers;
+                const int v = t + i * nthreads;
                 if (v < HV) {
-                    const float4 *gw = reinterpret_cast<const float4 *>(p.norm_w);
-                    const float4 lo = gw[2 * v], hi = gw[2 * v + 1];
+                    const float4 *gw4 = reinterpret_cast<const float4 *>(p.norm_w);
+                    const float4 lo = gw4[2 * v], hi = gw4[2 * v + 1];
                     const float g8[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
 #pragma unroll
                     for (int e = 0; e < 8; ++e) xv[b][i][e] = xv[b][i][e] * inv * g8[e];
@@ -332,15 +213,267 @@ __device__ void load_activations(const FusedParams &p, Shared<BT> &S, ConsumerSy
         for (int i = 0; i < VPT; ++i)
 #pragma unroll
             for (int e = 0; e < 4; ++e) xp[b][i][e] = pack2(xv[b][i][2 * e], xv[b][i][2 * e + 1]);
+    return true;
 }
 
-// Down projection of one W_ud stage: y[cols] += h_j * W_down[j, cols] for the
-// stage's rows, with h_j = am_j * u_j and u_j the cross-warp sum of the stage's
-// up partials.  Then releases the stage to the producer.
+// ------------------------------------------------------------------ gate producer
+template <int BT>
+__device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *gring)
+{
+    const uint64_t pol = l2_policy_evict_first();
+    const int H = p.H, N = p.N;
+    const uint32_t row_bytes = (uint32_t)H * 2u;
+    const int rows_per_stage = min(kChunk, kGateStageBytes / (int)row_bytes);
+    // this CTA's contiguous neuron range [nb0, nb1): N / gridDim neurons, +-1;
+    // its first `own` chunks are this CTA's, the rest go to the shared pool
+    const int nb0 = (int)((long long)blockIdx.x * N / gridDim.x);
+    const int nb1 = (int)((long long)(blockIdx.x + 1) * N / gridDim.x);
+    const int own = max(0, (nb1 - nb0 + kChunk - 1) / kChunk - kPoolChunksPerCta);
+    int next_k = own == 0 ? atomicAdd(p.ctl + kCtlPool, 1) : -1;   // a claimed, not yet used pool chunk
+    uint32_t stage = 0, phase = 0;
+    bool ok = true;
+    for (int seq = 0;; ++seq) {
+        const int buf = seq % kBufs;
+        // the buffer's previous list has been formed (first kBufs uses pass)
+        if (!mbar_wait(&S.bfree[buf], ((uint32_t)(seq / kBufs) & 1u) ^ 1u, &S.abort)) { ok = false; break; }
+        int n0 = -1, end = 0;
+        if (seq < own) {
+            n0 = nb0 + seq * kChunk;
+            end = nb1;
+            // claim the first pool chunk while the own chunks still stream
+            if (seq + 1 == own && next_k < 0) next_k = atomicAdd(p.ctl + kCtlPool, 1);
+        } else {
+            // pool chunk k: chunk (own_c + k % P) of CTA k / P's range; the
+            // next claim is issued before this chunk's rows are streamed
+            for (;;) {
+                const int k = next_k >= 0 ? next_k : atomicAdd(p.ctl + kCtlPool, 1);
+                next_k = -1;
+                if (k >= (int)gridDim.x * kPoolChunksPerCta) break;
+                const int c = k / kPoolChunksPerCta, j = k % kPoolChunksPerCta;
+                const int c0 = (int)((long long)c * N / gridDim.x), c1 = (int)((long long)(c + 1) * N / gridDim.x);
+                const int cown = max(0, (c1 - c0 + kChunk - 1) / kChunk - kPoolChunksPerCta);
+                const int m0 = c0 + (cown + j) * kChunk;
+                if (m0 < c1) {
+                    n0 = m0;
+                    end = c1;
+                    next_k = atomicAdd(p.ctl + kCtlPool, 1);
+                    break;
+                }
+            }
+        }
+        if (n0 < 0) {
+            S.chunkq[buf] = -1;                                   // end of work for the list producer
+            for (int w = 0; w < kGateWarps; ++w) mbar_arrive(&S.gsync[buf]);
+            break;
+        }
+        const int rows = min(kChunk, end - n0);
+        S.chunkq[buf] = n0;
+        S.chunkrows[buf] = rows;
+        for (int r0 = 0; r0 < rows; r0 += rows_per_stage) {
+            const int nr = min(rows_per_stage, rows - r0);
+            if (!mbar_wait(&S.gempty[stage], phase ^ 1u, &S.abort)) { ok = false; break; }
+            GateDesc &d = S.gdesc[stage];
+            d.kind = kRows;
+            d.nrows = nr;
+            d.chunk_pos = r0;
+            d.last = (r0 + nr >= rows) ? 1 : 0;
+            d.buf = buf;
+            S.gissued[stage] = (int)phase + 1;
+            mbar_arrive_expect_tx(&S.gfull[stage], (uint32_t)nr * row_bytes);
+            bulk_load(gring + (size_t)stage * kGateStageBytes, p.wg_t + (size_t)(n0 + r0) * H, (uint32_t)nr * row_bytes,
+                      &S.gfull[stage], pol);
+            if (++stage == kGateStages) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+    }
+    if (ok && mbar_wait(&S.gempty[stage], phase ^ 1u, &S.abort)) {
+        S.gdesc[stage].kind = kEnd;
+        mbar_arrive(&S.gfull[stage]);
+    } else {
+        S.abort = 1;
+        flag_status(p.ctl, kStatusTimeout);
+    }
+}
+
+// ------------------------------------------------------------------ gate warps
 template <int BT, int VPT>
-__device__ __forceinline__ void down_stage(const FusedParams &p, Shared<BT> &S, const uint8_t *sbase,
-                                           const StageDesc<BT> &d, int nr, int ub, uint32_t stage, int tid, int lane,
-                                           f32x2 (&yp)[BT][VPT][4])
+__device__ void gate_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *gring)
+{
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int H = p.H, HV = H >> 3;
+    const size_t row_bytes = (size_t)H * 2;
+    const uint4 zero4 = make_uint4(0u, 0u, 0u, 0u);
+    GroupSync gs{&S.gbar, 0u};
+    f32x2 xp[BT][VPT][4];
+    const bool loaded = load_activations<BT, VPT>(p, S, gs, t, kGateThreads, 0, xp);
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&S.xloaded);
+    if (!loaded) {
+        S.abort = 1;
+        flag_status(p.ctl, kStatusTimeout);
+        return;
+    }
+    uint32_t stage = 0, phase = 0;
+    for (;;) {
+        if (!mbar_wait(&S.gfull[stage], phase, &S.abort)) {
+            S.abort = 1;
+            flag_status(p.ctl, kStatusTimeout);
+            return;
+        }
+        const GateDesc &d = S.gdesc[stage];
+        if (d.kind == kEnd) break;
+        const int nr = d.nrows, r0 = d.chunk_pos, buf = d.buf, last = d.last;
+        const uint8_t *sbase = gring + (size_t)stage * kGateStageBytes;
+        for (int q = 0; q < nr; q += 2) {
+            // two rows at once: independent FMA chains, one transposed reduction
+            f32x2 acc[2][BT];
+#pragma unroll
+            for (int r = 0; r < 2; ++r)
+#pragma unroll
+                for (int b = 0; b < BT; ++b) acc[r][b] = 0ull;
+            const bool pair = q + 2 <= nr;
+#pragma unroll
+            for (int i = 0; i < VPT; ++i) {
+                const int v = t + i * kGateThreads;
+                if (v < HV) {
+                    const uint4 w0 = reinterpret_cast<const uint4 *>(sbase + (size_t)q * row_bytes)[v];
+                    const uint4 w1 = pair ? reinterpret_cast<const uint4 *>(sbase + (size_t)(q + 1) * row_bytes)[v] : zero4;
+#pragma unroll
+                    for (int b = 0; b < BT; ++b) {
+                        acc[0][b] = dot8_acc(w0, xp[b][i], acc[0][b]);
+                        acc[1][b] = dot8_acc(w1, xp[b][i], acc[1][b]);
+                    }
+                }
+            }
+#pragma unroll
+            for (int b = 0; b < BT; ++b) {
+                const float tot = warp_sum2_transposed(hsum2(acc[0][b]), hsum2(acc[1][b]), lane);
+                const int r = lane >> 4;
+                if ((lane & 15) == 0 && q + r < nr) S.gpart[buf][r0 + q + r][b][warp] = tot;
+            }
+        }
+        __syncwarp();
+        if (lane == 0) {
+            mbar_arrive(&S.gempty[stage]);
+            if (last) mbar_arrive(&S.gsync[buf]);   // this warp's partials of the chunk are written
+        }
+        if (++stage == kGateStages) { stage = 0; phase ^= 1u; }
+    }
+}
+
+// Row stride of the keep bytes (16-byte aligned rows, so they load as uint4).
+__device__ __forceinline__ int keep_stride(int N) { return (N + 15) & ~15; }
+
+// ------------------------------------------------------------------ list producer
+// Lane r = row r of the chunk: sums the gate partials across the gate warps,
+// SiLU (Eq. 2), CATS mask (Eqs. 4-5) per token, index outputs.  Returns the
+// union of rows kept by any token, with each lane's a values and keep bits.
+template <int BT>
+__device__ uint32_t chunk_keep(const FusedParams &p, Shared<BT> &S, int buf, int n0, int rows, int lane,
+                               float (&a)[BT], uint32_t (&bal)[BT])
+{
+    const bool in = lane < rows;
+    uint32_t uni = 0;
+#pragma unroll
+    for (int b = 0; b < BT; ++b) {
+        float g = 0.f;
+        if (in) {
+#pragma unroll
+            for (int w = 0; w < kGateWarps; ++w) g += S.gpart[buf][lane][b][w];
+        }
+        a[b] = g / (1.0f + expf(-g));                                   // SiLU, Eq. 2
+        const bool keep = in && b < p.nb && fabsf(a[b]) >= S.thr[b];    // Eqs. 4-5
+        bal[b] = __ballot_sync(0xffffffffu, keep);
+        uni |= bal[b];
+    }
+    if (in) {
+#pragma unroll
+        for (int b = 0; b < BT; ++b) {
+            if (b >= p.nb) break;
+            const uint8_t k = (uint8_t)((bal[b] >> lane) & 1u);
+            if (p.active_idx) p.keep_tmp[(size_t)b * keep_stride(p.N) + n0 + lane] = k;
+            if (p.keep_trace) p.keep_trace[(size_t)b * p.N + n0 + lane] = k;
+        }
+    }
+    return uni;
+}
+
+template <int BT>
+__device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *uring, int lane)
+{
+    const uint64_t pol = l2_policy_evict_first();
+    const int H = p.H;
+    const uint32_t ud_row_bytes = (uint32_t)H * 4u;
+    const UdGeometry geo(H);
+    const uint32_t lt = (1u << lane) - 1u;
+    uint32_t stage = 0, phase = 0;
+    bool ok = mbar_wait(&S.xloaded, 0u, &S.abort);
+    if (ok && lane == 0) {
+        // this CTA has read its activations and zeroed its slice of y
+        __threadfence();
+        atomicAdd(p.ctl + kCtlPrologue, 1);
+    }
+    __syncwarp();
+    for (int seq = 0; ok; ++seq) {
+        const int buf = seq % kBufs;
+        if (!mbar_wait(&S.gsync[buf], (uint32_t)(seq / kBufs) & 1u, &S.abort)) { ok = false; break; }
+        __syncwarp();
+        const int n0 = S.chunkq[buf];
+        if (n0 < 0) break;
+        const int rows = S.chunkrows[buf];
+        float a[BT];
+        uint32_t bal[BT];
+        const uint32_t uni = chunk_keep<BT>(p, S, buf, n0, rows, lane, a, bal);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&S.bfree[buf]);   // partials read: the gate producer may refill the buffer
+        const int cnt = __popc(uni);
+        const int pos = __popc(uni & lt);
+        const bool mine = (uni >> lane) & 1u;
+        const int nid = n0 + lane;
+        for (int k0 = 0; k0 < cnt; k0 += geo.rows) {
+            const int nr = min(geo.rows, cnt - k0);
+            if (!mbar_wait(&S.uempty[stage], phase ^ 1u, &S.abort)) { ok = false; break; }
+            UdDesc<BT> &d = S.udesc[stage];
+            const bool in_stage = mine && pos >= k0 && pos < k0 + nr;
+            if (in_stage) {
+#pragma unroll
+                for (int b = 0; b < BT; ++b) d.am[pos - k0][b] = ((bal[b] >> lane) & 1u) ? a[b] : 0.f;
+            }
+            __syncwarp();     // descriptor entries written before lane 0's release below
+            if (lane == 0) {
+                d.kind = kRows;
+                d.nrows = nr;
+                S.uissued[stage] = (int)phase + 1;
+                mbar_arrive_expect_tx(&S.ufull[stage], (uint32_t)nr * ud_row_bytes);
+            }
+            __syncwarp();
+            if (in_stage)
+                bulk_load(uring + (size_t)stage * geo.stage_bytes + (size_t)(pos - k0) * ud_row_bytes,
+                          p.w_ud + (size_t)nid * 2 * H, ud_row_bytes, &S.ufull[stage], pol);
+            __syncwarp();
+            if (++stage == (uint32_t)geo.stages) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+    }
+    if (ok && mbar_wait(&S.uempty[stage], phase ^ 1u, &S.abort)) {
+        if (lane == 0) {
+            S.udesc[stage].kind = kEnd;
+            mbar_arrive(&S.ufull[stage]);
+        }
+    } else if (lane == 0) {
+        S.abort = 1;
+        flag_status(p.ctl, kStatusTimeout);
+    }
+    __syncwarp();
+}
+
+// ------------------------------------------------------------------ up/down warps
+// Down projection of one W_ud stage: y[cols] += h_j * W_down[j, cols], with
+// h_j = am_j * u_j and u_j the cross-warp sum of the stage's up partials; then
+// releases the stage to the list producer.
+template <int BT, int VPT>
+__device__ __forceinline__ void down_stage(const FusedParams &p, Shared<BT> &S, const uint8_t *sbase, int nr,
+                                           int ub, int st, int t, int lane, f32x2 (&yp)[BT][VPT][4])
 {
     const int H = p.H, HV = H >> 3;
     const size_t ud_row_bytes = (size_t)H * 4;
@@ -348,16 +481,16 @@ __device__ __forceinline__ void down_stage(const FusedParams &p, Shared<BT> &S, 
         f32x2 hh[BT];
 #pragma unroll
         for (int b = 0; b < BT; ++b) {
-            float u = S.upart[ub][k][b][lane & (kConsumerWarps - 1)];
+            float u = S.upart[ub][k][b][lane & (kUdWarps - 1)];
 #pragma unroll
-            for (int o = kConsumerWarps / 2; o > 0; o >>= 1) u += __shfl_xor_sync(0xffffffffu, u, o);
-            const float h = d.am[k][b] * u;     // CATS_t(a) * (x W_up), Eqs. 1 and 5
+            for (int o = kUdWarps / 2; o > 0; o >>= 1) u += __shfl_xor_sync(0xffffffffu, u, o);
+            const float h = S.udesc[st].am[k][b] * u;     // CATS_t(a) * (x W_up), Eqs. 1 and 5
             hh[b] = pack2(h, h);
         }
         const uint4 *down = reinterpret_cast<const uint4 *>(sbase + (size_t)k * ud_row_bytes + (size_t)H * 2);
 #pragma unroll
         for (int i = 0; i < VPT; ++i) {
-            const int v = tid + i * kConsumers;
+            const int v = t + i * kUdThreads;
             if (v < HV) {
                 const uint4 w = down[v];
 #pragma unroll
@@ -366,18 +499,19 @@ __device__ __forceinline__ void down_stage(const FusedParams &p, Shared<BT> &S, 
         }
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(&S.empty[stage]);
+    if (lane == 0) mbar_arrive(&S.uempty[st]);
 }
 
 template <int BT, int VPT>
-__device__ void consumer(const FusedParams &p, Shared<BT> &S, const uint8_t *stages, f32x2 (&yp)[BT][VPT][4])
+__device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *uring, f32x2 (&yp)[BT][VPT][4])
 {
-    const int tid = threadIdx.x;
-    const int warp = tid >> 5, lane = tid & 31;
+    const int t = threadIdx.x - kGateThreads;
+    const int lane = t & 31, uw = t >> 5;
     const int H = p.H, HV = H >> 3;
-    const size_t gate_row_bytes = (size_t)H * 2, ud_row_bytes = (size_t)H * 4;
-    ConsumerSync csync{&S.csync, 0u};
+    const size_t ud_row_bytes = (size_t)H * 4;
+    const UdGeometry geo(H);
     const uint4 zero4 = make_uint4(0u, 0u, 0u, 0u);
+    GroupSync us{&S.ubar, 0u};
 
 #pragma unroll
     for (int b = 0; b < BT; ++b)
@@ -385,194 +519,137 @@ __device__ void consumer(const FusedParams &p, Shared<BT> &S, const uint8_t *sta
         for (int i = 0; i < VPT; ++i)
 #pragma unroll
             for (int e = 0; e < 4; ++e) yp[b][i][e] = 0ull;
-
     f32x2 xp[BT][VPT][4];
-    bool ok = true;
-    load_activations<BT, VPT>(p, S, csync, tid, xp, ok);
-    if (!ok) { S.abort = 1; flag_status(p.ctl, kStatusTimeout); return; }
-
+    const bool loaded = load_activations<BT, VPT>(p, S, us, t, kUdThreads, kGateWarps, xp);
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&S.xloaded);
+    if (!loaded) {
+        S.abort = 1;
+        flag_status(p.ctl, kStatusTimeout);
+        return;
+    }
     uint32_t stage = 0, phase = 0;
     int ud_seq = 0;
     // a W_ud stage whose up sums are complete but whose down projection is
-    // still to do (it is done while waiting on the next W_ud stage's barrier)
+    // still to do (done while waiting on the next stage's barrier)
     int pend_stage = -1, pend_nr = 0, pend_ub = 0;
     for (;;) {
-        if (!mbar_wait(&S.full[stage], phase, &S.abort)) {
+        if (!mbar_wait(&S.ufull[stage], phase, &S.abort)) {
             S.abort = 1;
             flag_status(p.ctl, kStatusTimeout);
             return;
         }
-        const StageDesc<BT> &d = S.desc[stage];
-        const int kind = d.kind;
-        if (kind != kUpDown && pend_stage >= 0) {
-            down_stage<BT, VPT>(p, S, stages + (size_t)pend_stage * kStageBytes, S.desc[pend_stage], pend_nr,
-                                pend_ub, (uint32_t)pend_stage, tid, lane, yp);
-            pend_stage = -1;
+        const UdDesc<BT> &d = S.udesc[stage];
+        if (d.kind == kEnd) {
+            if (pend_stage >= 0)
+                down_stage<BT, VPT>(p, S, uring + (size_t)pend_stage * geo.stage_bytes, pend_nr, pend_ub, pend_stage,
+                                    t, lane, yp);
+            break;
         }
-        if (kind == kEnd) break;
-        const uint8_t *sbase = stages + (size_t)stage * kStageBytes;
         const int nr = d.nrows;
-        if (kind == kGate) {
-            const int r0 = d.chunk_pos, buf = d.buf, last = d.last;
-            for (int q = 0; q < nr; q += 4) {
-                // four rows at once: independent FMA chains, one transposed reduction
-                f32x2 acc[4][BT];
+        const int ub = ud_seq % 3;
+        const uint8_t *sbase = uring + (size_t)stage * geo.stage_bytes;
+        // up dot products, two rows at a time
+        for (int q = 0; q < nr; q += 2) {
+            f32x2 acc[2][BT];
 #pragma unroll
-                for (int r = 0; r < 4; ++r)
+            for (int r = 0; r < 2; ++r)
 #pragma unroll
-                    for (int b = 0; b < BT; ++b) acc[r][b] = 0ull;
+                for (int b = 0; b < BT; ++b) acc[r][b] = 0ull;
 #pragma unroll
-                for (int i = 0; i < VPT; ++i) {
-                    const int v = tid + i * kConsumers;
-                    if (v < HV) {
-                        uint4 w[4];
+            for (int i = 0; i < VPT; ++i) {
+                const int v = t + i * kUdThreads;
+                if (v < HV) {
+                    uint4 w[2];
 #pragma unroll
-                        for (int r = 0; r < 4; ++r)
-                            w[r] = (q + r < nr)
-                                       ? reinterpret_cast<const uint4 *>(sbase + (size_t)(q + r) * gate_row_bytes)[v]
-                                       : zero4;
+                    for (int r = 0; r < 2; ++r)
+                        w[r] = (q + r < nr) ? reinterpret_cast<const uint4 *>(sbase + (size_t)(q + r) * ud_row_bytes)[v]
+                                            : zero4;
 #pragma unroll
-                        for (int r = 0; r < 4; ++r)
+                    for (int r = 0; r < 2; ++r)
 #pragma unroll
-                            for (int b = 0; b < BT; ++b) acc[r][b] = dot8_acc(w[r], xp[b][i], acc[r][b]);
-                    }
-                }
-#pragma unroll
-                for (int b = 0; b < BT; ++b) {
-                    const float tot = warp_sum4_transposed(hsum2(acc[0][b]), hsum2(acc[1][b]), hsum2(acc[2][b]),
-                                                           hsum2(acc[3][b]), lane);
-                    const int r = (lane >> 3) & 3;
-                    if ((lane & 7) == 0 && q + r < nr) S.gpart[buf][r0 + q + r][b][warp] = tot;
+                        for (int b = 0; b < BT; ++b) acc[r][b] = dot8_acc(w[r], xp[b][i], acc[r][b]);
                 }
             }
-            __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&S.empty[stage]);
-                if (last) mbar_arrive(&S.gsync[buf]);   // this warp's partials of the chunk are written
+#pragma unroll
+            for (int b = 0; b < BT; ++b) {
+                const float tot = warp_sum2_transposed(hsum2(acc[0][b]), hsum2(acc[1][b]), lane);
+                const int r = lane >> 4;
+                if ((lane & 15) == 0 && q + r < nr) S.upart[ub][q + r][b][uw] = tot;
             }
-        } else {
-            const int ub = ud_seq % 3;
-            // up dot products, two rows at a time
-            for (int q = 0; q < nr; q += 2) {
-                f32x2 acc[2][BT];
-#pragma unroll
-                for (int r = 0; r < 2; ++r)
-#pragma unroll
-                    for (int b = 0; b < BT; ++b) acc[r][b] = 0ull;
-#pragma unroll
-                for (int i = 0; i < VPT; ++i) {
-                    const int v = tid + i * kConsumers;
-                    if (v < HV) {
-                        uint4 w[2];
-#pragma unroll
-                        for (int r = 0; r < 2; ++r)
-                            w[r] = (q + r < nr) ? reinterpret_cast<const uint4 *>(sbase + (size_t)(q + r) * ud_row_bytes)[v]
-                                                : zero4;
-#pragma unroll
-                        for (int r = 0; r < 2; ++r)
-#pragma unroll
-                            for (int b = 0; b < BT; ++b) acc[r][b] = dot8_acc(w[r], xp[b][i], acc[r][b]);
-                    }
-                }
-#pragma unroll
-                for (int b = 0; b < BT; ++b) {
-                    const float tot = warp_sum2_transposed(hsum2(acc[0][b]), hsum2(acc[1][b]), lane);
-                    const int r = lane >> 4;
-                    if ((lane & 15) == 0 && q + r < nr) S.upart[ub][q + r][b][warp] = tot;
-                }
-            }
-            csync.arrive(lane);
-            if (pend_stage >= 0) {
-                down_stage<BT, VPT>(p, S, stages + (size_t)pend_stage * kStageBytes, S.desc[pend_stage], pend_nr,
-                                    pend_ub, (uint32_t)pend_stage, tid, lane, yp);
-            }
-            if (!csync.wait(&S.abort)) { S.abort = 1; flag_status(p.ctl, kStatusTimeout); return; }
-            pend_stage = (int)stage;
-            pend_nr = nr;
-            pend_ub = ub;
-            ++ud_seq;
         }
-        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        us.arrive(lane);
+        if (pend_stage >= 0)
+            down_stage<BT, VPT>(p, S, uring + (size_t)pend_stage * geo.stage_bytes, pend_nr, pend_ub, pend_stage, t,
+                                lane, yp);
+        if (!us.wait(&S.abort)) {
+            S.abort = 1;
+            flag_status(p.ctl, kStatusTimeout);
+            return;
+        }
+        pend_stage = (int)stage;
+        pend_nr = nr;
+        pend_ub = ub;
+        ++ud_seq;
+        if (++stage == (uint32_t)geo.stages) { stage = 0; phase ^= 1u; }
     }
 }
 
-// ------------------------------------------------------------------ grid-wide tail
-__device__ bool grid_barrier(int *ctl)
-{
-    __shared__ int ok_s;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        int ok = 1;
-        __threadfence();
-        const int gen = ld_acquire_gpu(ctl + kCtlBarGen);
-        const int arrived = atomicAdd(ctl + kCtlBarCount, 1);
-        if (arrived == (int)gridDim.x - 1) {
-            atomicExch(ctl + kCtlBarCount, 0);
-            atomicExch(ctl + kCtlChunk, 0);
-            __threadfence();
-            st_release_gpu(ctl + kCtlBarGen, gen + 1);
-        } else {
-            const unsigned long long t0 = global_ns();
-            while (ld_acquire_gpu(ctl + kCtlBarGen) == gen) {
-                if (global_ns() - t0 > kWaitLimitNs) {
-                    flag_status(ctl, kStatusTimeout);
-                    ok = 0;
-                    break;
-                }
-                __nanosleep(32);
-            }
-        }
-        __threadfence();
-        ok_s = ok;
-    }
-    __syncthreads();
-    return ok_s != 0;
-}
-
-__device__ void reduce_partials(const FusedParams &p)
-{
-    const int H4 = p.H >> 2;
-    const int total = p.nb * H4;                       // float4 elements of y for this pass
-    const int G = gridDim.x;
-    const int per = (total + G - 1) / G;
-    const int q0 = blockIdx.x * per;
-    const int q1 = min(total, q0 + per);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nwarps = kThreads / 32;
-    const float4 *part = reinterpret_cast<const float4 *>(p.partials);
-    for (int q = q0 + warp; q < q1; q += nwarps) {
-        const int b = q / H4, c4 = q - b * H4;
-        float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int g = lane; g < G; g += 32) {
-            const float4 v = __ldcg(part + ((size_t)g * kMaxTokensPerPass + b) * H4 + c4);
-            s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
-        }
-        s.x = warp_sum(s.x); s.y = warp_sum(s.y); s.z = warp_sum(s.z); s.w = warp_sum(s.w);
-        if (lane == 0) {
-            float4 *dst = reinterpret_cast<float4 *>(p.out) + (size_t)b * H4 + c4;
-            if (p.out_mode == kOutResid) {
-                const float4 r = __ldcg(dst);
-                s.x += r.x; s.y += r.y; s.z += r.z; s.w += r.w;
-            }
-            *dst = s;
-        }
-    }
-}
-
+// Bounded wait for every bulk copy still in flight (only on the error path).
 template <int BT>
-__device__ void compact_indices(const FusedParams &p, Shared<BT> &S, int *prefix)
+__device__ void drain_copies(Shared<BT> &S)
 {
+    int never = 0;
+    for (int s = 0; s < kGateStages; ++s)
+        if (S.gissued[s] > 0) (void)mbar_wait(&S.gfull[s], (uint32_t)(S.gissued[s] - 1), &never);
+    for (int s = 0; s < kUdSlots; ++s)
+        if (S.uissued[s] > 0) (void)mbar_wait(&S.ufull[s], (uint32_t)(S.uissued[s] - 1), &never);
+}
+
+// ------------------------------------------------------------------ tail
+// Waits (bounded) until every CTA has passed its prologue.
+__device__ bool wait_prologues(int *ctl)
+{
+    const unsigned long long t0 = global_ns();
+    while (ld_acquire_gpu(ctl + kCtlPrologue) < (int)gridDim.x) {
+        if (global_ns() - t0 > kWaitLimitNs) {
+            flag_status(ctl, kStatusTimeout);
+            return false;
+        }
+        __nanosleep(64);
+    }
+    return true;
+}
+
+// The ascending per-token kept lists from the keep bytes of all chunks; run by
+// the last CTA to finish, when every chunk's bytes are in memory.
+template <int BT>
+__device__ void compact_indices(const FusedParams &p, Shared<BT> &S)
+{
+    constexpr int kMaxBlocksPerThread = 8;                  // 16 keep bytes per block
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int nw = kThreads / 32;
-    const int nc = p.nchunks;
-    const int stride = nc * kChunk;
-    const int per = (nc + kThreads - 1) / kThreads;
+    const int N = p.N;
+    const int nblk = keep_stride(N) / 16;
+    const int bpt = (nblk + kThreads - 1) / kThreads;       // contiguous blocks per thread
+    const int q0 = tid * bpt;
     for (int b = 0; b < p.nb; ++b) {
-        // exclusive scan of the per-chunk counts of token b
-        const int c0 = min(nc, tid * per), c1 = min(nc, c0 + per);
-        int local = 0;
-        for (int c = c0; c < c1; ++c) local += __ldcg(p.chunk_cnt + c * kMaxTokensPerPass + b);
-        int incl = local;
+        const uint4 *kb = reinterpret_cast<const uint4 *>(p.keep_tmp + (size_t)b * keep_stride(N));
+        // one pass of independent 16-byte loads for the common sizes, then a loop
+        uint4 blk[kMaxBlocksPerThread];
+        int cnt = 0;
+#pragma unroll
+        for (int i = 0; i < kMaxBlocksPerThread; ++i) {
+            blk[i] = (i < bpt && q0 + i < nblk) ? __ldcg(kb + q0 + i) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int i = 0; i < kMaxBlocksPerThread; ++i)
+            cnt += __popc(blk[i].x) + __popc(blk[i].y) + __popc(blk[i].z) + __popc(blk[i].w);   // bytes are 0 or 1
+        for (int i = kMaxBlocksPerThread; i < bpt && q0 + i < nblk; ++i) {
+            const uint4 v = __ldcg(kb + q0 + i);
+            cnt += __popc(v.x) + __popc(v.y) + __popc(v.z) + __popc(v.w);
+        }
+        // block-wide exclusive scan of the counts
+        int incl = cnt;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int v = __shfl_up_sync(0xffffffffu, incl, o);
@@ -580,52 +657,56 @@ __device__ void compact_indices(const FusedParams &p, Shared<BT> &S, int *prefix
         }
         if (lane == 31) S.warp_sums[warp] = incl;
         __syncthreads();
-        int base = 0;
-        for (int w = 0; w < warp; ++w) base += S.warp_sums[w];
-        int run = base + incl - local;
-        for (int c = c0; c < c1; ++c) {
-            prefix[c] = run;
-            run += __ldcg(p.chunk_cnt + c * kMaxTokensPerPass + b);
+        int base = 0, total = 0;
+        for (int w = 0; w < kThreads / 32; ++w) {
+            if (w < warp) base += S.warp_sums[w];
+            total += S.warp_sums[w];
         }
-        if (blockIdx.x == 0 && tid == kThreads - 1) {
-            int tot = 0;
-            for (int w = 0; w < nw; ++w) tot += S.warp_sums[w];
-            if (p.active_cnt) p.active_cnt[b] = tot;
+        int pos = base + incl - cnt;
+        int32_t *dst = p.active_idx + (size_t)b * N;
+        for (int i = 0; i < bpt && q0 + i < nblk; ++i) {
+            const uint4 v = i < kMaxBlocksPerThread ? blk[i] : __ldcg(kb + q0 + i);
+            const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+            const int nbase = (q0 + i) * 16;
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if ((w4[j] >> (8 * e)) & 0xffu) dst[pos++] = nbase + 4 * j + e;
         }
-        __syncthreads();
-        // copy this CTA's chunks (c = blockIdx.x + k * gridDim.x)
-        const int slots = kThreads / kChunk;   // chunks per sweep
-        for (int s0 = 0;; s0 += slots) {
-            if (blockIdx.x + s0 * gridDim.x >= nc) break;
-            const int c = blockIdx.x + (s0 + tid / kChunk) * gridDim.x;
-            const int k = tid % kChunk;
-            if (c < nc && tid < slots * kChunk) {
-                const int cnt = __ldcg(p.chunk_cnt + c * kMaxTokensPerPass + b);
-                if (k < cnt)
-                    p.active_idx[(size_t)b * p.N + prefix[c] + k] = __ldcg(p.idx_tmp + b * stride + c * kChunk + k);
-            }
-        }
+        if (tid == 0 && p.active_cnt) p.active_cnt[b] = total;
         __syncthreads();
     }
 }
 
 template <int BT, int VPT>
-__global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParams p, int look)
+__global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParams p)
 {
     extern __shared__ __align__(128) uint8_t smem[];
-    uint8_t *stages = smem;
-    Shared<BT> &S = *reinterpret_cast<Shared<BT> *>(smem + (size_t)kStages * kStageBytes);
+    uint8_t *gring = smem;
+    uint8_t *uring = smem + (size_t)kGateStages * kGateStageBytes;
+    Shared<BT> &S = *reinterpret_cast<Shared<BT> *>(uring + kUdRingBytes);
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
 
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) {
-            mbar_init(&S.full[s], 1);
-            mbar_init(&S.empty[s], kConsumerWarps);
-            S.issued[s] = 0;
+        for (int s = 0; s < kGateStages; ++s) {
+            mbar_init(&S.gfull[s], 1);
+            mbar_init(&S.gempty[s], kGateWarps);
+            S.gissued[s] = 0;
         }
-        for (int b = 0; b < kBufs; ++b) mbar_init(&S.gsync[b], kConsumerWarps);
-        mbar_init(&S.csync, kConsumerWarps);
+        for (int s = 0; s < kUdSlots; ++s) {
+            mbar_init(&S.ufull[s], 1);
+            mbar_init(&S.uempty[s], kUdWarps);
+            S.uissued[s] = 0;
+        }
+        for (int b = 0; b < kBufs; ++b) {
+            mbar_init(&S.gsync[b], kGateWarps);
+            mbar_init(&S.bfree[b], 1);
+        }
+        mbar_init(&S.xloaded, kGateWarps + kUdWarps);
+        mbar_init(&S.gbar, kGateWarps);
+        mbar_init(&S.ubar, kUdWarps);
         S.abort = 0;
         mbar_init_fence();
     }
@@ -634,41 +715,77 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
         if (tid < p.nb) t = (p.dense_flags && p.dense_flags[tid]) ? 0.f : p.t_l;
         S.thr[tid] = t;
     }
+    if (p.out_mode == kOutY) {
+        // zero this CTA's slice of y; every CTA adds into y only after all
+        // CTAs have passed this point (kCtlPrologue)
+        const int total4 = p.nb * (p.H >> 2);
+        const int per = (total4 + gridDim.x - 1) / gridDim.x;
+        const int q1 = min(total4, (int)(blockIdx.x + 1) * per);
+        for (int q = blockIdx.x * per + tid; q < q1; q += kThreads)
+            reinterpret_cast<float4 *>(p.out)[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     __syncthreads();
 
     f32x2 yp[BT][VPT][4];
-    if (warp == kConsumerWarps) {
-        producer<BT>(p, S, stages, look, lane);
-        if (lane == 0 && S.abort) drain_copies<BT>(S);
+    if (warp < kGateWarps) {
+        gate_warps<BT, VPT>(p, S, gring);
+    } else if (warp < kGateProducerWarp) {
+        updown_warps<BT, VPT>(p, S, uring, yp);
+    } else if (warp == kGateProducerWarp) {
+        if (lane == 0) gate_producer<BT>(p, S, gring);
         __syncwarp();
     } else {
-        consumer<BT, VPT>(p, S, stages, yp);
-        // y partial of this CTA: partials[blockIdx.x][b][:]
+        list_producer<BT>(p, S, uring, lane);
+    }
+    __syncthreads();
+    if (tid == 0 && S.abort) drain_copies<BT>(S);
+
+    // add this CTA's partial y into the output, once every CTA has read its
+    // activations (and zeroed its slice of y)
+    __shared__ int go_s;
+    if (tid == 0) go_s = wait_prologues(p.ctl) ? 1 : 0;
+    __syncthreads();
+    if (go_s && warp >= kGateWarps && warp < kGateProducerWarp) {
+        const int t = tid - kGateThreads;
         const int HV = p.H >> 3;
 #pragma unroll
         for (int b = 0; b < BT; ++b) {
             if (b >= p.nb) break;
 #pragma unroll
             for (int i = 0; i < VPT; ++i) {
-                const int v = tid + i * kConsumers;
+                const int v = t + i * kUdThreads;
                 if (v < HV) {
-                    float4 *dst = reinterpret_cast<float4 *>(
-                        p.partials + ((size_t)blockIdx.x * kMaxTokensPerPass + b) * p.H + (size_t)v * 8);
+                    float *dst = p.out + (size_t)b * p.H + (size_t)v * 8;
                     const float2 y0 = unpack2(yp[b][i][0]), y1 = unpack2(yp[b][i][1]);
                     const float2 y2 = unpack2(yp[b][i][2]), y3 = unpack2(yp[b][i][3]);
-                    dst[0] = make_float4(y0.x, y0.y, y1.x, y1.y);
-                    dst[1] = make_float4(y2.x, y2.y, y3.x, y3.y);
+                    red_add_v4(dst, y0.x, y0.y, y1.x, y1.y);
+                    red_add_v4(dst + 4, y2.x, y2.y, y3.x, y3.y);
                 }
             }
         }
     }
-    if (!grid_barrier(p.ctl)) return;
-    reduce_partials(p);
-    if (p.active_idx && !S.abort) compact_indices<BT>(p, S, reinterpret_cast<int *>(stages));
+    __syncthreads();
+    __shared__ int last_s;
+    if (tid == 0) {
+        __threadfence();
+        last_s = atomicAdd(p.ctl + kCtlDone, 1) == (int)gridDim.x - 1;
+        __threadfence();
+    }
+    __syncthreads();
+    if (last_s) {
+        // every other CTA has added its y, written its keep bytes and is past
+        // its wait on kCtlPrologue
+        if (p.active_idx && !S.abort) compact_indices<BT>(p, S);
+        if (tid == 0) {
+            atomicExch(p.ctl + kCtlPrologue, 0);
+            atomicExch(p.ctl + kCtlPool, 0);
+            atomicExch(p.ctl + kCtlDone, 0);
+        }
+    }
 }
 
 template <int BT, int VPT>
-cudaError_t launch_t(const FusedParams &p, int grid, int look, cudaStream_t stream)
+cudaError_t launch_t(const FusedParams &p, int grid, cudaStream_t stream)
 {
     static unsigned long long configured = 0;   // one bit per device ordinal
     const size_t smem = smem_bytes<BT>();
@@ -691,7 +808,7 @@ cudaError_t launch_t(const FusedParams &p, int grid, int look, cudaStream_t stre
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, fused_mlp_kernel<BT, VPT>, p, look);
+    return cudaLaunchKernelEx(&cfg, fused_mlp_kernel<BT, VPT>, p);
 }
 
 }  // namespace
@@ -708,24 +825,25 @@ int fused_grid(int nchunks)
     return g < 1 ? 1 : g;
 }
 
-// 16-byte vectors per consumer thread and row: ceil(H / 8 / 512).
-static int fused_vectors_per_thread(int H) { return H <= 4096 ? 1 : 2; }
+// 16-byte vectors per gate or up/down thread and row: ceil(H / 8 / 256).
+static int fused_vectors_per_thread(int H) { return H <= 2048 ? 1 : (H <= 4096 ? 2 : 4); }
 
-int fused_tokens_per_pass(int H) { return fused_vectors_per_thread(H) == 1 ? 2 : 1; }
+int fused_tokens_per_pass(int H) { return fused_vectors_per_thread(H) == 4 ? 1 : 2; }
 
 cudaError_t launch_fused(const FusedParams &p, cudaStream_t stream)
 {
     const int grid = fused_grid(p.nchunks);
-    // chunks of gate rows kept in flight ahead of the W_ud rows: about 128 KB
-    int look = (128 * 1024) / (kChunk * 2 * p.H);
-    look = look < 1 ? 1 : (look > kMaxLook ? kMaxLook : look);
     const int vpt = fused_vectors_per_thread(p.H);
     if (p.nb < 1 || p.nb > fused_tokens_per_pass(p.H)) return cudaErrorInvalidValue;
     if (vpt == 1) {
-        if (p.nb <= 1) return launch_t<1, 1>(p, grid, look, stream);
-        return launch_t<2, 1>(p, grid, look, stream);
+        if (p.nb <= 1) return launch_t<1, 1>(p, grid, stream);
+        return launch_t<2, 1>(p, grid, stream);
     }
-    return launch_t<1, 2>(p, grid, look, stream);
+    if (vpt == 2) {
+        if (p.nb <= 1) return launch_t<1, 2>(p, grid, stream);
+        return launch_t<2, 2>(p, grid, stream);
+    }
+    return launch_t<1, 4>(p, grid, stream);
 }
 
 }  // namespace sats

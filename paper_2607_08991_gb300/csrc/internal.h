@@ -25,11 +25,14 @@ constexpr int kMaxN = 1 << 20;
 
 // Control block at the start of the workspace (ints).
 enum {
-    kCtlChunk = 0,      // dynamic chunk counter, reset to 0 by the grid barrier
+    kCtlChunk = 0,      // reserved
     kCtlBarCount = 1,   // grid barrier arrivals, reset to 0 by the last arrival
     kCtlBarGen = 2,     // grid barrier generation
     kCtlStatus = 3,     // device status word (kStatus* bits)
     kCtlNDense = 4,     // route output of the stack driver
+    kCtlPrologue = 5,   // CTAs that have read their activations (reset by the last CTA)
+    kCtlDone = 6,       // CTAs that have added their partial y (reset by the last CTA)
+    kCtlPool = 7,       // next chunk of the shared tail pool (reset by the last CTA)
     kCtlInts = 64
 };
 
@@ -56,8 +59,8 @@ struct FusedParams {
     float *out;                   // kOutY: y [nb][H]; kOutResid: residual [nb][H] (+=)
     int *ctl;                     // workspace control block
     float *partials;              // [kMaxGrid][kMaxTokensPerPass][H]
-    int *chunk_cnt;               // [nchunks][kMaxTokensPerPass]
-    int *idx_tmp;                 // [kMaxTokensPerPass][nchunks * kChunk]
+    int *chunk_cnt;               // unused
+    uint8_t *keep_tmp;            // [kMaxTokensPerPass][N]: keep byte per neuron (index output only)
     int32_t *active_idx;          // [nb][N] or nullptr
     int32_t *active_cnt;          // [nb] or nullptr
     uint8_t *keep_trace;          // [nb][N] or nullptr
