@@ -624,7 +624,7 @@ __device__ bool wait_prologues(int *ctl)
 // The ascending per-token kept lists from the keep bytes of all chunks; run by
 // the last CTA to finish, when every chunk's bytes are in memory.
 template <int BT>
-__device__ void compact_indices(const FusedParams &p, Shared<BT> &S)
+__device__ void compact_indices(const FusedParams &p, Shared<BT> &S, int *stage_buf, int stage_cap)
 {
     constexpr int kMaxBlocksPerThread = 8;                  // 16 keep bytes per block
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -663,7 +663,11 @@ __device__ void compact_indices(const FusedParams &p, Shared<BT> &S)
             total += S.warp_sums[w];
         }
         int pos = base + incl - cnt;
+        // the list is assembled in shared memory (the idle rings) and then
+        // written with coalesced stores; a list too long for it goes straight out
+        const bool staged = total <= stage_cap;
         int32_t *dst = p.active_idx + (size_t)b * N;
+        int32_t *out = staged ? stage_buf : dst;
         for (int i = 0; i < bpt && q0 + i < nblk; ++i) {
             const uint4 v = i < kMaxBlocksPerThread ? blk[i] : __ldcg(kb + q0 + i);
             const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
@@ -672,10 +676,14 @@ __device__ void compact_indices(const FusedParams &p, Shared<BT> &S)
             for (int j = 0; j < 4; ++j)
 #pragma unroll
                 for (int e = 0; e < 4; ++e)
-                    if ((w4[j] >> (8 * e)) & 0xffu) dst[pos++] = nbase + 4 * j + e;
+                    if ((w4[j] >> (8 * e)) & 0xffu) out[pos++] = nbase + 4 * j + e;
         }
         if (tid == 0 && p.active_cnt) p.active_cnt[b] = total;
         __syncthreads();
+        if (staged) {
+            for (int i = tid; i < total; i += kThreads) dst[i] = stage_buf[i];
+            __syncthreads();
+        }
     }
 }
 
@@ -775,7 +783,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
     if (last_s) {
         // every other CTA has added its y, written its keep bytes and is past
         // its wait on kCtlPrologue
-        if (p.active_idx && !S.abort) compact_indices<BT>(p, S);
+        if (p.active_idx && !S.abort)
+            compact_indices<BT>(p, S, reinterpret_cast<int *>(smem),
+                                (kGateStages * kGateStageBytes + kUdRingBytes) / (int)sizeof(int));
         if (tid == 0) {
             atomicExch(p.ctl + kCtlPrologue, 0);
             atomicExch(p.ctl + kCtlPool, 0);
