@@ -254,8 +254,6 @@ def run_gpu(args):
         for si, t in calls:
             one_call(si, t)
     K = args.steps
-    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in calls]
-           for _ in range(K)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = Clocks(local)
     if world > 1:
@@ -263,12 +261,25 @@ def run_gpu(args):
     torch.cuda.synchronize(dev)
     clocks.start()
     time.sleep(0.3)
+    # timed region: K steps, each the three calls back to back (launches overlap
+    # their prologue with the previous call's tail)
     start.record(stream)
     for k in range(K):
-        for (si, t), (e0, e1) in zip(calls, evs[k]):
-            one_call(si, t, e0, e1)
+        for si, t in calls:
+            one_call(si, t)
     stop.record(stream)
     stop.synchronize()
+    # average launch duration per sparsity level: K launches of that level back
+    # to back on the same stream, bracketed by events
+    mean_us = []
+    for si, t in calls:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for k in range(K):
+            one_call(si, t)
+        e1.record(stream)
+        e1.synchronize()
+        mean_us.append(1e3 * e0.elapsed_time(e1) / K)
     torch.cuda.synchronize(dev)
     if world > 1:
         dist.barrier()
@@ -277,8 +288,6 @@ def run_gpu(args):
     if status != sats.OK:
         raise RuntimeError("device status after the timed region: " + sats.status_string(status))
     total_ms = start.elapsed_time(stop)
-    per_call_us = [[1e3 * evs[k][i][0].elapsed_time(evs[k][i][1]) for k in range(K)] for i in range(len(calls))]
-    mean_us = [sum(v) / len(v) for v in per_call_us]
 
     if args.profile:
         if rank == 0:
@@ -288,16 +297,15 @@ def run_gpu(args):
         return
 
     # dense path on the same copies, for the speedup
-    dense_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    for i in range(3 + K):
-        layer = layers[i % len(layers)]
-        if i >= 3:
-            dense_ev[i - 3][0].record(stream)
-        sats.dense_mlp(layer, x, y, ws, stream=stream)
-        if i >= 3:
-            dense_ev[i - 3][1].record(stream)
-    stream.synchronize()
-    dense_us = 1e3 * sum(a.elapsed_time(b) for a, b in dense_ev) / K
+    for i in range(3):
+        sats.dense_mlp(layers[i % len(layers)], x, y, ws, stream=stream)
+    d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    d0.record(stream)
+    for i in range(K):
+        sats.dense_mlp(layers[i % len(layers)], x, y, ws, stream=stream)
+    d1.record(stream)
+    d1.synchronize()
+    dense_us = 1e3 * d0.elapsed_time(d1) / K
 
     # end to end through the C ABI with host buffers: x host->device, y and count device->host
     xh = torch.from_numpy(inputs.activations_bf16(1, H).view(np.int16)).pin_memory()

@@ -229,7 +229,13 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
     const int nb0 = (int)((long long)blockIdx.x * N / gridDim.x);
     const int nb1 = (int)((long long)(blockIdx.x + 1) * N / gridDim.x);
     const int own = max(0, (nb1 - nb0 + kChunk - 1) / kChunk - kPoolChunksPerCta);
-    int next_k = own == 0 ? atomicAdd(p.ctl + kCtlPool, 1) : -1;   // a claimed, not yet used pool chunk
+    int next_k = -1;   // a claimed, not yet used pool chunk
+    bool waited = false;   // the workspace's pool counter is used only after the previous grid ended
+    if (own == 0) {
+        grid_dependency_wait();
+        waited = true;
+        next_k = atomicAdd(p.ctl + kCtlPool, 1);
+    }
     uint32_t stage = 0, phase = 0;
     bool ok = true;
     for (int seq = 0;; ++seq) {
@@ -241,7 +247,10 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
             n0 = nb0 + seq * kChunk;
             end = nb1;
             // claim the first pool chunk while the own chunks still stream
-            if (seq + 1 == own && next_k < 0) next_k = atomicAdd(p.ctl + kCtlPool, 1);
+            if (seq + 1 == own && next_k < 0) {
+                if (!waited) { grid_dependency_wait(); waited = true; }
+                next_k = atomicAdd(p.ctl + kCtlPool, 1);
+            }
         } else {
             // pool chunk k: chunk (own_c + k % P) of CTA k / P's range; the
             // next claim is issued before this chunk's rows are streamed
@@ -305,6 +314,7 @@ __device__ void gate_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *g
     const uint4 zero4 = make_uint4(0u, 0u, 0u, 0u);
     GroupSync gs{&S.gbar, 0u};
     f32x2 xp[BT][VPT][4];
+    grid_dependency_wait();   // x may be the previous launch's output
     const bool loaded = load_activations<BT, VPT>(p, S, gs, t, kGateThreads, 0, xp);
     __syncwarp();
     if (lane == 0) mbar_arrive(&S.xloaded);
@@ -407,7 +417,18 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
     const UdGeometry geo(H);
     const uint32_t lt = (1u << lane) - 1u;
     uint32_t stage = 0, phase = 0;
+    grid_dependency_wait();   // the workspace and y belong to the previous launch until it ends
+    if (p.out_mode == kOutY) {
+        // zero this CTA's slice of y; every CTA adds into y only after all
+        // CTAs have passed their prologue (kCtlPrologue)
+        const int total4 = p.nb * (p.H >> 2);
+        const int per = (total4 + gridDim.x - 1) / gridDim.x;
+        const int q1 = min(total4, (int)(blockIdx.x + 1) * per);
+        for (int q = blockIdx.x * per + lane; q < q1; q += 32)
+            reinterpret_cast<float4 *>(p.out)[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     bool ok = mbar_wait(&S.xloaded, 0u, &S.abort);
+    __syncwarp();
     if (ok && lane == 0) {
         // this CTA has read its activations and zeroed its slice of y
         __threadfence();
@@ -520,6 +541,7 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
 #pragma unroll
             for (int e = 0; e < 4; ++e) yp[b][i][e] = 0ull;
     f32x2 xp[BT][VPT][4];
+    grid_dependency_wait();
     const bool loaded = load_activations<BT, VPT>(p, S, us, t, kUdThreads, kGateWarps, xp);
     __syncwarp();
     if (lane == 0) mbar_arrive(&S.xloaded);
@@ -723,16 +745,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
         if (tid < p.nb) t = (p.dense_flags && p.dense_flags[tid]) ? 0.f : p.t_l;
         S.thr[tid] = t;
     }
-    if (p.out_mode == kOutY) {
-        // zero this CTA's slice of y; every CTA adds into y only after all
-        // CTAs have passed this point (kCtlPrologue)
-        const int total4 = p.nb * (p.H >> 2);
-        const int per = (total4 + gridDim.x - 1) / gridDim.x;
-        const int q1 = min(total4, (int)(blockIdx.x + 1) * per);
-        for (int q = blockIdx.x * per + tid; q < q1; q += kThreads)
-            reinterpret_cast<float4 *>(p.out)[q] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
     __syncthreads();
+    // the next launch in the stream may start its weight stream on SMs this
+    // grid frees; it waits for this grid's end before touching x, y or the workspace
+    grid_launch_dependents();
 
     f32x2 yp[BT][VPT][4];
     if (warp < kGateWarps) {
@@ -814,8 +830,8 @@ cudaError_t launch_t(const FusedParams &p, int grid, cudaStream_t stream)
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeCooperative;
-    attr[0].val.cooperative = 1;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, fused_mlp_kernel<BT, VPT>, p);
