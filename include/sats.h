@@ -88,8 +88,9 @@ SATS_API sats_status sats_layer_shape(const sats_layer *layer, int *H, int *N);
 /*
  * Workspace.  Every compute call takes a device workspace `ws` of at least
  * sats_workspace_bytes(H, N, B) bytes (B = the largest batch the caller will
- * pass).  It holds cross-block partial sums, scheduling counters, the
- * compacted per-chunk index lists and the device status word.  It must be
+ * pass).  It holds scheduling counters, the device status word, one keep
+ * byte per neuron and token (for the index outputs) and the routing scratch of
+ * sats_mlp_stack; it is small (N * 4 bytes plus B * 5 plus 1 KB).  It must be
  * zero-filled once before first use (sats_workspace_init does that on
  * `stream`); every call leaves its counters at zero for the next call.  Calls
  * that share one workspace must not overlap on the GPU.

@@ -16,17 +16,13 @@ static int nchunks_of(int N) { return (N + kChunk - 1) / kChunk; }
 
 WsLayout ws_layout(int H, int N, int B)
 {
+    (void)H;
     WsLayout L{};
-    const size_t nc = (size_t)nchunks_of(N);
     size_t off = 0;
     L.ctl = off;
     off += align256(kCtlInts * sizeof(int));
-    L.partials = off;
-    off += align256((size_t)kMaxGrid * kMaxTokensPerPass * H * sizeof(float));
-    L.chunk_cnt = off;   // per-CTA kept counts
-    off += align256((size_t)kMaxGrid * kMaxTokensPerPass * sizeof(int));
-    L.idx_tmp = off;
-    off += align256((size_t)kMaxTokensPerPass * nc * kChunk * sizeof(int));
+    L.keep = off;   // one keep byte per neuron and token of a pass, rows padded to 16 bytes
+    off += align256((size_t)kMaxTokensPerPass * (((size_t)N + 15) & ~(size_t)15));
     L.route_perm = off;
     off += align256((size_t)(B > 0 ? B : 1) * sizeof(int32_t));
     L.route_flags = off;
@@ -69,9 +65,7 @@ static sats_status run_layer(const sats_layer *layer, int x_mode, const void *x,
         p.out_mode = out_mode;
         p.out = out + (size_t)b0 * H;
         p.ctl = reinterpret_cast<int *>(base + L.ctl);
-        p.partials = reinterpret_cast<float *>(base + L.partials);
-        p.chunk_cnt = reinterpret_cast<int *>(base + L.chunk_cnt);
-        p.keep_tmp = reinterpret_cast<uint8_t *>(base + L.idx_tmp);
+        p.keep_tmp = reinterpret_cast<uint8_t *>(base + L.keep);
         p.active_idx = active_idx ? active_idx + (size_t)b0 * N : nullptr;
         p.active_cnt = active_cnt ? active_cnt + b0 : nullptr;
         p.keep_trace = keep_trace ? keep_trace + (size_t)b0 * N : nullptr;

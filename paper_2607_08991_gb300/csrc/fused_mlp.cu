@@ -374,6 +374,24 @@ __device__ void gate_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *g
 // Row stride of the keep bytes (16-byte aligned rows, so they load as uint4).
 __device__ __forceinline__ int keep_stride(int N) { return (N + 15) & ~15; }
 
+// The 16 keep bytes of block q with the bytes of neurons >= N cleared: the
+// padding at the end of a row is never written and holds stale data.
+__device__ __forceinline__ uint4 keep_block(const uint4 *row, int q, int N)
+{
+    uint4 v = __ldcg(row + q);
+    const int valid = N - 16 * q;
+    if (valid < 16) {
+        uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int c = min(4, max(0, valid - 4 * j));
+            w[j] &= c == 4 ? 0xffffffffu : ((1u << (8 * c)) - 1u);
+        }
+        v = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+    return v;
+}
+
 // ------------------------------------------------------------------ list producer
 // Lane r = row r of the chunk: sums the gate partials across the gate warps,
 // SiLU (Eq. 2), CATS mask (Eqs. 4-5) per token, index outputs.  Returns the
@@ -661,13 +679,13 @@ __device__ void compact_indices(const FusedParams &p, Shared<BT> &S, int *stage_
         int cnt = 0;
 #pragma unroll
         for (int i = 0; i < kMaxBlocksPerThread; ++i) {
-            blk[i] = (i < bpt && q0 + i < nblk) ? __ldcg(kb + q0 + i) : make_uint4(0u, 0u, 0u, 0u);
+            blk[i] = (i < bpt && q0 + i < nblk) ? keep_block(kb, q0 + i, N) : make_uint4(0u, 0u, 0u, 0u);
         }
 #pragma unroll
         for (int i = 0; i < kMaxBlocksPerThread; ++i)
             cnt += __popc(blk[i].x) + __popc(blk[i].y) + __popc(blk[i].z) + __popc(blk[i].w);   // bytes are 0 or 1
         for (int i = kMaxBlocksPerThread; i < bpt && q0 + i < nblk; ++i) {
-            const uint4 v = __ldcg(kb + q0 + i);
+            const uint4 v = keep_block(kb, q0 + i, N);
             cnt += __popc(v.x) + __popc(v.y) + __popc(v.z) + __popc(v.w);
         }
         // block-wide exclusive scan of the counts
@@ -691,7 +709,7 @@ __device__ void compact_indices(const FusedParams &p, Shared<BT> &S, int *stage_
         int32_t *dst = p.active_idx + (size_t)b * N;
         int32_t *out = staged ? stage_buf : dst;
         for (int i = 0; i < bpt && q0 + i < nblk; ++i) {
-            const uint4 v = i < kMaxBlocksPerThread ? blk[i] : __ldcg(kb + q0 + i);
+            const uint4 v = i < kMaxBlocksPerThread ? blk[i] : keep_block(kb, q0 + i, N);
             const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
             const int nbase = (q0 + i) * 16;
 #pragma unroll

@@ -19,7 +19,7 @@ namespace sats {
 
 constexpr int kChunk = 8;               // neurons per scheduling unit of the fused kernel
 constexpr int kMaxTokensPerPass = 4;    // tokens one fused launch carries
-constexpr int kMaxGrid = 256;           // upper bound of the fused grid (partials rows)
+constexpr int kMaxGrid = 256;           // upper bound of the fused grid
 constexpr int kMaxH = 8192;
 constexpr int kMaxN = 1 << 20;
 
@@ -37,7 +37,7 @@ enum {
 };
 
 struct WsLayout {
-    size_t ctl, partials, chunk_cnt, idx_tmp, route_perm, route_flags, total;
+    size_t ctl, keep, route_perm, route_flags, total;
 };
 WsLayout ws_layout(int H, int N, int B);
 
@@ -58,8 +58,6 @@ struct FusedParams {
     int out_mode;
     float *out;                   // kOutY: y [nb][H]; kOutResid: residual [nb][H] (+=)
     int *ctl;                     // workspace control block
-    float *partials;              // [kMaxGrid][kMaxTokensPerPass][H]
-    int *chunk_cnt;               // unused
     uint8_t *keep_tmp;            // [kMaxTokensPerPass][N]: keep byte per neuron (index output only)
     int32_t *active_idx;          // [nb][N] or nullptr
     int32_t *active_cnt;          // [nb] or nullptr

@@ -66,11 +66,11 @@ def lib() -> ctypes.CDLL:
 
 
 def exported_symbols() -> Sequence[str]:
-    return [n for n in ("sats_version", "sats_status_string", "sats_layer_create", "sats_layer_destroy",
-                        "sats_layer_shape", "sats_workspace_bytes", "sats_workspace_init", "sats_sparse_mlp",
-                        "sats_sparse_mlp_f32", "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
-                        "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_get_error",
-                        "sats_get_status_word")]
+    """Every C entry point this binding forwards to."""
+    return ("sats_version", "sats_status_string", "sats_layer_create", "sats_layer_destroy", "sats_layer_shape",
+            "sats_workspace_bytes", "sats_workspace_init", "sats_sparse_mlp", "sats_sparse_mlp_f32",
+            "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
+            "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_get_error", "sats_get_status_word")
 
 
 def status_string(s: int) -> str:

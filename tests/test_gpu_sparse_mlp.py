@@ -156,7 +156,7 @@ def test_repeat_calls_agree(sats):
 
 
 def test_argument_errors(sats):
-    H, N = 64, 64
+    H, N = 64, 4096
     w = inputs.mlp_weights(H, N)
     layer = sats.Layer(P.dev_u16(w.Wg), P.dev_u16(w.Wu), P.dev_u16(w.Wd))
     ws = sats.Workspace(H, N, 1)
