@@ -117,6 +117,34 @@ SATS_API sats_status sats_sparse_mlp(const sats_layer *layer, const void *x, int
                             float *y, int32_t *active_idx, int32_t *active_cnt,
                             void *ws, size_t ws_bytes, void *stream);
 
+/*
+ * sats_sparse_mlp_fixed_scratch -- sats_sparse_mlp with no workspace argument,
+ * for callers that cannot allocate device memory.  The paper has no
+ * counterpart to this call.  Such callers include plug-ins whose host
+ * application owns every device allocation through its own allocator, code
+ * that runs where cudaMalloc is not permitted or would stall (it synchronises
+ * the device), and plain C callers that link only this library and have no
+ * device allocator at all.
+ *
+ * Arguments, results and errors are those of sats_sparse_mlp.  Instead of a
+ * workspace the call uses one 1 MiB array in the library's device memory; every
+ * GPU that loads the library holds this array until the process exits.  A
+ * shape whose workspace (sats_workspace_bytes(H, N, B)) exceeds 1 MiB is
+ * rejected with SATS_ENOSPACE; with four keep bytes per neuron that admits
+ * N up to about 260,000.  The call allocates nothing: before its kernel it
+ * clears the array's control words with cudaMemsetAsync on `stream`.
+ *
+ * The first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress); make that first call before any stream capture.
+ * All calls share the one array, so calls that can overlap on the GPU (on
+ * different streams, or from several host threads without ordering) race and
+ * must be serialised by the caller.  Device-side errors of this call (a
+ * bounded wait that gave up) are not reported.
+ */
+SATS_API sats_status sats_sparse_mlp_fixed_scratch(const sats_layer *layer, const void *x, int B, float t_l,
+                                                   float *y, int32_t *active_idx, int32_t *active_cnt,
+                                                   void *stream);
+
 /* As sats_sparse_mlp, with fp32 activations x: device fp32 [B][H]. */
 SATS_API sats_status sats_sparse_mlp_f32(const sats_layer *layer, const float *x, int B, float t_l,
                                 float *y, int32_t *active_idx, int32_t *active_cnt,

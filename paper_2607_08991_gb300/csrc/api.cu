@@ -3,6 +3,7 @@
 // of the fused kernel and chain the blocks of a stack.
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <new>
 
 #include "common.cuh"
@@ -97,6 +98,32 @@ static sats_status sparse_common(const sats_layer *layer, int x_mode, const void
                      ws, static_cast<cudaStream_t>(stream));
 }
 
+// ---------------------------------------------------------------------------
+// Fixed scratch for sats_sparse_mlp_fixed_scratch: one array in this file's
+// device memory, present on every GPU that loads the library until the
+// process exits.  Host code cannot use the symbol itself as a device address;
+// the address is looked up per device with cudaGetSymbolAddress.
+constexpr size_t kFixedScratchBytes = (size_t)1 << 20;   // 1 MiB
+static __device__ __align__(256) unsigned char g_fixed_scratch[kFixedScratchBytes];
+
+static std::mutex g_fixed_scratch_mu;
+static void *g_fixed_scratch_ptr[64] = {};
+
+// Device address of g_fixed_scratch on the current device (looked up on the
+// first call for that device), or nullptr on failure.
+static void *fixed_scratch_current_device()
+{
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(g_fixed_scratch_mu);
+    if (!g_fixed_scratch_ptr[dev]) {
+        void *ptr = nullptr;
+        if (cudaGetSymbolAddress(&ptr, g_fixed_scratch) != cudaSuccess || !ptr) return nullptr;
+        g_fixed_scratch_ptr[dev] = ptr;
+    }
+    return g_fixed_scratch_ptr[dev];
+}
+
 }  // namespace sats
 
 using namespace sats;
@@ -182,6 +209,24 @@ sats_status sats_sparse_mlp(const sats_layer *layer, const void *x, int B, float
                             int32_t *active_cnt, void *ws, size_t ws_bytes, void *stream)
 {
     return sparse_common(layer, kXBf16, x, B, t_l, y, active_idx, active_cnt, ws, ws_bytes, stream);
+}
+
+sats_status sats_sparse_mlp_fixed_scratch(const sats_layer *layer, const void *x, int B, float t_l, float *y,
+                                          int32_t *active_idx, int32_t *active_cnt, void *stream)
+{
+    if (!layer || B < 0) return SATS_EINVAL;
+    if (ws_layout(layer->H, layer->N, B).total > kFixedScratchBytes) return SATS_ENOSPACE;
+    if (bad_threshold(t_l)) return SATS_EINVAL;
+    if ((active_idx == nullptr) != (active_cnt == nullptr)) return SATS_EINVAL;
+    if (B == 0) return SATS_OK;
+    if (!x || !y || !aligned16(x) || !aligned16(y)) return SATS_EINVAL;
+    void *ws = fixed_scratch_current_device();
+    if (!ws) return SATS_ECUDA;
+    // the array keeps the previous call's contents: the control words
+    // (scheduling counters, status) must start at zero
+    if (cudaMemsetAsync(ws, 0, kCtlInts * sizeof(int), static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return SATS_ECUDA;
+    return sparse_common(layer, kXBf16, x, B, t_l, y, active_idx, active_cnt, ws, kFixedScratchBytes, stream);
 }
 
 sats_status sats_sparse_mlp_f32(const sats_layer *layer, const float *x, int B, float t_l, float *y,

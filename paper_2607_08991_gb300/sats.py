@@ -48,6 +48,7 @@ def lib() -> ctypes.CDLL:
             "sats_workspace_init": (I, [P, Z, P]),
             "sats_sparse_mlp": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_sparse_mlp_f32": (I, [P, P, I, F, P, P, P, P, Z, P]),
+            "sats_sparse_mlp_fixed_scratch": (I, [P, P, I, F, P, P, P, P]),
             "sats_dense_mlp": (I, [P, P, I, P, P, Z, P]),
             "sats_route": (I, [P, I, P, I, P, P, P, P]),
             "sats_mlp_stack": (I, [P, P, P, I, F, P, P, I, P, I, P, P, Z, P]),
@@ -69,7 +70,7 @@ def exported_symbols() -> Sequence[str]:
     """Every C entry point this binding forwards to."""
     return ("sats_version", "sats_status_string", "sats_layer_create", "sats_layer_destroy", "sats_layer_shape",
             "sats_workspace_bytes", "sats_workspace_init", "sats_sparse_mlp", "sats_sparse_mlp_f32",
-            "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
+            "sats_sparse_mlp_fixed_scratch", "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
             "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_get_error", "sats_get_status_word")
 
 
@@ -161,6 +162,16 @@ def sparse_mlp_f32(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor, w
     _check(lib().sats_sparse_mlp_f32(layer.handle, _ptr(x, "x", 4), B, float(t_l), _ptr(y, "y", 4),
                                      _ptr(active_idx, "active_idx", 4), _ptr(active_cnt, "active_cnt", 4),
                                      ws.ptr, ws.nbytes, _stream(stream)), "sats_sparse_mlp_f32")
+
+
+def sparse_mlp_fixed_scratch(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor,
+                             active_idx: Optional[torch.Tensor] = None, active_cnt: Optional[torch.Tensor] = None,
+                             stream: Optional[torch.cuda.Stream] = None):
+    """sats_sparse_mlp without a workspace (the library's fixed 1 MiB device scratch)."""
+    B = x.shape[0]
+    _check(lib().sats_sparse_mlp_fixed_scratch(layer.handle, _ptr(x, "x", 2), B, float(t_l), _ptr(y, "y", 4),
+                                               _ptr(active_idx, "active_idx", 4), _ptr(active_cnt, "active_cnt", 4),
+                                               _stream(stream)), "sats_sparse_mlp_fixed_scratch")
 
 
 def dense_mlp(layer: Layer, x: torch.Tensor, y: torch.Tensor, ws: Workspace,
