@@ -90,7 +90,10 @@ SATS_API sats_status sats_layer_shape(const sats_layer *layer, int *H, int *N);
  * sats_workspace_bytes(H, N, B) bytes (B = the largest batch the caller will
  * pass).  It holds scheduling counters, the device status word, one keep
  * byte per neuron and token (for the index outputs) and the routing scratch of
- * sats_mlp_stack; it is small (N * 4 bytes plus B * 5 plus 1 KB).  It must be
+ * sats_mlp_stack: N * 4 bytes plus B * 5 plus 1 KB.  A batch that runs on the
+ * tensor cores (sats_uses_tensor_cores) also needs, per token, bf16 copies of
+ * its activations and of h plus one keep byte per neuron: about
+ * B * (4 H + 3 N) bytes more.  It must be
  * zero-filled once before first use (sats_workspace_init does that on
  * `stream`); every call leaves its counters at zero for the next call.  Calls
  * that share one workspace must not overlap on the GPU.
@@ -101,8 +104,17 @@ SATS_API sats_status sats_workspace_init(void *ws, size_t ws_bytes, void *stream
 /*
  * sats_sparse_mlp -- the CATS-thresholded gated MLP (Sec. 2, Eqs. 1-5):
  *   a = SiLU(x W_gate);  keep_j = |a_j| >= t_l;  y = ((keep * a) * (x W_up)) W_down
- * for each of B tokens, bf16 weights with fp32 accumulation.  Only the
- * W_up columns and W_down rows of kept neurons are read.
+ * for each of B tokens, bf16 weights with fp32 accumulation.
+ *
+ * Two execution paths, chosen by batch size (sats_uses_tensor_cores):
+ *  - small batches (B <= 2 for H <= 4096, B = 1 above) stream W_gate once per
+ *    call and read only the W_up columns and W_down rows of kept neurons;
+ *  - larger batches run as two tensor-core GEMMs over all neurons,
+ *    [x W_gate | x W_up] and then h W_down, with the mask applied to
+ *    h = CATS(SiLU(x W_gate)) * (x W_up) between them; h is rounded to bf16
+ *    there (a relative error of at most 2^-9 per element), and fp32
+ *    activations are split into two bf16 parts so that they keep ~16
+ *    significant bits.
  *   x          : device bf16 [B][H]
  *   t_l        : threshold, >= 0 (0 keeps every neuron: the dense MLP;
  *                +inf keeps none and gives y = 0).  NaN or < 0 -> SATS_EINVAL.
@@ -144,6 +156,14 @@ SATS_API sats_status sats_sparse_mlp(const sats_layer *layer, const void *x, int
 SATS_API sats_status sats_sparse_mlp_fixed_scratch(const sats_layer *layer, const void *x, int B, float t_l,
                                                    float *y, int32_t *active_idx, int32_t *active_cnt,
                                                    void *stream);
+
+/*
+ * sats_uses_tensor_cores -- 1 if a call with batch B on a layer of hidden size
+ * H runs on the tensor-core path described under sats_sparse_mlp (also for
+ * sats_dense_mlp and for each block of sats_mlp_stack), 0 if it runs on the
+ * fused small-batch kernel.  Pure host function.
+ */
+SATS_API int sats_uses_tensor_cores(int H, int B);
 
 /* As sats_sparse_mlp, with fp32 activations x: device fp32 [B][H]. */
 SATS_API sats_status sats_sparse_mlp_f32(const sats_layer *layer, const float *x, int B, float t_l,

@@ -17,7 +17,6 @@ static int nchunks_of(int N) { return (N + kChunk - 1) / kChunk; }
 
 WsLayout ws_layout(int H, int N, int B)
 {
-    (void)H;
     WsLayout L{};
     size_t off = 0;
     L.ctl = off;
@@ -28,6 +27,8 @@ WsLayout ws_layout(int H, int N, int B)
     off += align256((size_t)(B > 0 ? B : 1) * sizeof(int32_t));
     L.route_flags = off;
     off += align256((size_t)(B > 0 ? B : 1));
+    L.tc = off;   // bf16 activations, h and keep bytes of the tensor-core path (batches only)
+    if (use_tc_path(H, B)) off += tc_workspace_bytes(H, N, B);
     L.total = off;
     return L;
 }
@@ -38,7 +39,9 @@ static sats_status from_cuda(cudaError_t e) { return e == cudaSuccess ? SATS_OK 
 
 static bool bad_threshold(float t) { return std::isnan(t) || t < 0.0f; }
 
-// Runs the fused kernel over B tokens in passes of up to 4 (H <= 4096) or 2.
+// Runs one block over B tokens: on the tensor cores when the batch is larger
+// than one pass of the fused kernel, else the fused kernel in passes of
+// fused_tokens_per_pass(H) tokens.
 static sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B, const float *t_per_pass_l,
                              const float *norm_w, float eps, const uint8_t *dense_flags, int out_mode, float *out,
                              int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws,
@@ -47,6 +50,12 @@ static sats_status run_layer(const sats_layer *layer, int x_mode, const void *x,
     const int H = layer->H, N = layer->N;
     const WsLayout L = ws_layout(H, N, B);
     char *base = static_cast<char *>(ws);
+    if (use_tc_path(H, B)) {
+        const cudaError_t e = run_tc_layer(layer, x_mode, x, B, *t_per_pass_l, norm_w, eps, dense_flags, out_mode,
+                                           out, active_idx, active_cnt, keep_trace, base + L.tc,
+                                           reinterpret_cast<int *>(base + L.ctl), stream);
+        return e == cudaSuccess ? SATS_OK : SATS_ECUDA;
+    }
     const int per_pass = fused_tokens_per_pass(H);
     const size_t x_elem = (x_mode == kXBf16) ? 2 : 4;
     for (int b0 = 0; b0 < B; b0 += per_pass) {
@@ -158,16 +167,20 @@ sats_status sats_layer_create(const void *W_gate, const void *W_up, const void *
     l->H = H;
     l->N = N;
     cudaGetDevice(&l->device);
+    l->ldn = (N + 7) & ~7;
     const size_t row_elems = (size_t)N * H;
-    if (cudaMalloc(&l->wg_t, row_elems * 2) != cudaSuccess) { delete l; return SATS_ECUDA; }
-    if (cudaMalloc(&l->w_ud, row_elems * 4) != cudaSuccess) { cudaFree(l->wg_t); delete l; return SATS_ECUDA; }
+    cudaError_t e = cudaMalloc(&l->wg_t, row_elems * 2);
+    if (e == cudaSuccess) e = cudaMalloc(&l->w_ud, row_elems * 4);
+    if (e == cudaSuccess) e = cudaMalloc(&l->wd_t, (size_t)H * l->ldn * 2);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    cudaError_t e = launch_pack(static_cast<const uint16_t *>(W_gate), static_cast<const uint16_t *>(W_up),
-                                static_cast<const uint16_t *>(W_down), H, N, l->wg_t, l->w_ud, s);
+    if (e == cudaSuccess)
+        e = launch_pack(static_cast<const uint16_t *>(W_gate), static_cast<const uint16_t *>(W_up),
+                        static_cast<const uint16_t *>(W_down), H, N, l->wg_t, l->w_ud, l->wd_t, l->ldn, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) {
         cudaFree(l->wg_t);
         cudaFree(l->w_ud);
+        cudaFree(l->wd_t);
         delete l;
         return SATS_ECUDA;
     }
@@ -179,10 +192,11 @@ sats_status sats_layer_destroy(sats_layer *layer)
 {
     if (!layer) return SATS_EINVAL;
     cudaDeviceSynchronize();
-    cudaError_t e1 = cudaFree(layer->wg_t);
-    cudaError_t e2 = cudaFree(layer->w_ud);
+    const cudaError_t e1 = cudaFree(layer->wg_t);
+    const cudaError_t e2 = cudaFree(layer->w_ud);
+    const cudaError_t e3 = cudaFree(layer->wd_t);
     delete layer;
-    return (e1 == cudaSuccess && e2 == cudaSuccess) ? SATS_OK : SATS_ECUDA;
+    return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess) ? SATS_OK : SATS_ECUDA;
 }
 
 sats_status sats_layer_shape(const sats_layer *layer, int *H, int *N)
@@ -228,6 +242,8 @@ sats_status sats_sparse_mlp_fixed_scratch(const sats_layer *layer, const void *x
         return SATS_ECUDA;
     return sparse_common(layer, kXBf16, x, B, t_l, y, active_idx, active_cnt, ws, kFixedScratchBytes, stream);
 }
+
+int sats_uses_tensor_cores(int H, int B) { return use_tc_path(H, B) ? 1 : 0; }
 
 sats_status sats_sparse_mlp_f32(const sats_layer *layer, const float *x, int B, float t_l, float *y,
                                 int32_t *active_idx, int32_t *active_cnt, void *ws, size_t ws_bytes, void *stream)

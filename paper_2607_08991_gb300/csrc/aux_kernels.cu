@@ -172,13 +172,11 @@ __global__ void __launch_bounds__(1024) find_bin_kernel(const unsigned *__restri
                                                         int *__restrict__ sel, float *__restrict__ t_out)
 {
     __shared__ unsigned long long warp_tot[32];
-    __shared__ unsigned long long thr_tot[1024];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const long long r = level ? (long long)sel[1] : (long long)m;
     constexpr int kPer = kBins / 1024;
     unsigned long long s = 0;
     for (int i = 0; i < kPer; ++i) s += hist[tid * kPer + i];
-    thr_tot[tid] = s;
     unsigned long long incl = s;
     for (int o = 1; o < 32; o <<= 1) {
         const unsigned long long t = __shfl_up_sync(0xffffffffu, incl, o);
@@ -212,13 +210,17 @@ __global__ void __launch_bounds__(1024) find_bin_kernel(const unsigned *__restri
 }  // namespace
 
 cudaError_t launch_pack(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd, int H, int N,
-                        uint16_t *wg_t, uint16_t *w_ud, cudaStream_t stream)
+                        uint16_t *wg_t, uint16_t *w_ud, uint16_t *wd_t, int ldn, cudaStream_t stream)
 {
     const dim3 block(kTile, 8);
     const dim3 grid((N + kTile - 1) / kTile, (H + kTile - 1) / kTile);
     transpose_kernel<<<grid, block, 0, stream>>>(Wg, H, N, wg_t, H);
     transpose_kernel<<<grid, block, 0, stream>>>(Wu, H, N, w_ud, 2 * H);
     copy_rows_kernel<<<1024, 256, 0, stream>>>(Wd, N, H, w_ud + H, 2 * H);
+    cudaError_t e = cudaMemsetAsync(wd_t, 0, (size_t)H * ldn * sizeof(uint16_t), stream);
+    if (e != cudaSuccess) return e;
+    const dim3 grid_d((H + kTile - 1) / kTile, (N + kTile - 1) / kTile);
+    transpose_kernel<<<grid_d, block, 0, stream>>>(Wd, N, H, wd_t, ldn);
     return cudaGetLastError();
 }
 

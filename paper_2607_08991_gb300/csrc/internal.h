@@ -13,6 +13,8 @@ struct sats_layer {
     int device = 0;
     uint16_t *wg_t = nullptr;   // [N][H]: row j = column j of W_gate
     uint16_t *w_ud = nullptr;   // [N][2H]: row j = column j of W_up, then row j of W_down
+    uint16_t *wd_t = nullptr;   // [H][ldn]: row h = column h of W_down (tensor-core path)
+    int ldn = 0;                // N rounded up to a multiple of 8 (16-byte rows)
 };
 
 namespace sats {
@@ -37,7 +39,7 @@ enum {
 };
 
 struct WsLayout {
-    size_t ctl, keep, route_perm, route_flags, total;
+    size_t ctl, keep, route_perm, route_flags, tc, total;
 };
 WsLayout ws_layout(int H, int N, int B);
 
@@ -70,7 +72,14 @@ int fused_tokens_per_pass(int H);
 cudaError_t launch_fused(const FusedParams &p, cudaStream_t stream);
 
 cudaError_t launch_pack(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd, int H, int N,
-                        uint16_t *wg_t, uint16_t *w_ud, cudaStream_t stream);
+                        uint16_t *wg_t, uint16_t *w_ud, uint16_t *wd_t, int ldn, cudaStream_t stream);
+
+// Tensor-core path (gemm_tc.cu) for batches larger than one fused pass.
+bool use_tc_path(int H, int B);
+size_t tc_workspace_bytes(int H, int N, int B);
+cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int B, float t_l, const float *norm_w,
+                         float eps, const uint8_t *dense_flags, int out_mode, float *out, int32_t *active_idx,
+                         int32_t *active_cnt, uint8_t *keep_trace, void *tc_ws, int *ctl, cudaStream_t stream);
 cudaError_t launch_route(const int32_t *ids, int B, const uint8_t *lut, int V, int32_t *perm,
                          int32_t *n_dense, uint8_t *flags, int32_t *status, cudaStream_t stream);
 cudaError_t launch_gate_act(const sats_layer *layer, const uint16_t *x, int B, float *a,

@@ -49,6 +49,7 @@ def lib() -> ctypes.CDLL:
             "sats_sparse_mlp": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_sparse_mlp_f32": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_sparse_mlp_fixed_scratch": (I, [P, P, I, F, P, P, P, P]),
+            "sats_uses_tensor_cores": (I, [I, I]),
             "sats_dense_mlp": (I, [P, P, I, P, P, Z, P]),
             "sats_route": (I, [P, I, P, I, P, P, P, P]),
             "sats_mlp_stack": (I, [P, P, P, I, F, P, P, I, P, I, P, P, Z, P]),
@@ -70,7 +71,7 @@ def exported_symbols() -> Sequence[str]:
     """Every C entry point this binding forwards to."""
     return ("sats_version", "sats_status_string", "sats_layer_create", "sats_layer_destroy", "sats_layer_shape",
             "sats_workspace_bytes", "sats_workspace_init", "sats_sparse_mlp", "sats_sparse_mlp_f32",
-            "sats_sparse_mlp_fixed_scratch", "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
+            "sats_sparse_mlp_fixed_scratch", "sats_uses_tensor_cores", "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
             "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_get_error", "sats_get_status_word")
 
 
@@ -172,6 +173,11 @@ def sparse_mlp_fixed_scratch(layer: Layer, x: torch.Tensor, t_l: float, y: torch
     _check(lib().sats_sparse_mlp_fixed_scratch(layer.handle, _ptr(x, "x", 2), B, float(t_l), _ptr(y, "y", 4),
                                                _ptr(active_idx, "active_idx", 4), _ptr(active_cnt, "active_cnt", 4),
                                                _stream(stream)), "sats_sparse_mlp_fixed_scratch")
+
+
+def uses_tensor_cores(H: int, B: int) -> bool:
+    """True if a batch of B tokens on hidden size H runs on the tensor-core path."""
+    return bool(lib().sats_uses_tensor_cores(int(H), int(B)))
 
 
 def dense_mlp(layer: Layer, x: torch.Tensor, y: torch.Tensor, ws: Workspace,

@@ -84,7 +84,7 @@ def _stack(sats, oracle, L, H, N, B, targets, eps, routed=False, V=1000, p_dense
                                            [w.Wd for w in ws_], nw, t, eps, ids=ids, lut=lut,
                                            keep_hint=keep_gpu, band_rel=P.BAND_REL, want_keep=True)
     assert np.array_equal(keep_gpu, keep_ref), "per-layer kept sets differ outside the band"
-    P.assert_close(x.cpu().numpy(), x_ref)
+    P.assert_close(x.cpu().numpy(), x_ref, tight=not sats.uses_tensor_cores(H, B))
     for l in layers:
         l.close()
     return keep_ref, ids, lut
@@ -96,7 +96,7 @@ def test_stack_matches_oracle(sats, oracle, L, H, N, B):
     _stack(sats, oracle, L, H, N, B, targets, 1e-5)
 
 
-@pytest.mark.parametrize("B", [1, 8])
+@pytest.mark.parametrize("B", [1, 8, 64])
 def test_routed_stack_matches_oracle(sats, oracle, B):
     L, H, N = 3, 512, 1408
     keep, ids, lut = _stack(sats, oracle, L, H, N, B, [0.5] * L, 1e-6, routed=True, p_dense=0.4, seed=B)
