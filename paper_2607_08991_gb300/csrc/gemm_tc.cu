@@ -20,6 +20,7 @@
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
+#include <atomic>
 #include <cmath>
 #include <mutex>
 
@@ -296,7 +297,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool k0 = fabsf(a0) >= thr, k1 = fabsf(a1) >= thr;  // Eqs. 4-5
                 hw[e / 2] = (uint32_t)bf16_bits(k0 ? a0 * u[e] : 0.f) |
                             ((uint32_t)bf16_bits(k1 ? a1 * u[e + 1] : 0.f) << 16);
-                kw[e / 8] |= ((k0 ? 1u : 0u) << (8 * (e % 4))) | ((k1 ? 1u : 0u) << (8 * (e % 4) + 8));
+                kw[e / 4] |=((k0 ? 1u : 0u) << (8 * (e % 4))) | ((k1 ? 1u : 0u) << (8 * (e % 4) + 8));
             }
             uint16_t *hrow = p.hact + (size_t)m * p.ldh + n;
             uint8_t *krow = p.keep ? p.keep + (size_t)m * p.keep_stride + n : nullptr;
@@ -538,16 +539,17 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols, 
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Raises the kernel's dynamic shared-memory limit once per device; `configured`
+// is the caller's flag word, one per kernel instantiation.
 template <typename K>
-cudaError_t set_smem(K kernel, size_t bytes)
+cudaError_t set_smem(K kernel, size_t bytes, std::atomic<unsigned long long> &configured)
 {
-    static unsigned long long configured = 0;
     int dev = 0;
     cudaGetDevice(&dev);
     const unsigned long long bit = 1ull << (dev & 63);
-    if (configured & bit) return cudaSuccess;
+    if (configured.load() & bit) return cudaSuccess;
     const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-    if (e == cudaSuccess) configured |= bit;
+    if (e == cudaSuccess) configured.fetch_or(bit);
     return e;
 }
 
@@ -556,7 +558,8 @@ cudaError_t launch_gu_t(const CUtensorMap &a, const CUtensorMap &a2, const CUten
                         const GuParams &p, cudaStream_t stream)
 {
     using Sh = GuShape<BN, SPLIT>;
-    cudaError_t e = set_smem(gu_kernel<BN, SPLIT>, Sh::kSmem);
+    static std::atomic<unsigned long long> configured{0};
+    cudaError_t e = set_smem(gu_kernel<BN, SPLIT>, Sh::kSmem, configured);
     if (e != cudaSuccess) return e;
     const dim3 grid((p.N + BN - 1) / BN, (p.M + BM - 1) / BM);
     gu_kernel<BN, SPLIT><<<grid, kThreads, Sh::kSmem, stream>>>(a, a2, g, u, p);
@@ -568,7 +571,8 @@ cudaError_t launch_down_t(const CUtensorMap &a, const CUtensorMap &b, const Down
                           cudaStream_t stream)
 {
     using Sh = DownShape<BN>;
-    cudaError_t e = set_smem(down_kernel<BN>, Sh::kSmem);
+    static std::atomic<unsigned long long> configured{0};
+    cudaError_t e = set_smem(down_kernel<BN>, Sh::kSmem, configured);
     if (e != cudaSuccess) return e;
     const dim3 grid((p.H + BN - 1) / BN, (p.M + BM - 1) / BM, splits);
     down_kernel<BN><<<grid, kThreads, Sh::kSmem, stream>>>(a, b, p);

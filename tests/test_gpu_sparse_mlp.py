@@ -159,7 +159,8 @@ def test_dense_mlp_matches_oracle(sats, oracle):
     y = torch.empty(B, H, dtype=torch.float32, device="cuda")
     sats.dense_mlp(layer, P.dev_u16(xb), y, ws)
     assert sats.get_error(ws) == sats.OK
-    P.assert_close(y.cpu().numpy(), oracle.dense_mlp(oracle.bf16_to_f64(xb), w.Wg, w.Wu, w.Wd))
+    P.assert_close(y.cpu().numpy(), oracle.dense_mlp(oracle.bf16_to_f64(xb), w.Wg, w.Wu, w.Wd),
+                   tight=not sats.uses_tensor_cores(H, B))
 
 
 def test_skipped_rows_are_not_read(sats, oracle):
