@@ -167,20 +167,19 @@ sats_status sats_layer_create(const void *W_gate, const void *W_up, const void *
     l->H = H;
     l->N = N;
     cudaGetDevice(&l->device);
-    l->ldn = (N + 7) & ~7;
     const size_t row_elems = (size_t)N * H;
     cudaError_t e = cudaMalloc(&l->wg_t, row_elems * 2);
     if (e == cudaSuccess) e = cudaMalloc(&l->w_ud, row_elems * 4);
-    if (e == cudaSuccess) e = cudaMalloc(&l->wd_t, (size_t)H * l->ldn * 2);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (e == cudaSuccess)
         e = launch_pack(static_cast<const uint16_t *>(W_gate), static_cast<const uint16_t *>(W_up),
-                        static_cast<const uint16_t *>(W_down), H, N, l->wg_t, l->w_ud, l->wd_t, l->ldn, s);
+                        static_cast<const uint16_t *>(W_down), H, N, l->wg_t, l->w_ud, s);
+    if (e == cudaSuccess) e = tc_pack_layer(l, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) {
         cudaFree(l->wg_t);
         cudaFree(l->w_ud);
-        cudaFree(l->wd_t);
+        tc_free_layer(l);
         delete l;
         return SATS_ECUDA;
     }
@@ -194,7 +193,7 @@ sats_status sats_layer_destroy(sats_layer *layer)
     cudaDeviceSynchronize();
     const cudaError_t e1 = cudaFree(layer->wg_t);
     const cudaError_t e2 = cudaFree(layer->w_ud);
-    const cudaError_t e3 = cudaFree(layer->wd_t);
+    const cudaError_t e3 = tc_free_layer(layer);
     delete layer;
     return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess) ? SATS_OK : SATS_ECUDA;
 }

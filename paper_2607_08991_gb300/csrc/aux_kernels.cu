@@ -210,17 +210,13 @@ __global__ void __launch_bounds__(1024) find_bin_kernel(const unsigned *__restri
 }  // namespace
 
 cudaError_t launch_pack(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd, int H, int N,
-                        uint16_t *wg_t, uint16_t *w_ud, uint16_t *wd_t, int ldn, cudaStream_t stream)
+                        uint16_t *wg_t, uint16_t *w_ud, cudaStream_t stream)
 {
     const dim3 block(kTile, 8);
     const dim3 grid((N + kTile - 1) / kTile, (H + kTile - 1) / kTile);
     transpose_kernel<<<grid, block, 0, stream>>>(Wg, H, N, wg_t, H);
     transpose_kernel<<<grid, block, 0, stream>>>(Wu, H, N, w_ud, 2 * H);
     copy_rows_kernel<<<1024, 256, 0, stream>>>(Wd, N, H, w_ud + H, 2 * H);
-    cudaError_t e = cudaMemsetAsync(wd_t, 0, (size_t)H * ldn * sizeof(uint16_t), stream);
-    if (e != cudaSuccess) return e;
-    const dim3 grid_d((H + kTile - 1) / kTile, (N + kTile - 1) / kTile);
-    transpose_kernel<<<grid_d, block, 0, stream>>>(Wd, N, H, wd_t, ldn);
     return cudaGetLastError();
 }
 

@@ -12,10 +12,21 @@
 // the same accumulator, so that the gate values keep ~fp32 accuracy.  h is
 // kept in bf16 between the two GEMMs.
 //
-// Kernel layout (one output tile per CTA, 192 threads): warp 0 lane 0 issues
-// the TMA loads, warp 1 owns the TMEM allocation and lane 0 issues the MMAs,
-// warps 2-5 run the epilogue (warp w reads TMEM lanes 32 (w mod 4) ..).
-// Every wait is bounded in time and sets the status word when it gives up.
+// Two orientations:
+//  - skinny (M <= 256 tokens, bandwidth-bound): the weights are the MMA's A
+//    operand (128 rows: neurons, or hidden units for the down projection) and
+//    the tokens its N dimension, so no MMA row is spent on absent tokens.  The
+//    down projection splits its 64-neuron K blocks evenly over one CTA per SM
+//    and adds partial sums into y with L2 reductions.
+//  - wide (prefill): tokens are the A operand in tiles of 128, the weights the
+//    B operand; CTAs that run together share weight tiles through L2.
+// The weights are read from tile-contiguous copies made at layer creation
+// (gu_blk, wd_blk), so that every TMA box is one contiguous DRAM read.
+//
+// Kernel layout (192 threads): warp 0 lane 0 issues the TMA loads, warp 1 owns
+// the TMEM allocation and lane 0 issues the MMAs, warps 2-5 run the epilogue
+// (warp w reads TMEM lanes 32 (w mod 4) .. 32 (w mod 4) + 31).  Every wait is
+// bounded in time and sets the status word when it gives up.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
@@ -31,11 +42,13 @@ namespace sats {
 namespace tc {
 namespace {
 
-constexpr int BM = 128;              // tokens per tile (MMA M)
-constexpr int BK = 64;               // K per stage: one 128-byte swizzle row of bf16
+constexpr int BM = 128;              // MMA M: rows of the A operand
+constexpr int BK = 64;               // K per TMA box: one 128-byte swizzle row of bf16
 constexpr int kThreads = 192;
 constexpr int kSmemBudget = 196608;  // stage ring
-constexpr uint32_t kTmemCols = 256;
+constexpr int kMaxStages = 8;
+constexpr int kMaxSkinny = 256;      // largest batch on the skinny orientation (MMA N <= 256)
+constexpr int kTileBytes = BK * 2;   // bytes of one tile row
 
 // ---------------------------------------------------------------------- device helpers
 // Shared-memory matrix descriptor of a K-major bf16 tile written by TMA with
@@ -135,6 +148,13 @@ __device__ __forceinline__ uint8_t *align1024(uint8_t *p)
     return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(p) + 1023) & ~(uintptr_t)1023);
 }
 
+
+__device__ __forceinline__ void set_timeout(int *ctl, volatile int *abort_flag)
+{
+    *abort_flag = 1;
+    atomicOr(ctl + kCtlStatus, kStatusTimeout);
+}
+
 // ---------------------------------------------------------------------- activations
 // Row m of X (fp32, optionally RMS-normalised with gain w) -> bf16 hi + lo.
 __global__ void __launch_bounds__(256) split_kernel(const float *__restrict__ x, int H, const float *__restrict__ w,
@@ -163,50 +183,82 @@ __global__ void __launch_bounds__(256) split_kernel(const float *__restrict__ x,
     }
 }
 
-// ---------------------------------------------------------------------- gate + up GEMM
-struct GuParams {
-    int M, N, H;
+// ---------------------------------------------------------------------- weight tiles
+// gu_blk[t][kb][g][r][c] = (g ? W_up : W_gate)[k][n] with n = t R + r,
+// k = kb 64 + c, read from wg_t [N][H] and the W_up half of w_ud [N][2H].
+// One thread per 8 consecutive c (16 bytes; H is a multiple of 8).
+__global__ void pack_gu_kernel(const uint16_t *__restrict__ wg_t, const uint16_t *__restrict__ w_ud, int H, int N,
+                               int R, int KBh, size_t total8, uint16_t *__restrict__ dst)
+{
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total8; i += (size_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % 8) * 8;
+        size_t rest = i / 8;
+        const int r = (int)(rest % R);
+        rest /= R;
+        const int g = (int)(rest % 2);
+        rest /= 2;
+        const int kb = (int)(rest % KBh);
+        const int t = (int)(rest / KBh);
+        const int n = t * R + r, k = kb * BK + c;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (n < N && k < H)
+            v = *reinterpret_cast<const uint4 *>(g ? w_ud + (size_t)n * 2 * H + k : wg_t + (size_t)n * H + k);
+        reinterpret_cast<uint4 *>(dst)[i] = v;
+    }
+}
+
+// wd_blk[d][kb][r][c] = W_down[n][h] with n = kb 64 + c, h = d 128 + r (W_down
+// row n is the second half of w_ud row n).  One CTA per (kb, d) tile, through
+// shared memory so that both sides are read and written in rows.
+__global__ void __launch_bounds__(256) pack_wd_kernel(const uint16_t *__restrict__ w_ud, int H, int N, int KBn,
+                                                      uint16_t *__restrict__ dst)
+{
+    __shared__ uint16_t tile[BK][BM + 2];
+    const int kb = blockIdx.x, d = blockIdx.y;
+    for (int i = threadIdx.x; i < BK * BM; i += 256) {
+        const int c = i / BM, r = i % BM;
+        const int n = kb * BK + c, h = d * BM + r;
+        tile[c][r] = (n < N && h < H) ? w_ud[(size_t)n * 2 * H + H + h] : (uint16_t)0;
+    }
+    __syncthreads();
+    uint16_t *out = dst + ((size_t)d * KBn + kb) * BM * BK;
+    for (int i = threadIdx.x; i < BM * BK; i += 256) out[i] = tile[i % BK][i / BK];
+}
+
+// ---------------------------------------------------------------------- skinny gate + up
+struct SkinnyGuParams {
+    int M, N, R, KBh, NT;
+    int split;                    // 1: two B operands (bf16 hi and lo parts of fp32 x)
     float t_l;                    // threshold of sparse-path tokens
     const uint8_t *dense_flags;   // [M] (1 = base path, threshold 0) or nullptr
     uint16_t *hact;               // [M][ldh] bf16
     int ldh;
     uint8_t *keep;                // [M][keep_stride] or nullptr
-    int keep_stride;              // a multiple of 16
+    int keep_stride;
     uint8_t *keep_trace;          // [M][N] or nullptr
     int *ctl;
+    int stages, stage_bytes, a_bytes, x_bytes;
+    uint32_t tmem_cols;
 };
 
-template <int BN, bool SPLIT>
-struct GuShape {
-    static constexpr int kA = BM * 128, kB = BN * 128;
-    static constexpr int kStage = kA * (SPLIT ? 2 : 1) + 2 * kB;
-    static constexpr int kStages = (kSmemBudget / kStage) > 6 ? 6 : (kSmemBudget / kStage);
-    static constexpr size_t kSmem = (size_t)kStages * kStage + 1024 + 256;
-    static_assert(kStage % 1024 == 0, "stages keep the 1024-byte alignment of the swizzle atoms");
-    static_assert(2 * BN <= (int)kTmemCols, "gate and up accumulators fit the TMEM allocation");
-};
-
-// One 128-token x BN-neuron tile of G = X W_gate and U = X W_up (K = H), then
-// h = CATS(SiLU(G)) * U in the epilogue.  Grid: (ceil(N / BN), ceil(M / 128)).
-template <int BN, bool SPLIT>
+// One tile of R neurons (gate and up) against all M tokens: D[r][j] in TMEM
+// lane r, column j (gate) and NT + j (up).  Grid: tc_T CTAs.
 __global__ void __launch_bounds__(kThreads, 1)
-    gu_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
-              const __grid_constant__ CUtensorMap tmG, const __grid_constant__ CUtensorMap tmU, const GuParams p)
+    gu_skinny_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+                     const __grid_constant__ CUtensorMap tmX2, const SkinnyGuParams p)
 {
-    using Sh = GuShape<BN, SPLIT>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *ring = align1024(smem_raw);
-    uint64_t *full = reinterpret_cast<uint64_t *>(ring + (size_t)Sh::kStages * Sh::kStage);
-    uint64_t *empty = full + Sh::kStages;
-    uint64_t *acc_full = empty + Sh::kStages;
+    uint64_t *full = reinterpret_cast<uint64_t *>(ring + (size_t)p.stages * p.stage_bytes);
+    uint64_t *empty = full + kMaxStages;
+    uint64_t *acc_full = empty + kMaxStages;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_full + 1);
     __shared__ int abort_flag, issued_s, consumed_s;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
-    const int KB = (p.H + BK - 1) / BK;
+    const int t = blockIdx.x, R = p.R, NT = p.NT, S = p.stages;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < Sh::kStages; ++s) {
+        for (int s = 0; s < S; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
@@ -216,65 +268,328 @@ __global__ void __launch_bounds__(kThreads, 1)
         consumed_s = 0;
         mbar_init_fence();
     }
-    if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
+    if (warp == 1) tmem_alloc(tmem_slot, p.tmem_cols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    grid_launch_dependents();   // the down projection may start prefetching its weights
+
+    if (warp == 0 && lane == 0) {
+        const uint32_t load_bytes = (uint32_t)(2 * R * kTileBytes + p.x_bytes * (p.split ? 2 : 1));
+        int kb = 0;
+        for (int s = 0, ph = 0; kb < p.KBh; ++kb) {
+            if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
+            uint8_t *st = ring + (size_t)s * p.stage_bytes;
+            mbar_arrive_expect_tx(&full[s], load_bytes);
+            tma_load(st, &tmW, 0, (t * p.KBh + kb) * 2 * R, &full[s]);
+            tma_load(st + p.a_bytes, &tmX, kb * BK, 0, &full[s]);
+            if (p.split) tma_load(st + p.a_bytes + p.x_bytes, &tmX2, kb * BK, 0, &full[s]);
+            if (++s == S) { s = 0; ph ^= 1; }
+        }
+        issued_s = kb;
+    } else if (warp == 1 && lane == 0) {
+        const uint32_t idesc = instr_desc(BM, NT);
+        int kb = 0;
+        for (int s = 0, ph = 0; kb < p.KBh; ++kb) {
+            if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
+            tc_fence_after();
+            const uint32_t st = smem_addr(ring + (size_t)s * p.stage_bytes);
+            const uint32_t xa = st + p.a_bytes;
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk) {
+                const uint32_t acc = (kb | kk) ? 1u : 0u;
+                const uint64_t ag = smem_desc(st + kk * 32);
+                const uint64_t au = smem_desc(st + R * kTileBytes + kk * 32);
+                const uint64_t b = smem_desc(xa + kk * 32);
+                mma_bf16(tmem, ag, b, idesc, acc);
+                mma_bf16(tmem + NT, au, b, idesc, acc);
+                if (p.split) {
+                    const uint64_t b2 = smem_desc(xa + p.x_bytes + kk * 32);
+                    mma_bf16(tmem, ag, b2, idesc, 1u);
+                    mma_bf16(tmem + NT, au, b2, idesc, 1u);
+                }
+            }
+            mma_commit(&empty[s]);
+            if (++s == S) { s = 0; ph ^= 1; }
+        }
+        consumed_s = kb;
+        mma_commit(acc_full);
+    } else if (warp >= 2) {
+        // epilogue: thread = neuron r of the tile, columns = tokens
+        const bool ok = mbar_wait(acc_full, 0u, &abort_flag);
+        tc_fence_after();
+        const int lb = 32 * (warp & 3);
+        const int r = lb + lane, n = t * R + r;
+        const bool row_ok = ok && r < R && n < p.N;
+        for (int c0 = 0; c0 < NT; c0 += 16) {
+            float g[16], u[16];
+            tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)c0, g);
+            tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(NT + c0), u);
+            tmem_ld_wait();
+            if (!row_ok) continue;
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int j = c0 + e;
+                if (j < p.M) {
+                    const float thr = (p.dense_flags && p.dense_flags[j]) ? 0.f : p.t_l;
+                    const float a = g[e] / (1.0f + expf(-g[e]));   // SiLU, Eq. 2
+                    const bool keep = fabsf(a) >= thr;             // Eqs. 4-5
+                    p.hact[(size_t)j * p.ldh + n] = bf16_bits(keep ? a * u[e] : 0.f);
+                    if (p.keep) p.keep[(size_t)j * p.keep_stride + n] = keep ? 1 : 0;
+                    if (p.keep_trace) p.keep_trace[(size_t)j * p.N + n] = keep ? 1 : 0;
+                }
+            }
+        }
+        tc_fence_before();
+    }
+    __syncthreads();
+    if (abort_flag && threadIdx.x == 0) drain_after_abort(full, S, issued_s, consumed_s, acc_full);
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, p.tmem_cols);
+    }
+}
+
+// ---------------------------------------------------------------------- skinny down
+struct SkinnyDownParams {
+    int M, H, NT, KBn, units;     // units = tc_dt * KBn (hidden tile, neuron block) pairs
+    float *out;                   // [M][H] fp32, added to with L2 reductions
+    int *ctl;
+    int stages, stage_bytes, a_bytes;
+    uint32_t tmem_cols;           // two accumulators of NT columns
+};
+
+// CTA c handles units [c U / G, (c+1) U / G) in order; consecutive units of one
+// hidden tile form a segment accumulated in TMEM (two buffers, so that the
+// epilogue of one segment overlaps the MMAs of the next) and added into y.
+// Unit u's weight tile starts at row u * 128 of wd_blk.
+__global__ void __launch_bounds__(kThreads, 1)
+    down_skinny_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmH,
+                       const SkinnyDownParams p)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *ring = align1024(smem_raw);
+    uint64_t *full = reinterpret_cast<uint64_t *>(ring + (size_t)p.stages * p.stage_bytes);
+    uint64_t *empty = full + kMaxStages;
+    uint64_t *acc_full = empty + kMaxStages;   // [2]
+    uint64_t *acc_empty = acc_full + 2;        // [2]
+    uint64_t *mma_done = acc_empty + 2;        // every MMA of this CTA has completed
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mma_done + 1);
+    __shared__ int abort_flag, issued_s, consumed_s;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int S = p.stages, NT = p.NT, KBn = p.KBn;
+    const int u0 = (int)((long long)blockIdx.x * p.units / gridDim.x);
+    const int u1 = (int)((long long)(blockIdx.x + 1) * p.units / gridDim.x);
+    const int nu = u1 - u0;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], 128);
+        }
+        mbar_init(mma_done, 1);
+        abort_flag = 0;
+        issued_s = 0;
+        consumed_s = 0;
+        mbar_init_fence();
+    }
+    if (warp == 1) tmem_alloc(tmem_slot, p.tmem_cols);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
     if (warp == 0 && lane == 0) {
-        // TMA producer
-        int kb = 0;
-        for (uint32_t s = 0, ph = 0; kb < KB; ++kb) {
-            if (!mbar_wait(&empty[s], ph ^ 1u, &abort_flag)) {
-                abort_flag = 1;
-                atomicOr(p.ctl + kCtlStatus, kStatusTimeout);
-                break;
-            }
-            uint8_t *st = ring + (size_t)s * Sh::kStage;
-            uint8_t *g = st + Sh::kA * (SPLIT ? 2 : 1);
-            mbar_arrive_expect_tx(&full[s], (uint32_t)Sh::kStage);
-            tma_load(st, &tmA, kb * BK, m0, &full[s]);
-            if (SPLIT) tma_load(st + Sh::kA, &tmA2, kb * BK, m0, &full[s]);
-            tma_load(g, &tmG, kb * BK, n0, &full[s]);
-            tma_load(g + Sh::kB, &tmU, kb * BK, n0, &full[s]);
-            if (++s == (uint32_t)Sh::kStages) { s = 0; ph ^= 1u; }
+        const uint32_t load_bytes = (uint32_t)(BM * kTileBytes + NT * kTileBytes);
+        // the weight tiles do not depend on the preceding kernel: start them first
+        const int npre = nu < S ? nu : S;
+        for (int i = 0; i < npre; ++i) {
+            mbar_arrive_expect_tx(&full[i], load_bytes);
+            tma_load(ring + (size_t)i * p.stage_bytes, &tmW, 0, (u0 + i) * BM, &full[i]);
         }
-        issued_s = kb;
+        grid_dependency_wait();   // h is written by the preceding gate/up kernel
+        int i = 0;
+        for (int s = 0, ph = 0; i < nu; ++i) {
+            const int u = u0 + i;
+            uint8_t *st = ring + (size_t)s * p.stage_bytes;
+            if (i >= npre) {
+                if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
+                mbar_arrive_expect_tx(&full[s], load_bytes);
+                tma_load(st, &tmW, 0, u * BM, &full[s]);
+            }
+            tma_load(st + p.a_bytes, &tmH, (u % KBn) * BK, 0, &full[s]);
+            if (++s == S) { s = 0; ph ^= 1; }
+        }
+        issued_s = i;   // a break happens only before stage i's loads are issued (i >= npre)
     } else if (warp == 1 && lane == 0) {
-        // MMA issuer: gate accumulator at TMEM column 0, up accumulator at column BN
-        constexpr uint32_t idesc = instr_desc(BM, BN);
-        int kb = 0;
-        for (uint32_t s = 0, ph = 0; kb < KB; ++kb) {
-            if (!mbar_wait(&full[s], ph, &abort_flag)) {
-                abort_flag = 1;
-                atomicOr(p.ctl + kCtlStatus, kStatusTimeout);
+        const uint32_t idesc = instr_desc(BM, NT);
+        int i = 0, q = 0;
+        int s = 0, ph = 0;
+        for (int u = u0; u < u1 && !abort_flag;) {
+            const int seg_end = min(u1, (u / KBn + 1) * KBn);
+            const int buf = q & 1;
+            if (!mbar_wait(&acc_empty[buf], (uint32_t)((q >> 1) & 1) ^ 1u, &abort_flag)) {
+                set_timeout(p.ctl, &abort_flag);
                 break;
             }
             tc_fence_after();
-            const uint32_t st = smem_addr(ring + (size_t)s * Sh::kStage);
-            const uint32_t ga = st + Sh::kA * (SPLIT ? 2 : 1);
+            bool first = true;
+            for (; u < seg_end; ++u, ++i) {
+                if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
+                tc_fence_after();
+                const uint32_t st = smem_addr(ring + (size_t)s * p.stage_bytes);
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk)
+                    mma_bf16(tmem + (uint32_t)(buf * NT), smem_desc(st + kk * 32), smem_desc(st + p.a_bytes + kk * 32),
+                             idesc, (first && kk == 0) ? 0u : 1u);
+                first = false;
+                mma_commit(&empty[s]);
+                if (++s == S) { s = 0; ph ^= 1; }
+            }
+            mma_commit(&acc_full[buf]);
+            ++q;
+        }
+        consumed_s = i;
+        mma_commit(mma_done);
+    } else if (warp >= 2) {
+        const int lb = 32 * (warp & 3);
+        int q = 0;
+        for (int u = u0; u < u1; ++q) {
+            const int d = u / KBn;
+            const int seg_end = min(u1, (d + 1) * KBn);
+            const int buf = q & 1;
+            const bool ok = mbar_wait(&acc_full[buf], (uint32_t)((q >> 1) & 1), &abort_flag);
+            tc_fence_after();
+            const int h = d * BM + lb + lane;
+            for (int c0 = 0; c0 < NT; c0 += 16) {
+                float v[16];
+                tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * NT + c0), v);
+                tmem_ld_wait();
+                if (!ok || h >= p.H) continue;
+#pragma unroll
+                for (int e = 0; e < 16; ++e)
+                    if (c0 + e < p.M) atomicAdd(p.out + (size_t)(c0 + e) * p.H + h, v[e]);
+            }
+            tc_fence_before();
+            mbar_arrive(&acc_empty[buf]);
+            if (!ok) break;
+            u = seg_end;
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        // the arrival on mma_done must land before this CTA's shared memory is released
+        int never = 0;
+        if (abort_flag)
+            for (int k = consumed_s; k < issued_s; ++k) mbar_wait(&full[k % S], (uint32_t)((k / S) & 1), &never);
+        mbar_wait(mma_done, 0u, &never);
+    }
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, p.tmem_cols);
+    }
+}
+
+// ---------------------------------------------------------------------- wide gate + up
+struct WideGuParams {
+    int M, N, R, KBh;
+    int split;
+    float t_l;
+    const uint8_t *dense_flags;
+    uint16_t *hact;
+    int ldh;
+    uint8_t *keep;
+    int keep_stride;              // a multiple of 16
+    uint8_t *keep_trace;
+    int *ctl;
+    int stages, stage_bytes;
+};
+
+// One 128-token x R-neuron tile of G and U: D[m][c] in TMEM lane m, column c
+// (gate) and R + c (up).  Grid: (ceil(M / 128), tc_T); the token tiles of one
+// weight tile are adjacent in launch order, so they read it from L2.
+__global__ void __launch_bounds__(kThreads, 1)
+    gu_wide_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmX2,
+                   const __grid_constant__ CUtensorMap tmW, const WideGuParams p)
+{
+    constexpr int kA = BM * kTileBytes;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *ring = align1024(smem_raw);
+    uint64_t *full = reinterpret_cast<uint64_t *>(ring + (size_t)p.stages * p.stage_bytes);
+    uint64_t *empty = full + kMaxStages;
+    uint64_t *acc_full = empty + kMaxStages;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_full + 1);
+    __shared__ int abort_flag, issued_s, consumed_s;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.x * BM, t = blockIdx.y, R = p.R, S = p.stages;
+    const int wofs = kA * (p.split ? 2 : 1);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(acc_full, 1);
+        abort_flag = 0;
+        issued_s = 0;
+        consumed_s = 0;
+        mbar_init_fence();
+    }
+    if (warp == 1) tmem_alloc(tmem_slot, 256);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        const uint32_t load_bytes = (uint32_t)(wofs + 2 * R * kTileBytes);
+        int kb = 0;
+        for (int s = 0, ph = 0; kb < p.KBh; ++kb) {
+            if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
+            uint8_t *st = ring + (size_t)s * p.stage_bytes;
+            mbar_arrive_expect_tx(&full[s], load_bytes);
+            tma_load(st, &tmX, kb * BK, m0, &full[s]);
+            if (p.split) tma_load(st + kA, &tmX2, kb * BK, m0, &full[s]);
+            tma_load(st + wofs, &tmW, 0, (t * p.KBh + kb) * 2 * R, &full[s]);
+            if (++s == S) { s = 0; ph ^= 1; }
+        }
+        issued_s = kb;
+    } else if (warp == 1 && lane == 0) {
+        const uint32_t idesc = instr_desc(BM, R);
+        int kb = 0;
+        for (int s = 0, ph = 0; kb < p.KBh; ++kb) {
+            if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
+            tc_fence_after();
+            const uint32_t st = smem_addr(ring + (size_t)s * p.stage_bytes);
+            const uint32_t wa = st + wofs;
 #pragma unroll
             for (int kk = 0; kk < BK / 16; ++kk) {
                 const uint32_t acc = (kb | kk) ? 1u : 0u;
                 const uint64_t a = smem_desc(st + kk * 32);
-                const uint64_t g = smem_desc(ga + kk * 32);
-                const uint64_t u = smem_desc(ga + Sh::kB + kk * 32);
+                const uint64_t g = smem_desc(wa + kk * 32);
+                const uint64_t u = smem_desc(wa + R * kTileBytes + kk * 32);
                 mma_bf16(tmem, a, g, idesc, acc);
-                mma_bf16(tmem + BN, a, u, idesc, acc);
-                if (SPLIT) {
-                    const uint64_t a2 = smem_desc(st + Sh::kA + kk * 32);
+                mma_bf16(tmem + R, a, u, idesc, acc);
+                if (p.split) {
+                    const uint64_t a2 = smem_desc(st + kA + kk * 32);
                     mma_bf16(tmem, a2, g, idesc, 1u);
-                    mma_bf16(tmem + BN, a2, u, idesc, 1u);
+                    mma_bf16(tmem + R, a2, u, idesc, 1u);
                 }
             }
-            mma_commit(&empty[s]);   // the stage is free once these MMAs have read it
-            if (++s == (uint32_t)Sh::kStages) { s = 0; ph ^= 1u; }
+            mma_commit(&empty[s]);
+            if (++s == S) { s = 0; ph ^= 1; }
         }
         consumed_s = kb;
         mma_commit(acc_full);
     } else if (warp >= 2) {
-        // epilogue: thread = one token row of the tile
+        // epilogue: thread = token row of the tile, 16 neurons at a time
         const bool ok = mbar_wait(acc_full, 0u, &abort_flag);
         tc_fence_after();
         const int lb = 32 * (warp & 3);
@@ -282,26 +597,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool row_ok = ok && m < p.M;
         float thr = INFINITY;
         if (row_ok) thr = (p.dense_flags && p.dense_flags[m]) ? 0.f : p.t_l;
-        for (int c0 = 0; c0 < BN; c0 += 16) {
+        for (int c0 = 0; c0 < R; c0 += 16) {
             float g[16], u[16];
             tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)c0, g);
-            tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(BN + c0), u);
+            tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(R + c0), u);
             tmem_ld_wait();
-            const int n = n0 + c0;
+            const int n = t * R + c0;
             if (!row_ok || n >= p.N) continue;
             uint32_t hw[8], kw[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
             for (int e = 0; e < 16; e += 2) {
-                const float a0 = g[e] / (1.0f + expf(-g[e]));            // SiLU, Eq. 2
+                const float a0 = g[e] / (1.0f + expf(-g[e]));             // SiLU, Eq. 2
                 const float a1 = g[e + 1] / (1.0f + expf(-g[e + 1]));
-                const bool k0 = fabsf(a0) >= thr, k1 = fabsf(a1) >= thr;  // Eqs. 4-5
+                const bool k0 = fabsf(a0) >= thr, k1 = fabsf(a1) >= thr;   // Eqs. 4-5
                 hw[e / 2] = (uint32_t)bf16_bits(k0 ? a0 * u[e] : 0.f) |
                             ((uint32_t)bf16_bits(k1 ? a1 * u[e + 1] : 0.f) << 16);
-                kw[e / 4] |=((k0 ? 1u : 0u) << (8 * (e % 4))) | ((k1 ? 1u : 0u) << (8 * (e % 4) + 8));
+                kw[e / 4] |= ((k0 ? 1u : 0u) << (8 * (e % 4))) | ((k1 ? 1u : 0u) << (8 * (e % 4) + 8));
             }
             uint16_t *hrow = p.hact + (size_t)m * p.ldh + n;
             uint8_t *krow = p.keep ? p.keep + (size_t)m * p.keep_stride + n : nullptr;
-            if (n + 16 <= p.N) {
+            if (n + 16 <= p.N) {   // n is a multiple of 16: 32-byte aligned h, 16-byte aligned keep
                 reinterpret_cast<uint4 *>(hrow)[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
                 reinterpret_cast<uint4 *>(hrow)[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
                 if (krow) *reinterpret_cast<uint4 *>(krow) = make_uint4(kw[0], kw[1], kw[2], kw[3]);
@@ -324,56 +639,48 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
     }
     __syncthreads();
-    if (abort_flag && threadIdx.x == 0) drain_after_abort(full, Sh::kStages, issued_s, consumed_s, acc_full);
+    if (abort_flag && threadIdx.x == 0) drain_after_abort(full, S, issued_s, consumed_s, acc_full);
     __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem, kTmemCols);
+        tmem_dealloc(tmem, 256);
     }
 }
 
-// ---------------------------------------------------------------------- down GEMM
-struct DownParams {
-    int M, N, H;          // tokens, K (neurons), output columns
+// ---------------------------------------------------------------------- wide down
+struct WideDownParams {
+    int M, H, KBn;
+    int dtiles;           // 128-row hidden tiles per CTA tile (1 or 2: MMA N = 128 dtiles)
     int kb_per_split;     // K blocks of 64 neurons per split (blockIdx.z)
     int atomic_out;       // 1: add into out with L2 reductions (split K); 0: one writer per element
     int add_residual;     // with atomic_out == 0: out += tile, else out = tile
     float *out;           // [M][H] fp32
     int *ctl;
+    int stages, stage_bytes;
 };
 
-template <int BN>
-struct DownShape {
-    static constexpr int kA = BM * 128, kB = BN * 128;
-    static constexpr int kStage = kA + kB;
-    static constexpr int kStages = (kSmemBudget / kStage) > 6 ? 6 : (kSmemBudget / kStage);
-    static constexpr size_t kSmem = (size_t)kStages * kStage + 1024 + 256;
-    static_assert(kStage % 1024 == 0, "stages keep the 1024-byte alignment of the swizzle atoms");
-    static_assert(BN <= (int)kTmemCols, "the accumulator fits the TMEM allocation");
-};
-
-// One 128-token x BN-column tile of Y = h W_down over one split of the K range.
-// Grid: (ceil(H / BN), ceil(M / 128), splits).
-template <int BN>
+// One 128-token x (128 dtiles)-column tile of Y = h W_down over one split of
+// the neuron range.  Grid: (ceil(M / 128), tc_dt / dtiles, splits).
 __global__ void __launch_bounds__(kThreads, 1)
-    down_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const DownParams p)
+    down_wide_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmW,
+                     const WideDownParams p)
 {
-    using Sh = DownShape<BN>;
+    constexpr int kA = BM * kTileBytes;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *ring = align1024(smem_raw);
-    uint64_t *full = reinterpret_cast<uint64_t *>(ring + (size_t)Sh::kStages * Sh::kStage);
-    uint64_t *empty = full + Sh::kStages;
-    uint64_t *acc_full = empty + Sh::kStages;
+    uint64_t *full = reinterpret_cast<uint64_t *>(ring + (size_t)p.stages * p.stage_bytes);
+    uint64_t *empty = full + kMaxStages;
+    uint64_t *acc_full = empty + kMaxStages;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_full + 1);
     __shared__ int abort_flag, issued_s, consumed_s;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.y * BM, h0 = blockIdx.x * BN;
-    const int KB = (p.N + BK - 1) / BK;
+    const int m0 = blockIdx.x * BM, d0 = blockIdx.y * p.dtiles, S = p.stages;
+    const int BN = BM * p.dtiles;
     const int kb0 = blockIdx.z * p.kb_per_split;
-    const int kb1 = min(KB, kb0 + p.kb_per_split);
+    const int kb1 = min(p.KBn, kb0 + p.kb_per_split);
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < Sh::kStages; ++s) {
+        for (int s = 0; s < S; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
@@ -383,44 +690,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         consumed_s = 0;
         mbar_init_fence();
     }
-    if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
+    if (warp == 1) tmem_alloc(tmem_slot, 256);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
     if (warp == 0 && lane == 0) {
+        const uint32_t load_bytes = (uint32_t)(kA + BN * kTileBytes);
         int i = 0;
-        for (uint32_t s = 0, ph = 0; kb0 + i < kb1; ++i) {
-            if (!mbar_wait(&empty[s], ph ^ 1u, &abort_flag)) {
-                abort_flag = 1;
-                atomicOr(p.ctl + kCtlStatus, kStatusTimeout);
-                break;
-            }
-            uint8_t *st = ring + (size_t)s * Sh::kStage;
-            mbar_arrive_expect_tx(&full[s], (uint32_t)Sh::kStage);
-            tma_load(st, &tmA, (kb0 + i) * BK, m0, &full[s]);
-            tma_load(st + Sh::kA, &tmB, (kb0 + i) * BK, h0, &full[s]);
-            if (++s == (uint32_t)Sh::kStages) { s = 0; ph ^= 1u; }
+        for (int s = 0, ph = 0; kb0 + i < kb1; ++i) {
+            if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
+            const int kb = kb0 + i;
+            uint8_t *st = ring + (size_t)s * p.stage_bytes;
+            mbar_arrive_expect_tx(&full[s], load_bytes);
+            tma_load(st, &tmH, kb * BK, m0, &full[s]);
+            for (int q = 0; q < p.dtiles; ++q)
+                tma_load(st + kA + q * kA, &tmW, 0, ((d0 + q) * p.KBn + kb) * BM, &full[s]);
+            if (++s == S) { s = 0; ph ^= 1; }
         }
         issued_s = i;
     } else if (warp == 1 && lane == 0) {
-        constexpr uint32_t idesc = instr_desc(BM, BN);
+        const uint32_t idesc = instr_desc(BM, BN);
         int i = 0;
-        for (uint32_t s = 0, ph = 0; kb0 + i < kb1; ++i) {
-            if (!mbar_wait(&full[s], ph, &abort_flag)) {
-                abort_flag = 1;
-                atomicOr(p.ctl + kCtlStatus, kStatusTimeout);
-                break;
-            }
+        for (int s = 0, ph = 0; kb0 + i < kb1; ++i) {
+            if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
             tc_fence_after();
-            const uint32_t st = smem_addr(ring + (size_t)s * Sh::kStage);
+            const uint32_t st = smem_addr(ring + (size_t)s * p.stage_bytes);
 #pragma unroll
             for (int kk = 0; kk < BK / 16; ++kk)
-                mma_bf16(tmem, smem_desc(st + kk * 32), smem_desc(st + Sh::kA + kk * 32), idesc,
-                         (i | kk) ? 1u : 0u);
+                mma_bf16(tmem, smem_desc(st + kk * 32), smem_desc(st + kA + kk * 32), idesc, (i | kk) ? 1u : 0u);
             mma_commit(&empty[s]);
-            if (++s == (uint32_t)Sh::kStages) { s = 0; ph ^= 1u; }
+            if (++s == S) { s = 0; ph ^= 1; }
         }
         consumed_s = i;
         mma_commit(acc_full);
@@ -434,7 +735,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             float v[16];
             tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)c0, v);
             tmem_ld_wait();
-            const int h = h0 + c0;
+            const int h = d0 * BM + c0;
             if (!row_ok || h >= p.H) continue;
             float *dst = p.out + (size_t)m * p.H + h;
             const bool vec = h + 16 <= p.H;   // H is a multiple of 8: dst is 16-byte aligned
@@ -467,11 +768,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
     }
     __syncthreads();
-    if (abort_flag && threadIdx.x == 0) drain_after_abort(full, Sh::kStages, issued_s, consumed_s, acc_full);
+    if (abort_flag && threadIdx.x == 0) drain_after_abort(full, S, issued_s, consumed_s, acc_full);
     __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem, kTmemCols);
+        tmem_dealloc(tmem, 256);
     }
 }
 
@@ -507,6 +808,7 @@ __global__ void __launch_bounds__(512) keep_list_kernel(const uint8_t *__restric
     if (threadIdx.x == 0 && cnt) cnt[m] = base_s;
 }
 
+
 // ---------------------------------------------------------------------- host
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
 {
@@ -523,8 +825,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
-// bf16 matrix [rows][cols] with the given row stride, read in boxes of
-// box_rows x 64 with 128-byte swizzle.
+// bf16 matrix [rows][cols] with the given row stride (a multiple of 16 bytes),
+// read in boxes of box_rows x 64 with 128-byte swizzle.
 bool make_map(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols, uint64_t row_stride_bytes,
               uint32_t box_rows)
 {
@@ -540,47 +842,96 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols, 
 }
 
 // Raises the kernel's dynamic shared-memory limit once per device; `configured`
-// is the caller's flag word, one per kernel instantiation.
+// is the caller's flag word, one per kernel.
 template <typename K>
-cudaError_t set_smem(K kernel, size_t bytes, std::atomic<unsigned long long> &configured)
+cudaError_t set_smem(K kernel, std::atomic<unsigned long long> &configured)
 {
     int dev = 0;
     cudaGetDevice(&dev);
     const unsigned long long bit = 1ull << (dev & 63);
     if (configured.load() & bit) return cudaSuccess;
-    const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    const int bytes = kSmemBudget + 2048;
+    const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     if (e == cudaSuccess) configured.fetch_or(bit);
     return e;
 }
 
-template <int BN, bool SPLIT>
-cudaError_t launch_gu_t(const CUtensorMap &a, const CUtensorMap &a2, const CUtensorMap &g, const CUtensorMap &u,
-                        const GuParams &p, cudaStream_t stream)
+// Dynamic shared memory of a launch: the stage ring, 1 KB of alignment slack and the barriers.
+size_t smem_for(int stages, int stage_bytes) { return (size_t)stages * stage_bytes + 1024 + 256; }
+
+int stages_for(int stage_bytes)
 {
-    using Sh = GuShape<BN, SPLIT>;
-    static std::atomic<unsigned long long> configured{0};
-    cudaError_t e = set_smem(gu_kernel<BN, SPLIT>, Sh::kSmem, configured);
-    if (e != cudaSuccess) return e;
-    const dim3 grid((p.N + BN - 1) / BN, (p.M + BM - 1) / BM);
-    gu_kernel<BN, SPLIT><<<grid, kThreads, Sh::kSmem, stream>>>(a, a2, g, u, p);
-    return cudaGetLastError();
+    const int s = kSmemBudget / stage_bytes;
+    return s > kMaxStages ? kMaxStages : s;
 }
 
-template <int BN>
-cudaError_t launch_down_t(const CUtensorMap &a, const CUtensorMap &b, const DownParams &p, int splits,
-                          cudaStream_t stream)
+uint32_t tmem_cols_for(int cols)
 {
-    using Sh = DownShape<BN>;
-    static std::atomic<unsigned long long> configured{0};
-    cudaError_t e = set_smem(down_kernel<BN>, Sh::kSmem, configured);
-    if (e != cudaSuccess) return e;
-    const dim3 grid((p.H + BN - 1) / BN, (p.M + BM - 1) / BM, splits);
-    down_kernel<BN><<<grid, kThreads, Sh::kSmem, stream>>>(a, b, p);
-    return cudaGetLastError();
+    uint32_t c = 32;
+    while ((int)c < cols) c <<= 1;
+    return c;
+}
+
+int sm_count()
+{
+    static int by_dev[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    int &n = by_dev[dev & 63];
+    if (n == 0) cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    return n > 0 ? n : 1;
+}
+
+// Neurons per tile: the multiple of 16 (<= 128) that minimises waves x rows,
+// so that the neuron tiles cover the SMs in about one wave.
+int choose_rows(int N, int sms)
+{
+    int best = 16;
+    long long best_cost = -1;
+    for (int R = 16; R <= BM; R += 16) {
+        const long long tiles = (N + R - 1) / R;
+        const long long cost = ((tiles + sms - 1) / sms) * R;
+        if (best_cost < 0 || cost <= best_cost) {
+            best_cost = cost;
+            best = R;
+        }
+    }
+    return best;
 }
 
 }  // namespace
 }  // namespace tc
+
+cudaError_t tc_pack_layer(sats_layer *l, cudaStream_t stream)
+{
+    using namespace tc;
+    const int H = l->H, N = l->N;
+    l->tc_R = choose_rows(N, sm_count());
+    l->tc_T = (N + l->tc_R - 1) / l->tc_R;
+    l->tc_kbh = (H + BK - 1) / BK;
+    l->tc_dt = (H + BM - 1) / BM;
+    l->tc_kbn = (N + BK - 1) / BK;
+    l->ldn = (N + 7) & ~7;
+    const size_t gu_elems = (size_t)l->tc_T * l->tc_kbh * 2 * l->tc_R * BK;
+    const size_t wd_elems = (size_t)l->tc_dt * l->tc_kbn * BM * BK;
+    cudaError_t e = cudaMalloc(&l->gu_blk, gu_elems * 2);
+    if (e == cudaSuccess) e = cudaMalloc(&l->wd_blk, wd_elems * 2);
+    if (e != cudaSuccess) return e;
+    const size_t total8 = gu_elems / 8;
+    const size_t blocks = (total8 + 255) / 256;
+    pack_gu_kernel<<<(unsigned)(blocks < 8192 ? blocks : 8192), 256, 0, stream>>>(l->wg_t, l->w_ud, H, N, l->tc_R,
+                                                                                 l->tc_kbh, total8, l->gu_blk);
+    pack_wd_kernel<<<dim3(l->tc_kbn, l->tc_dt), 256, 0, stream>>>(l->w_ud, H, N, l->tc_kbn, l->wd_blk);
+    return cudaGetLastError();
+}
+
+cudaError_t tc_free_layer(sats_layer *l)
+{
+    const cudaError_t e1 = cudaFree(l->gu_blk);
+    const cudaError_t e2 = cudaFree(l->wd_blk);
+    l->gu_blk = l->wd_blk = nullptr;
+    return e1 != cudaSuccess ? e1 : e2;
+}
 
 namespace {
 struct TcLayout {
@@ -619,7 +970,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
                          int32_t *active_cnt, uint8_t *keep_trace, void *tc_ws, int *ctl, cudaStream_t stream)
 {
     using namespace tc;
-    const int H = layer->H, N = layer->N, ldn = layer->ldn;
+    const int H = layer->H, N = layer->N, ldn = layer->ldn, R = layer->tc_R;
     const TcLayout W = tc_layout(H, N, B);
     uint8_t *base = static_cast<uint8_t *>(tc_ws);
     uint16_t *xhi = reinterpret_cast<uint16_t *>(base + W.xhi);
@@ -627,70 +978,140 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
     uint16_t *hact = reinterpret_cast<uint16_t *>(base + W.hact);
     uint8_t *keep = base + W.keep;
     const int kstride = (N + 15) & ~15;
-
+    const int sms = sm_count();
     const bool split = x_mode != kXBf16;
-    const uint16_t *a_ptr = split ? xhi : static_cast<const uint16_t *>(x);
+    const uint16_t *xa = split ? xhi : static_cast<const uint16_t *>(x);
+    const uint64_t gu_rows = (uint64_t)layer->tc_T * layer->tc_kbh * 2 * R;
+    const uint64_t wd_rows = (uint64_t)layer->tc_dt * layer->tc_kbn * BM;
     cudaError_t e;
+
     if (split) {
         split_kernel<<<B, 256, 0, stream>>>(static_cast<const float *>(x), H,
                                             x_mode == kXResidNorm ? norm_w : nullptr, eps, xhi, xlo);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
-    // 96-neuron tiles give ~150 CTAs for N = 14336 at one token tile
-    const int bn = B <= BM ? 96 : 128;
-    CUtensorMap mA, mA2, mG, mU, mH, mD;
-    if (!make_map(&mA, a_ptr, B, H, (uint64_t)H * 2, BM) ||
-        !make_map(&mA2, split ? xlo : a_ptr, B, H, (uint64_t)H * 2, BM) ||
-        !make_map(&mG, layer->wg_t, N, H, (uint64_t)H * 2, bn) ||
-        !make_map(&mU, layer->w_ud, N, H, (uint64_t)H * 4, bn))
-        return cudaErrorInvalidValue;
-    GuParams gp{};
-    gp.M = B;
-    gp.N = N;
-    gp.H = H;
-    gp.t_l = t_l;
-    gp.dense_flags = dense_flags;
-    gp.hact = hact;
-    gp.ldh = ldn;
-    gp.keep = active_idx ? keep : nullptr;
-    gp.keep_stride = kstride;
-    gp.keep_trace = keep_trace;
-    gp.ctl = ctl;
-    if (bn == 96)
-        e = split ? launch_gu_t<96, true>(mA, mA2, mG, mU, gp, stream)
-                  : launch_gu_t<96, false>(mA, mA2, mG, mU, gp, stream);
-    else
-        e = split ? launch_gu_t<128, true>(mA, mA2, mG, mU, gp, stream)
-                  : launch_gu_t<128, false>(mA, mA2, mG, mU, gp, stream);
-    if (e != cudaSuccess) return e;
 
-    // down projection; split K (neurons) when the tile grid alone leaves SMs idle
-    const int dbn = B <= BM ? 128 : 256;
-    const int tiles = ((H + dbn - 1) / dbn) * ((B + BM - 1) / BM);
-    const int KB = (N + BK - 1) / BK;
-    int sms = 0, dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    int splits = tiles >= sms ? 1 : (sms + tiles - 1) / tiles;
-    if (splits > KB) splits = KB;
-    const int kbps = (KB + splits - 1) / splits;
-    splits = (KB + kbps - 1) / kbps;
-    if (!make_map(&mH, hact, B, N, (uint64_t)ldn * 2, BM) || !make_map(&mD, layer->wd_t, H, N, (uint64_t)ldn * 2, dbn))
-        return cudaErrorInvalidValue;
-    DownParams dp{};
-    dp.M = B;
-    dp.N = N;
-    dp.H = H;
-    dp.kb_per_split = kbps;
-    dp.atomic_out = splits > 1 ? 1 : 0;
-    dp.add_residual = out_mode == kOutResid ? 1 : 0;
-    dp.out = out;
-    dp.ctl = ctl;
-    if (splits > 1 && out_mode == kOutY) {
-        if ((e = cudaMemsetAsync(out, 0, (size_t)B * H * sizeof(float), stream)) != cudaSuccess) return e;
+    if (B <= kMaxSkinny) {
+        const int NT = (B + 15) & ~15;
+        CUtensorMap mW, mX, mX2, mWd, mH;
+        if (!make_map(&mW, layer->gu_blk, gu_rows, BK, kTileBytes, 2 * R) ||
+            !make_map(&mX, xa, B, H, (uint64_t)H * 2, NT) || !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, NT) ||
+            !make_map(&mWd, layer->wd_blk, wd_rows, BK, kTileBytes, BM) ||
+            !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, NT))
+            return cudaErrorInvalidValue;
+        if (out_mode == kOutY && (e = cudaMemsetAsync(out, 0, (size_t)B * H * sizeof(float), stream)) != cudaSuccess)
+            return e;
+
+        SkinnyGuParams gp{};
+        gp.M = B;
+        gp.N = N;
+        gp.R = R;
+        gp.KBh = layer->tc_kbh;
+        gp.NT = NT;
+        gp.split = split ? 1 : 0;
+        gp.t_l = t_l;
+        gp.dense_flags = dense_flags;
+        gp.hact = hact;
+        gp.ldh = ldn;
+        gp.keep = active_idx ? keep : nullptr;
+        gp.keep_stride = kstride;
+        gp.keep_trace = keep_trace;
+        gp.ctl = ctl;
+        const int rows_a = 2 * R > R + BM ? 2 * R : R + BM;   // the up tile's MMA reads 128 rows from row R
+        gp.a_bytes = (rows_a * kTileBytes + 1023) & ~1023;
+        gp.x_bytes = NT * kTileBytes;
+        gp.stage_bytes = gp.a_bytes + gp.x_bytes * (split ? 2 : 1);
+        gp.stages = stages_for(gp.stage_bytes);
+        gp.tmem_cols = tmem_cols_for(2 * NT);
+        static std::atomic<unsigned long long> cfg_gu{0};
+        if ((e = set_smem(gu_skinny_kernel, cfg_gu)) != cudaSuccess) return e;
+        gu_skinny_kernel<<<layer->tc_T, kThreads, smem_for(gp.stages, gp.stage_bytes), stream>>>(mW, mX, mX2, gp);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+
+        SkinnyDownParams dp{};
+        dp.M = B;
+        dp.H = H;
+        dp.NT = NT;
+        dp.KBn = layer->tc_kbn;
+        dp.units = layer->tc_dt * layer->tc_kbn;
+        dp.out = out;
+        dp.ctl = ctl;
+        dp.a_bytes = BM * kTileBytes;
+        dp.stage_bytes = dp.a_bytes + NT * kTileBytes;
+        dp.stages = stages_for(dp.stage_bytes);
+        dp.tmem_cols = tmem_cols_for(2 * NT);
+        static std::atomic<unsigned long long> cfg_dn{0};
+        if ((e = set_smem(down_skinny_kernel, cfg_dn)) != cudaSuccess) return e;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(dp.units < sms ? dp.units : sms);
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = smem_for(dp.stages, dp.stage_bytes);
+        cfg.stream = stream;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if ((e = cudaLaunchKernelEx(&cfg, down_skinny_kernel, mWd, mH, dp)) != cudaSuccess) return e;
+    } else {
+        CUtensorMap mX, mX2, mW, mH, mWd;
+        if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, BM) ||
+            !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, BM) ||
+            !make_map(&mW, layer->gu_blk, gu_rows, BK, kTileBytes, 2 * R) ||
+            !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, BM) ||
+            !make_map(&mWd, layer->wd_blk, wd_rows, BK, kTileBytes, BM))
+            return cudaErrorInvalidValue;
+        const int mtiles = (B + BM - 1) / BM;
+
+        WideGuParams gp{};
+        gp.M = B;
+        gp.N = N;
+        gp.R = R;
+        gp.KBh = layer->tc_kbh;
+        gp.split = split ? 1 : 0;
+        gp.t_l = t_l;
+        gp.dense_flags = dense_flags;
+        gp.hact = hact;
+        gp.ldh = ldn;
+        gp.keep = active_idx ? keep : nullptr;
+        gp.keep_stride = kstride;
+        gp.keep_trace = keep_trace;
+        gp.ctl = ctl;
+        gp.stage_bytes = BM * kTileBytes * (split ? 2 : 1) + 2 * R * kTileBytes;
+        gp.stages = stages_for(gp.stage_bytes);
+        static std::atomic<unsigned long long> cfg_gu{0};
+        if ((e = set_smem(gu_wide_kernel, cfg_gu)) != cudaSuccess) return e;
+        gu_wide_kernel<<<dim3(mtiles, layer->tc_T), kThreads, smem_for(gp.stages, gp.stage_bytes), stream>>>(
+            mX, mX2, mW, gp);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+
+        // down projection: 256 output columns per tile when the hidden tiles pair up;
+        // split K (neurons) when the tile grid alone leaves SMs idle
+        WideDownParams dp{};
+        dp.M = B;
+        dp.H = H;
+        dp.KBn = layer->tc_kbn;
+        dp.dtiles = (layer->tc_dt % 2 == 0) ? 2 : 1;
+        const int tiles = mtiles * (layer->tc_dt / dp.dtiles);
+        int splits = tiles >= sms ? 1 : (sms + tiles - 1) / tiles;
+        if (splits > dp.KBn) splits = dp.KBn;
+        dp.kb_per_split = (dp.KBn + splits - 1) / splits;
+        splits = (dp.KBn + dp.kb_per_split - 1) / dp.kb_per_split;
+        dp.atomic_out = splits > 1 ? 1 : 0;
+        dp.add_residual = out_mode == kOutResid ? 1 : 0;
+        dp.out = out;
+        dp.ctl = ctl;
+        dp.stage_bytes = BM * kTileBytes * (1 + dp.dtiles);
+        dp.stages = stages_for(dp.stage_bytes);
+        if (splits > 1 && out_mode == kOutY &&
+            (e = cudaMemsetAsync(out, 0, (size_t)B * H * sizeof(float), stream)) != cudaSuccess)
+            return e;
+        static std::atomic<unsigned long long> cfg_dn{0};
+        if ((e = set_smem(down_wide_kernel, cfg_dn)) != cudaSuccess) return e;
+        down_wide_kernel<<<dim3(mtiles, layer->tc_dt / dp.dtiles, splits), kThreads,
+                           smem_for(dp.stages, dp.stage_bytes), stream>>>(mH, mWd, dp);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
-    e = dbn == 128 ? launch_down_t<128>(mH, mD, dp, splits, stream) : launch_down_t<256>(mH, mD, dp, splits, stream);
-    if (e != cudaSuccess) return e;
     if (active_idx) {
         keep_list_kernel<<<B, 512, 0, stream>>>(keep, kstride, N, active_idx, active_cnt);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;

@@ -13,8 +13,17 @@ struct sats_layer {
     int device = 0;
     uint16_t *wg_t = nullptr;   // [N][H]: row j = column j of W_gate
     uint16_t *w_ud = nullptr;   // [N][2H]: row j = column j of W_up, then row j of W_down
-    uint16_t *wd_t = nullptr;   // [H][ldn]: row h = column h of W_down (tensor-core path)
-    int ldn = 0;                // N rounded up to a multiple of 8 (16-byte rows)
+    // Tensor-core path: the same weights cut into tiles of 64 K-elements whose
+    // rows (128 bytes each) are contiguous, so that one TMA box is one
+    // contiguous read.  Padding rows and columns are zero.
+    uint16_t *gu_blk = nullptr;   // [tc_T][tc_kbh][2][tc_R][64]: W_gate then W_up columns of neuron tile t
+    uint16_t *wd_blk = nullptr;   // [tc_dt][tc_kbn][128][64]: W_down columns of hidden tile d, neuron block kb
+    int tc_R = 0;                 // neurons per tile (a multiple of 16, at most 128)
+    int tc_T = 0;                 // neuron tiles, ceil(N / tc_R)
+    int tc_kbh = 0;               // ceil(H / 64)
+    int tc_dt = 0;                // hidden tiles, ceil(H / 128)
+    int tc_kbn = 0;               // ceil(N / 64)
+    int ldn = 0;                  // row stride of h (N rounded up to a multiple of 8)
 };
 
 namespace sats {
@@ -72,9 +81,13 @@ int fused_tokens_per_pass(int H);
 cudaError_t launch_fused(const FusedParams &p, cudaStream_t stream);
 
 cudaError_t launch_pack(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd, int H, int N,
-                        uint16_t *wg_t, uint16_t *w_ud, uint16_t *wd_t, int ldn, cudaStream_t stream);
+                        uint16_t *wg_t, uint16_t *w_ud, cudaStream_t stream);
 
 // Tensor-core path (gemm_tc.cu) for batches larger than one fused pass.
+// tc_pack_layer allocates and fills gu_blk / wd_blk from wg_t and w_ud;
+// tc_free_layer releases them.
+cudaError_t tc_pack_layer(sats_layer *layer, cudaStream_t stream);
+cudaError_t tc_free_layer(sats_layer *layer);
 bool use_tc_path(int H, int B);
 size_t tc_workspace_bytes(int H, int N, int B);
 cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int B, float t_l, const float *norm_w,
