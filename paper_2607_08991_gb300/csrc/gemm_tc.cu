@@ -184,14 +184,23 @@ __global__ void __launch_bounds__(256) split_kernel(const float *__restrict__ x,
 }
 
 // ---------------------------------------------------------------------- weight tiles
-// gu_blk[t][kb][g][r][c] = (g ? W_up : W_gate)[k][n] with n = t R + r,
-// k = kb 64 + c, read from wg_t [N][H] and the W_up half of w_ud [N][2H].
-// One thread per 8 consecutive c (16 bytes; H is a multiple of 8).
+// Tiles are stored exactly as the MMA reads them from shared memory: rows of
+// 128 bytes whose 16-byte chunks are permuted by the 128-byte swizzle (chunk c
+// of row r at position c ^ (r mod 8)), so that one bulk copy of a whole tile to
+// a 1024-byte aligned address yields a valid SWIZZLE_128B K-major operand.
+__device__ __forceinline__ size_t swizzled_chunk(size_t row_elem_base, int r, int chunk)
+{
+    return row_elem_base + (size_t)((chunk ^ (r & 7)) * 8);
+}
+
+// gu_blk[t][kb][g][r][.] holds (g ? W_up : W_gate)[k][n] for n = t R + r and
+// k = kb 64 + c at chunk c / 8 (swizzled), read from wg_t [N][H] and the W_up
+// half of w_ud [N][2H].  One thread per 16-byte chunk (H is a multiple of 8).
 __global__ void pack_gu_kernel(const uint16_t *__restrict__ wg_t, const uint16_t *__restrict__ w_ud, int H, int N,
                                int R, int KBh, size_t total8, uint16_t *__restrict__ dst)
 {
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total8; i += (size_t)gridDim.x * blockDim.x) {
-        const int c = (int)(i % 8) * 8;
+        const int chunk = (int)(i % 8), c = chunk * 8;
         size_t rest = i / 8;
         const int r = (int)(rest % R);
         rest /= R;
@@ -203,13 +212,15 @@ __global__ void pack_gu_kernel(const uint16_t *__restrict__ wg_t, const uint16_t
         uint4 v = make_uint4(0u, 0u, 0u, 0u);
         if (n < N && k < H)
             v = *reinterpret_cast<const uint4 *>(g ? w_ud + (size_t)n * 2 * H + k : wg_t + (size_t)n * H + k);
-        reinterpret_cast<uint4 *>(dst)[i] = v;
+        // row g R + r of the tile; R is a multiple of 16, so its swizzle phase is r mod 8
+        *reinterpret_cast<uint4 *>(dst + swizzled_chunk((i / 8) * BK, r, chunk)) = v;
     }
 }
 
-// wd_blk[d][kb][r][c] = W_down[n][h] with n = kb 64 + c, h = d 128 + r (W_down
-// row n is the second half of w_ud row n).  One CTA per (kb, d) tile, through
-// shared memory so that both sides are read and written in rows.
+// wd_blk[d][kb][r][.] holds W_down[n][h] for n = kb 64 + c, h = d 128 + r at
+// chunk c / 8 (swizzled); W_down row n is the second half of w_ud row n.  One
+// CTA per (kb, d) tile, through shared memory so that both sides are read and
+// written in rows.
 __global__ void __launch_bounds__(256) pack_wd_kernel(const uint16_t *__restrict__ w_ud, int H, int N, int KBn,
                                                       uint16_t *__restrict__ dst)
 {
@@ -222,11 +233,15 @@ __global__ void __launch_bounds__(256) pack_wd_kernel(const uint16_t *__restrict
     }
     __syncthreads();
     uint16_t *out = dst + ((size_t)d * KBn + kb) * BM * BK;
-    for (int i = threadIdx.x; i < BM * BK; i += 256) out[i] = tile[i % BK][i / BK];
+    for (int i = threadIdx.x; i < BM * BK; i += 256) {
+        const int r = i / BK, c = i % BK;
+        out[swizzled_chunk((size_t)r * BK, r, c / 8) + (c % 8)] = tile[c][r];
+    }
 }
 
 // ---------------------------------------------------------------------- skinny gate + up
 struct SkinnyGuParams {
+    const uint16_t *w;            // gu_blk
     int M, N, R, KBh, NT;
     int split;                    // 1: two B operands (bf16 hi and lo parts of fp32 x)
     float t_l;                    // threshold of sparse-path tokens
@@ -244,8 +259,8 @@ struct SkinnyGuParams {
 // One tile of R neurons (gate and up) against all M tokens: D[r][j] in TMEM
 // lane r, column j (gate) and NT + j (up).  Grid: tc_T CTAs.
 __global__ void __launch_bounds__(kThreads, 1)
-    gu_skinny_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
-                     const __grid_constant__ CUtensorMap tmX2, const SkinnyGuParams p)
+    gu_skinny_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmX2,
+                     const SkinnyGuParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *ring = align1024(smem_raw);
@@ -276,13 +291,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     grid_launch_dependents();   // the down projection may start prefetching its weights
 
     if (warp == 0 && lane == 0) {
-        const uint32_t load_bytes = (uint32_t)(2 * R * kTileBytes + p.x_bytes * (p.split ? 2 : 1));
+        const uint32_t w_bytes = (uint32_t)(2 * R * kTileBytes);
+        const uint32_t load_bytes = w_bytes + (uint32_t)(p.x_bytes * (p.split ? 2 : 1));
+        const uint64_t policy = l2_policy_evict_first();   // each weight tile is read by this CTA only
         int kb = 0;
         for (int s = 0, ph = 0; kb < p.KBh; ++kb) {
             if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
             uint8_t *st = ring + (size_t)s * p.stage_bytes;
             mbar_arrive_expect_tx(&full[s], load_bytes);
-            tma_load(st, &tmW, 0, (t * p.KBh + kb) * 2 * R, &full[s]);
+            bulk_load(st, p.w + (size_t)(t * p.KBh + kb) * 2 * R * BK, w_bytes, &full[s], policy);
             tma_load(st + p.a_bytes, &tmX, kb * BK, 0, &full[s]);
             if (p.split) tma_load(st + p.a_bytes + p.x_bytes, &tmX2, kb * BK, 0, &full[s]);
             if (++s == S) { s = 0; ph ^= 1; }
@@ -354,6 +371,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ---------------------------------------------------------------------- skinny down
 struct SkinnyDownParams {
+    const uint16_t *w;            // wd_blk
     int M, H, NT, KBn, units;     // units = tc_dt * KBn (hidden tile, neuron block) pairs
     float *out;                   // [M][H] fp32, added to with L2 reductions
     int *ctl;
@@ -364,10 +382,9 @@ struct SkinnyDownParams {
 // CTA c handles units [c U / G, (c+1) U / G) in order; consecutive units of one
 // hidden tile form a segment accumulated in TMEM (two buffers, so that the
 // epilogue of one segment overlaps the MMAs of the next) and added into y.
-// Unit u's weight tile starts at row u * 128 of wd_blk.
+// Unit u's weight tile is tile u of wd_blk.
 __global__ void __launch_bounds__(kThreads, 1)
-    down_skinny_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmH,
-                       const SkinnyDownParams p)
+    down_skinny_kernel(const __grid_constant__ CUtensorMap tmH, const SkinnyDownParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *ring = align1024(smem_raw);
@@ -406,12 +423,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = *tmem_slot;
 
     if (warp == 0 && lane == 0) {
-        const uint32_t load_bytes = (uint32_t)(BM * kTileBytes + NT * kTileBytes);
+        const uint32_t w_bytes = (uint32_t)(BM * kTileBytes);
+        const uint32_t load_bytes = w_bytes + (uint32_t)(NT * kTileBytes);
+        const uint64_t policy = l2_policy_evict_first();
         // the weight tiles do not depend on the preceding kernel: start them first
         const int npre = nu < S ? nu : S;
         for (int i = 0; i < npre; ++i) {
             mbar_arrive_expect_tx(&full[i], load_bytes);
-            tma_load(ring + (size_t)i * p.stage_bytes, &tmW, 0, (u0 + i) * BM, &full[i]);
+            bulk_load(ring + (size_t)i * p.stage_bytes, p.w + (size_t)(u0 + i) * BM * BK, w_bytes, &full[i], policy);
         }
         grid_dependency_wait();   // h is written by the preceding gate/up kernel
         int i = 0;
@@ -421,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (i >= npre) {
                 if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
                 mbar_arrive_expect_tx(&full[s], load_bytes);
-                tma_load(st, &tmW, 0, u * BM, &full[s]);
+                bulk_load(st, p.w + (size_t)u * BM * BK, w_bytes, &full[s], policy);
             }
             tma_load(st + p.a_bytes, &tmH, (u % KBn) * BK, 0, &full[s]);
             if (++s == S) { s = 0; ph ^= 1; }
@@ -499,6 +518,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ---------------------------------------------------------------------- wide gate + up
 struct WideGuParams {
+    const uint16_t *w;            // gu_blk
     int M, N, R, KBh;
     int split;
     float t_l;
@@ -517,7 +537,7 @@ struct WideGuParams {
 // weight tile are adjacent in launch order, so they read it from L2.
 __global__ void __launch_bounds__(kThreads, 1)
     gu_wide_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmX2,
-                   const __grid_constant__ CUtensorMap tmW, const WideGuParams p)
+                   const WideGuParams p)
 {
     constexpr int kA = BM * kTileBytes;
     extern __shared__ uint8_t smem_raw[];
@@ -557,7 +577,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_arrive_expect_tx(&full[s], load_bytes);
             tma_load(st, &tmX, kb * BK, m0, &full[s]);
             if (p.split) tma_load(st + kA, &tmX2, kb * BK, m0, &full[s]);
-            tma_load(st + wofs, &tmW, 0, (t * p.KBh + kb) * 2 * R, &full[s]);
+            bulk_load_shared(st + wofs, p.w + (size_t)(t * p.KBh + kb) * 2 * R * BK, (uint32_t)(2 * R * kTileBytes),
+                             &full[s]);
             if (++s == S) { s = 0; ph ^= 1; }
         }
         issued_s = kb;
@@ -649,6 +670,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ---------------------------------------------------------------------- wide down
 struct WideDownParams {
+    const uint16_t *w;    // wd_blk
     int M, H, KBn;
     int dtiles;           // 128-row hidden tiles per CTA tile (1 or 2: MMA N = 128 dtiles)
     int kb_per_split;     // K blocks of 64 neurons per split (blockIdx.z)
@@ -662,8 +684,7 @@ struct WideDownParams {
 // One 128-token x (128 dtiles)-column tile of Y = h W_down over one split of
 // the neuron range.  Grid: (ceil(M / 128), tc_dt / dtiles, splits).
 __global__ void __launch_bounds__(kThreads, 1)
-    down_wide_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmW,
-                     const WideDownParams p)
+    down_wide_kernel(const __grid_constant__ CUtensorMap tmH, const WideDownParams p)
 {
     constexpr int kA = BM * kTileBytes;
     extern __shared__ uint8_t smem_raw[];
@@ -706,7 +727,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_arrive_expect_tx(&full[s], load_bytes);
             tma_load(st, &tmH, kb * BK, m0, &full[s]);
             for (int q = 0; q < p.dtiles; ++q)
-                tma_load(st + kA + q * kA, &tmW, 0, ((d0 + q) * p.KBn + kb) * BM, &full[s]);
+                bulk_load_shared(st + kA + q * kA, p.w + ((size_t)(d0 + q) * p.KBn + kb) * BM * BK, (uint32_t)kA,
+                                 &full[s]);
             if (++s == S) { s = 0; ph ^= 1; }
         }
         issued_s = i;
@@ -981,8 +1003,6 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
     const int sms = sm_count();
     const bool split = x_mode != kXBf16;
     const uint16_t *xa = split ? xhi : static_cast<const uint16_t *>(x);
-    const uint64_t gu_rows = (uint64_t)layer->tc_T * layer->tc_kbh * 2 * R;
-    const uint64_t wd_rows = (uint64_t)layer->tc_dt * layer->tc_kbn * BM;
     cudaError_t e;
 
     if (split) {
@@ -993,16 +1013,15 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
 
     if (B <= kMaxSkinny) {
         const int NT = (B + 15) & ~15;
-        CUtensorMap mW, mX, mX2, mWd, mH;
-        if (!make_map(&mW, layer->gu_blk, gu_rows, BK, kTileBytes, 2 * R) ||
-            !make_map(&mX, xa, B, H, (uint64_t)H * 2, NT) || !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, NT) ||
-            !make_map(&mWd, layer->wd_blk, wd_rows, BK, kTileBytes, BM) ||
+        CUtensorMap mX, mX2, mH;
+        if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, NT) || !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, NT) ||
             !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, NT))
             return cudaErrorInvalidValue;
         if (out_mode == kOutY && (e = cudaMemsetAsync(out, 0, (size_t)B * H * sizeof(float), stream)) != cudaSuccess)
             return e;
 
         SkinnyGuParams gp{};
+        gp.w = layer->gu_blk;
         gp.M = B;
         gp.N = N;
         gp.R = R;
@@ -1025,10 +1044,11 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.tmem_cols = tmem_cols_for(2 * NT);
         static std::atomic<unsigned long long> cfg_gu{0};
         if ((e = set_smem(gu_skinny_kernel, cfg_gu)) != cudaSuccess) return e;
-        gu_skinny_kernel<<<layer->tc_T, kThreads, smem_for(gp.stages, gp.stage_bytes), stream>>>(mW, mX, mX2, gp);
+        gu_skinny_kernel<<<layer->tc_T, kThreads, smem_for(gp.stages, gp.stage_bytes), stream>>>(mX, mX2, gp);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
         SkinnyDownParams dp{};
+        dp.w = layer->wd_blk;
         dp.M = B;
         dp.H = H;
         dp.NT = NT;
@@ -1052,18 +1072,17 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         attr[0].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        if ((e = cudaLaunchKernelEx(&cfg, down_skinny_kernel, mWd, mH, dp)) != cudaSuccess) return e;
+        if ((e = cudaLaunchKernelEx(&cfg, down_skinny_kernel, mH, dp)) != cudaSuccess) return e;
     } else {
-        CUtensorMap mX, mX2, mW, mH, mWd;
+        CUtensorMap mX, mX2, mH;
         if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, BM) ||
             !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, BM) ||
-            !make_map(&mW, layer->gu_blk, gu_rows, BK, kTileBytes, 2 * R) ||
-            !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, BM) ||
-            !make_map(&mWd, layer->wd_blk, wd_rows, BK, kTileBytes, BM))
+            !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, BM))
             return cudaErrorInvalidValue;
         const int mtiles = (B + BM - 1) / BM;
 
         WideGuParams gp{};
+        gp.w = layer->gu_blk;
         gp.M = B;
         gp.N = N;
         gp.R = R;
@@ -1082,12 +1101,13 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         static std::atomic<unsigned long long> cfg_gu{0};
         if ((e = set_smem(gu_wide_kernel, cfg_gu)) != cudaSuccess) return e;
         gu_wide_kernel<<<dim3(mtiles, layer->tc_T), kThreads, smem_for(gp.stages, gp.stage_bytes), stream>>>(
-            mX, mX2, mW, gp);
+            mX, mX2, gp);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
         // down projection: 256 output columns per tile when the hidden tiles pair up;
         // split K (neurons) when the tile grid alone leaves SMs idle
         WideDownParams dp{};
+        dp.w = layer->wd_blk;
         dp.M = B;
         dp.H = H;
         dp.KBn = layer->tc_kbn;
@@ -1109,7 +1129,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         static std::atomic<unsigned long long> cfg_dn{0};
         if ((e = set_smem(down_wide_kernel, cfg_dn)) != cudaSuccess) return e;
         down_wide_kernel<<<dim3(mtiles, layer->tc_dt / dp.dtiles, splits), kThreads,
-                           smem_for(dp.stages, dp.stage_bytes), stream>>>(mH, mWd, dp);
+                           smem_for(dp.stages, dp.stage_bytes), stream>>>(mH, dp);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     if (active_idx) {
