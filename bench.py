@@ -9,6 +9,11 @@ Each call reads a different one of four device copies of the layer, so a copy
 is reused only after >= 420 MB of other weights have streamed (inputs larger
 than the 129 MB L2).
 
+The line also carries, under "batched", the same layer at decode-batch and
+prefill sizes (8, 64, 256 and 2048 tokens per call, 50 % threshold), which run
+on the tensor-core path: microseconds per call, tokens/s, weight-stream GB/s
+and dense-equivalent TFLOP/s against the measured bf16 peak.
+
 Prints one JSON line.  `--impl reference` times the CPU oracle instead (the
 reference arm of this comparison), on a bounded sample of the same workload.
 """
@@ -39,6 +44,7 @@ N_CALIB = 256
 FUSED_SRC = os.path.join(ROOT, "paper_2607_08991_gb300", "csrc", "fused_mlp.cu")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fused_mlp_llama_layer_b1.md")
 NOMINAL_HBM_GBS = 8000.0
+BATCHES = (8, 64, 256, 2048)
 
 
 def _peaks():
@@ -48,6 +54,15 @@ def _peaks():
         return float(pk["hbm_gbs"]), "measured"
     except Exception:
         return 6800.0, "fallback"
+
+
+def _bf16_peak():
+    """Dense bf16 tensor peak (TFLOP/s): the measured burst figure, else the fallback."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
 
 
 def _src_hash(path):
@@ -211,7 +226,7 @@ def run_gpu(args):
     H, N = inputs.LLAMA_H, inputs.LLAMA_N
     stream = torch.cuda.Stream(device=dev)
     w = inputs.mlp_weights(H, N)
-    copies = 1 if args.profile else LAYER_COPIES
+    copies = 1 if (args.profile or args.profile_batch) else LAYER_COPIES
     with torch.cuda.stream(stream):
         src = [torch.from_numpy(m.view(np.int16)).to(dev) for m in (w.Wg, w.Wu, w.Wd)]
         layers = [sats.Layer(*src, stream=stream) for _ in range(copies)]
@@ -229,6 +244,25 @@ def run_gpu(args):
         idx = torch.empty(1, N, dtype=torch.int32, device=dev)
         cnt = torch.empty(1, dtype=torch.int32, device=dev)
     stream.synchronize()
+
+    if args.profile_batch:
+        # small capture case for ncu: one layer copy, `steps` calls at one batch size
+        B = args.profile_batch
+        xb = torch.randn(B, H, device=dev, dtype=torch.float32).to(torch.bfloat16).view(torch.int16)
+        yb = torch.empty(B, H, dtype=torch.float32, device=dev)
+        wsb = sats.Workspace(H, N, B, device=dev, stream=stream)
+        for i in range(max(args.warmup, 1) + args.steps):
+            sats.sparse_mlp(layers[0], xb, ts[0], yb, wsb, stream=stream)
+        stream.synchronize()
+        ok = sats.get_error(wsb, stream=stream) == sats.OK
+        if rank == 0:
+            print(json.dumps({"profile_case": "llama_layer_4096x14336_b%d" % B, "calls": max(args.warmup, 1) + args.steps,
+                              "tensor_cores": sats.uses_tensor_cores(H, B), "status_ok": ok}))
+        for l in layers:
+            l.close()
+        if not ok:
+            raise RuntimeError("device status after the profile calls")
+        return
 
     calls = [(i, ts[i]) for i in range(len(SPARSITY))]
     copy = [0]
@@ -307,6 +341,34 @@ def run_gpu(args):
     d1.synchronize()
     dense_us = 1e3 * d0.elapsed_time(d1) / K
 
+    # batched decode and prefill on the tensor-core path (50 % threshold), same rotating copies
+    batched = {}
+    if not args.no_batched:
+        bf16_peak, bf16_kind = _bf16_peak()
+        for B in BATCHES:
+            xb = torch.randn(B, H, device=dev, dtype=torch.float32).to(torch.bfloat16).view(torch.int16)
+            yb = torch.empty(B, H, dtype=torch.float32, device=dev)
+            wsb = sats.Workspace(H, N, B, device=dev, stream=stream)
+            Kb = max(4, min(K, int(4e4 / (60 + 0.33 * B))))
+            for i in range(3):
+                sats.sparse_mlp(layers[i % len(layers)], xb, ts[0], yb, wsb, stream=stream)
+            b0, b1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            b0.record(stream)
+            for i in range(Kb):
+                sats.sparse_mlp(layers[i % len(layers)], xb, ts[0], yb, wsb, stream=stream)
+            b1.record(stream)
+            b1.synchronize()
+            if sats.get_error(wsb, stream=stream) != sats.OK:
+                raise RuntimeError("device status after the batched calls")
+            us = 1e3 * b0.elapsed_time(b1) / Kb
+            wbytes = 6.0 * H * N + B * H * 2.0 + B * H * 4.0
+            flops = 6.0 * B * H * N
+            batched[str(B)] = {"us_per_call": us, "tokens_per_s": B / (us * 1e-6),
+                               "hbm_gbs": wbytes / (us * 1e-6) / 1e9, "tflops": flops / (us * 1e-6) / 1e12,
+                               "tensor_frac_of_%s" % bf16_kind: flops / (us * 1e-6) / 1e12 / bf16_peak,
+                               "calls": Kb, "path": "tensor cores" if sats.uses_tensor_cores(H, B) else "fused"}
+            del xb, yb, wsb
+
     # end to end through the C ABI with host buffers: x host->device, y and count device->host
     xh = torch.from_numpy(inputs.activations_bf16(1, H).view(np.int16)).pin_memory()
     yh = torch.empty(1, H, dtype=torch.float32).pin_memory()
@@ -362,6 +424,7 @@ def run_gpu(args):
                        "parallelism": "replicas" if world > 1 else "single"},
             "per_sparsity": per,
             "dense": {"us": dense_us},
+            "batched": batched,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                          "frac": achieved / hbm_peak, "peak_kind": peak_kind,
                          "traffic": None if traffic is None else
@@ -390,11 +453,15 @@ def main():
     ap.add_argument("--impl", default="sats", choices=["sats", "reference"])
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-batched", action="store_true", help="skip the batched tensor-core measurements")
+    ap.add_argument("--profile-batch", type=int, default=0,
+                    help="small capture case for ncu: `warmup + steps` calls at this batch size on one layer copy")
     ap.add_argument("--profile", action="store_true",
                     help="small capture case for ncu: one layer copy, timed calls only, no CPU baseline")
     args = ap.parse_args()
-    if args.profile:
+    if args.profile or args.profile_batch:
         args.no_cpu_baseline = True
+        args.no_batched = True
     if args.impl == "reference":
         run_reference(args)
     else:

@@ -34,6 +34,7 @@
 #include <atomic>
 #include <cmath>
 #include <mutex>
+#include <utility>
 
 #include "common.cuh"
 #include "internal.h"
@@ -45,7 +46,7 @@ namespace {
 constexpr int BM = 128;              // MMA M: rows of the A operand
 constexpr int BK = 64;               // K per TMA box: one 128-byte swizzle row of bf16
 constexpr int kThreads = 192;
-constexpr int kSmemBudget = 196608;  // stage ring
+constexpr int kSmemBudget = 196608;  // stage ring (one CTA per SM)
 constexpr int kMaxStages = 8;
 constexpr int kMaxSkinny = 256;      // largest batch on the skinny orientation (MMA N <= 256)
 constexpr int kTileBytes = BK * 2;   // bytes of one tile row
@@ -160,6 +161,8 @@ __device__ __forceinline__ void set_timeout(int *ctl, volatile int *abort_flag)
 __global__ void __launch_bounds__(256) split_kernel(const float *__restrict__ x, int H, const float *__restrict__ w,
                                                     float eps, uint16_t *__restrict__ hi, uint16_t *__restrict__ lo)
 {
+    grid_dependency_wait();   // x may be the residual written by the preceding kernel
+    grid_launch_dependents();
     const int m = blockIdx.x;
     const float *xr = x + (size_t)m * H;
     __shared__ float red[8];
@@ -252,7 +255,10 @@ struct SkinnyGuParams {
     int keep_stride;
     uint8_t *keep_trace;          // [M][N] or nullptr
     int *ctl;
+    float *zero;                  // y [M][H] to clear for the down projection's additions, or nullptr
+    int zero_count;               // M H (a multiple of 8)
     int stages, stage_bytes, a_bytes, x_bytes;
+    int ring_bytes;               // stages * stage_bytes + room for the last up tile's 128-row read
     uint32_t tmem_cols;
 };
 
@@ -264,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *ring = align1024(smem_raw);
-    uint64_t *full = reinterpret_cast<uint64_t *>(ring + (size_t)p.stages * p.stage_bytes);
+    uint64_t *full = reinterpret_cast<uint64_t *>(ring + p.ring_bytes);
     uint64_t *empty = full + kMaxStages;
     uint64_t *acc_full = empty + kMaxStages;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_full + 1);
@@ -294,17 +300,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t w_bytes = (uint32_t)(2 * R * kTileBytes);
         const uint32_t load_bytes = w_bytes + (uint32_t)(p.x_bytes * (p.split ? 2 : 1));
         const uint64_t policy = l2_policy_evict_first();   // each weight tile is read by this CTA only
+        // the weight tiles do not depend on the preceding kernel: start them before waiting for it
+        const int npre = p.KBh < S ? p.KBh : S;
+        for (int i = 0; i < npre; ++i) {
+            mbar_arrive_expect_tx(&full[i], load_bytes);
+            bulk_load(ring + (size_t)i * p.stage_bytes, p.w + (size_t)(t * p.KBh + i) * 2 * R * BK, w_bytes, &full[i],
+                      policy);
+        }
+        grid_dependency_wait();   // x (and this call's buffers) may belong to the preceding kernel
         int kb = 0;
         for (int s = 0, ph = 0; kb < p.KBh; ++kb) {
-            if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
             uint8_t *st = ring + (size_t)s * p.stage_bytes;
-            mbar_arrive_expect_tx(&full[s], load_bytes);
-            bulk_load(st, p.w + (size_t)(t * p.KBh + kb) * 2 * R * BK, w_bytes, &full[s], policy);
+            if (kb >= npre) {
+                if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
+                mbar_arrive_expect_tx(&full[s], load_bytes);
+                bulk_load(st, p.w + (size_t)(t * p.KBh + kb) * 2 * R * BK, w_bytes, &full[s], policy);
+            }
             tma_load(st + p.a_bytes, &tmX, kb * BK, 0, &full[s]);
             if (p.split) tma_load(st + p.a_bytes + p.x_bytes, &tmX2, kb * BK, 0, &full[s]);
             if (++s == S) { s = 0; ph ^= 1; }
         }
-        issued_s = kb;
+        issued_s = kb;   // a break happens only before stage kb's loads are issued (kb >= npre)
     } else if (warp == 1 && lane == 0) {
         const uint32_t idesc = instr_desc(BM, NT);
         int kb = 0;
@@ -333,6 +349,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         consumed_s = kb;
         mma_commit(acc_full);
     } else if (warp >= 2) {
+        grid_dependency_wait();   // y, h and the keep bytes may still be in use by the preceding kernel
+        if (p.zero) {
+            // this CTA's share of y, cleared for the down projection's additions
+            const int per = (((p.zero_count + (int)gridDim.x - 1) / (int)gridDim.x) + 7) & ~7;
+            const int z0 = (int)blockIdx.x * per, z1 = min(p.zero_count, z0 + per);
+            float4 *z = reinterpret_cast<float4 *>(p.zero);
+            for (int i = z0 / 4 + (int)threadIdx.x - 64; i < z1 / 4; i += 128) z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
         // epilogue: thread = neuron r of the tile, columns = tokens
         const bool ok = mbar_wait(acc_full, 0u, &abort_flag);
         tc_fence_after();
@@ -421,6 +445,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    grid_launch_dependents();   // the next call's kernels may start their prologue as SMs free up
 
     if (warp == 0 && lane == 0) {
         const uint32_t w_bytes = (uint32_t)(BM * kTileBytes);
@@ -803,6 +828,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 __global__ void __launch_bounds__(512) keep_list_kernel(const uint8_t *__restrict__ keep, int stride, int N,
                                                         int32_t *__restrict__ idx, int32_t *__restrict__ cnt)
 {
+    grid_dependency_wait();   // the keep bytes are written by the preceding kernel
+    grid_launch_dependents();
     const int m = blockIdx.x;
     const uint8_t *k = keep + (size_t)m * stride;
     __shared__ int warp_sums[16];
@@ -878,12 +905,48 @@ cudaError_t set_smem(K kernel, std::atomic<unsigned long long> &configured)
     return e;
 }
 
+// Launch with programmatic dependent launch: the kernel may start while the
+// preceding kernel in the stream finishes; it calls griddepcontrol.wait before
+// touching anything that kernel produces.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, size_t smem, cudaStream_t stream, Args &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// As launch_pdl, for the small kernels (no dynamic shared memory, `threads` per CTA).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl_threads(void (*kernel)(KArgs...), dim3 grid, int threads, cudaStream_t stream, Args &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // Dynamic shared memory of a launch: the stage ring, 1 KB of alignment slack and the barriers.
 size_t smem_for(int stages, int stage_bytes) { return (size_t)stages * stage_bytes + 1024 + 256; }
 
-int stages_for(int stage_bytes)
+int stages_for(int stage_bytes, int budget = kSmemBudget)
 {
-    const int s = kSmemBudget / stage_bytes;
+    const int s = budget / stage_bytes;
     return s > kMaxStages ? kMaxStages : s;
 }
 
@@ -1006,9 +1069,9 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
     cudaError_t e;
 
     if (split) {
-        split_kernel<<<B, 256, 0, stream>>>(static_cast<const float *>(x), H,
-                                            x_mode == kXResidNorm ? norm_w : nullptr, eps, xhi, xlo);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        e = launch_pdl_threads(split_kernel, dim3(B), 256, stream, static_cast<const float *>(x), H,
+                               x_mode == kXResidNorm ? norm_w : nullptr, eps, xhi, xlo);
+        if (e != cudaSuccess) return e;
     }
 
     if (B <= kMaxSkinny) {
@@ -1017,9 +1080,6 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, NT) || !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, NT) ||
             !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, NT))
             return cudaErrorInvalidValue;
-        if (out_mode == kOutY && (e = cudaMemsetAsync(out, 0, (size_t)B * H * sizeof(float), stream)) != cudaSuccess)
-            return e;
-
         SkinnyGuParams gp{};
         gp.w = layer->gu_blk;
         gp.M = B;
@@ -1036,16 +1096,23 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.keep_stride = kstride;
         gp.keep_trace = keep_trace;
         gp.ctl = ctl;
-        const int rows_a = 2 * R > R + BM ? 2 * R : R + BM;   // the up tile's MMA reads 128 rows from row R
-        gp.a_bytes = (rows_a * kTileBytes + 1023) & ~1023;
+        gp.zero = out_mode == kOutY ? out : nullptr;   // the down projection adds into y
+        gp.zero_count = B * H;
+        // stage: gate + up rows, then the token tile(s).  The up tile's MMA reads 128 rows from
+        // row R; past 2R they are other data of the ring (rows R..127 of D are not used), and the
+        // ring ends with enough room for the last stage's read.
+        gp.a_bytes = 2 * R * kTileBytes;
         gp.x_bytes = NT * kTileBytes;
         gp.stage_bytes = gp.a_bytes + gp.x_bytes * (split ? 2 : 1);
-        gp.stages = stages_for(gp.stage_bytes);
+        const int over = (R + BM) * kTileBytes - gp.stage_bytes;
+        const int slack = over > 0 ? ((over + 1023) & ~1023) : 0;
+        gp.stages = stages_for(gp.stage_bytes, kSmemBudget - slack);
+        gp.ring_bytes = gp.stages * gp.stage_bytes + slack;
         gp.tmem_cols = tmem_cols_for(2 * NT);
         static std::atomic<unsigned long long> cfg_gu{0};
         if ((e = set_smem(gu_skinny_kernel, cfg_gu)) != cudaSuccess) return e;
-        gu_skinny_kernel<<<layer->tc_T, kThreads, smem_for(gp.stages, gp.stage_bytes), stream>>>(mX, mX2, gp);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        e = launch_pdl(gu_skinny_kernel, dim3(layer->tc_T), smem_for(1, gp.ring_bytes), stream, mX, mX2, gp);
+        if (e != cudaSuccess) return e;
 
         SkinnyDownParams dp{};
         dp.w = layer->wd_blk;
@@ -1062,17 +1129,9 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         dp.tmem_cols = tmem_cols_for(2 * NT);
         static std::atomic<unsigned long long> cfg_dn{0};
         if ((e = set_smem(down_skinny_kernel, cfg_dn)) != cudaSuccess) return e;
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(dp.units < sms ? dp.units : sms);
-        cfg.blockDim = dim3(kThreads);
-        cfg.dynamicSmemBytes = smem_for(dp.stages, dp.stage_bytes);
-        cfg.stream = stream;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr[0].val.programmaticStreamSerializationAllowed = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        if ((e = cudaLaunchKernelEx(&cfg, down_skinny_kernel, mH, dp)) != cudaSuccess) return e;
+        e = launch_pdl(down_skinny_kernel, dim3(dp.units < sms ? dp.units : sms), smem_for(dp.stages, dp.stage_bytes),
+                       stream, mH, dp);
+        if (e != cudaSuccess) return e;
     } else {
         CUtensorMap mX, mX2, mH;
         if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, BM) ||
@@ -1133,8 +1192,9 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     if (active_idx) {
-        keep_list_kernel<<<B, 512, 0, stream>>>(keep, kstride, N, active_idx, active_cnt);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        e = launch_pdl_threads(keep_list_kernel, dim3(B), 512, stream, static_cast<const uint8_t *>(keep), kstride, N,
+                               active_idx, active_cnt);
+        if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
 }
