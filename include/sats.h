@@ -165,6 +165,13 @@ SATS_API sats_status sats_sparse_mlp_fixed_scratch(const sats_layer *layer, cons
  */
 SATS_API int sats_uses_tensor_cores(int H, int B);
 
+/*
+ * sats_last_cuda_error -- text of the CUDA error behind the most recent
+ * SATS_ECUDA returned on the calling host thread, with the step that failed
+ * (a static or thread-local string, valid until the thread's next call).
+ */
+SATS_API const char *sats_last_cuda_error(void);
+
 /* As sats_sparse_mlp, with fp32 activations x: device fp32 [B][H]. */
 SATS_API sats_status sats_sparse_mlp_f32(const sats_layer *layer, const float *x, int B, float t_l,
                                 float *y, int32_t *active_idx, int32_t *active_cnt,

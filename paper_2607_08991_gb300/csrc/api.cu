@@ -2,6 +2,7 @@
 // workspace layout, and the host-side drivers that split a batch into passes
 // of the fused kernel and chain the blocks of a stack.
 #include <cmath>
+#include <cstdio>
 #include <cstring>
 #include <mutex>
 #include <new>
@@ -35,7 +36,21 @@ WsLayout ws_layout(int H, int N, int B)
 
 static bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-static sats_status from_cuda(cudaError_t e) { return e == cudaSuccess ? SATS_OK : SATS_ECUDA; }
+static thread_local cudaError_t g_last_cuda = cudaSuccess;
+static thread_local const char *g_last_where = nullptr;
+static thread_local char g_last_text[256];
+
+sats_status cuda_fail(cudaError_t e, const char *where)
+{
+    g_last_cuda = e;
+    g_last_where = where;
+    return SATS_ECUDA;
+}
+
+static sats_status from_cuda(cudaError_t e, const char *where = "CUDA call")
+{
+    return e == cudaSuccess ? SATS_OK : cuda_fail(e, where);
+}
 
 static bool bad_threshold(float t) { return std::isnan(t) || t < 0.0f; }
 
@@ -54,7 +69,7 @@ static sats_status run_layer(const sats_layer *layer, int x_mode, const void *x,
         const cudaError_t e = run_tc_layer(layer, x_mode, x, B, *t_per_pass_l, norm_w, eps, dense_flags, out_mode,
                                            out, active_idx, active_cnt, keep_trace, base + L.tc,
                                            reinterpret_cast<int *>(base + L.ctl), stream);
-        return e == cudaSuccess ? SATS_OK : SATS_ECUDA;
+        return e == cudaSuccess ? SATS_OK : SATS_ECUDA;   // run_tc_layer recorded the failing step
     }
     const int per_pass = fused_tokens_per_pass(H);
     const size_t x_elem = (x_mode == kXBf16) ? 2 : 4;
@@ -80,7 +95,7 @@ static sats_status run_layer(const sats_layer *layer, int x_mode, const void *x,
         p.active_cnt = active_cnt ? active_cnt + b0 : nullptr;
         p.keep_trace = keep_trace ? keep_trace + (size_t)b0 * N : nullptr;
         const cudaError_t e = launch_fused(p, stream);
-        if (e != cudaSuccess) return SATS_ECUDA;
+        if (e != cudaSuccess) return cuda_fail(e, "fused kernel launch");
     }
     return SATS_OK;
 }
@@ -163,7 +178,7 @@ sats_status sats_layer_create(const void *W_gate, const void *W_up, const void *
     if (!W_gate || !W_up || !W_down) return SATS_EINVAL;
     if (H < 8 || H > kMaxH || (H % 8) != 0 || N < 1 || N > kMaxN) return SATS_ESHAPE;
     sats_layer *l = new (std::nothrow) sats_layer();
-    if (!l) return SATS_ECUDA;
+    if (!l) return cuda_fail(cudaErrorMemoryAllocation, "host allocation");
     l->H = H;
     l->N = N;
     cudaGetDevice(&l->device);
@@ -181,7 +196,7 @@ sats_status sats_layer_create(const void *W_gate, const void *W_up, const void *
         cudaFree(l->w_ud);
         tc_free_layer(l);
         delete l;
-        return SATS_ECUDA;
+        return cuda_fail(e, "layer allocation or repacking");
     }
     *out = l;
     return SATS_OK;
@@ -195,7 +210,9 @@ sats_status sats_layer_destroy(sats_layer *layer)
     const cudaError_t e2 = cudaFree(layer->w_ud);
     const cudaError_t e3 = tc_free_layer(layer);
     delete layer;
-    return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess) ? SATS_OK : SATS_ECUDA;
+    if (e1 != cudaSuccess) return cuda_fail(e1, "cudaFree");
+    if (e2 != cudaSuccess) return cuda_fail(e2, "cudaFree");
+    return from_cuda(e3, "cudaFree");
 }
 
 sats_status sats_layer_shape(const sats_layer *layer, int *H, int *N)
@@ -234,15 +251,23 @@ sats_status sats_sparse_mlp_fixed_scratch(const sats_layer *layer, const void *x
     if (B == 0) return SATS_OK;
     if (!x || !y || !aligned16(x) || !aligned16(y)) return SATS_EINVAL;
     void *ws = fixed_scratch_current_device();
-    if (!ws) return SATS_ECUDA;
+    if (!ws) return cuda_fail(cudaErrorInvalidSymbol, "fixed scratch lookup");
     // the array keeps the previous call's contents: the control words
     // (scheduling counters, status) must start at zero
-    if (cudaMemsetAsync(ws, 0, kCtlInts * sizeof(int), static_cast<cudaStream_t>(stream)) != cudaSuccess)
-        return SATS_ECUDA;
+    const cudaError_t ez = cudaMemsetAsync(ws, 0, kCtlInts * sizeof(int), static_cast<cudaStream_t>(stream));
+    if (ez != cudaSuccess) return cuda_fail(ez, "fixed scratch clear");
     return sparse_common(layer, kXBf16, x, B, t_l, y, active_idx, active_cnt, ws, kFixedScratchBytes, stream);
 }
 
 int sats_uses_tensor_cores(int H, int B) { return use_tc_path(H, B) ? 1 : 0; }
+
+const char *sats_last_cuda_error(void)
+{
+    if (g_last_cuda == cudaSuccess) return "no CUDA error recorded";
+    snprintf(g_last_text, sizeof g_last_text, "%s: %s (%s)", g_last_where ? g_last_where : "CUDA call",
+             cudaGetErrorString(g_last_cuda), cudaGetErrorName(g_last_cuda));
+    return g_last_text;
+}
 
 sats_status sats_sparse_mlp_f32(const sats_layer *layer, const float *x, int B, float t_l, float *y,
                                 int32_t *active_idx, int32_t *active_cnt, void *ws, size_t ws_bytes, void *stream)
@@ -291,7 +316,7 @@ sats_status sats_mlp_stack(const sats_layer *const *layers, const float *const *
         flags = reinterpret_cast<uint8_t *>(base + W.route_flags);
         cudaError_t e = launch_route(token_ids, B, lut, V, reinterpret_cast<int32_t *>(base + W.route_perm),
                                      ctl + kCtlNDense, flags, ctl + kCtlStatus, st);
-        if (e != cudaSuccess) return SATS_ECUDA;
+        if (e != cudaSuccess) return cuda_fail(e, "route kernel launch");
     }
     for (int l = 0; l < L; ++l) {
         s = run_layer(layers[l], kXResidNorm, x, B, &t[l], norm_w[l], eps, flags, kOutResid, x, nullptr, nullptr,
@@ -339,7 +364,7 @@ static sats_status read_status(int32_t *word, cudaStream_t st)
     cudaError_t e = cudaStreamSynchronize(st);
     if (e == cudaSuccess) e = cudaMemcpy(&v, word, sizeof v, cudaMemcpyDeviceToHost);
     if (e == cudaSuccess && v != 0) e = cudaMemset(word, 0, sizeof v);
-    if (e != cudaSuccess) return SATS_ECUDA;
+    if (e != cudaSuccess) return cuda_fail(e, "status read");
     if (v & kStatusTimeout) return SATS_ETIMEOUT;
     if (v & kStatusBadToken) return SATS_EDEVICE;
     return SATS_OK;

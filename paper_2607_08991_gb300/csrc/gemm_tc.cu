@@ -47,6 +47,7 @@ constexpr int BM = 128;              // MMA M: rows of the A operand
 constexpr int BK = 64;               // K per TMA box: one 128-byte swizzle row of bf16
 constexpr int kThreads = 192;
 constexpr int kSmemBudget = 196608;  // stage ring (one CTA per SM)
+constexpr int kSmemWide = 225280;    // stage ring of the persistent prefill kernels, at most
 constexpr int kMaxStages = 8;
 constexpr int kMaxSkinny = 256;      // largest batch on the skinny orientation (MMA N <= 256)
 constexpr int kTileBytes = BK * 2;   // bytes of one tile row
@@ -545,6 +546,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 struct WideGuParams {
     const uint16_t *w;            // gu_blk
     int M, N, R, KBh;
+    int mtiles, tiles;            // token tiles; tiles = mtiles * tc_T
     int split;
     float t_l;
     const uint8_t *dense_flags;
@@ -555,11 +557,15 @@ struct WideGuParams {
     uint8_t *keep_trace;
     int *ctl;
     int stages, stage_bytes;
+    uint32_t tmem_cols;           // two accumulator buffers of 2R columns
 };
 
-// One 128-token x R-neuron tile of G and U: D[m][c] in TMEM lane m, column c
-// (gate) and R + c (up).  Grid: (ceil(M / 128), tc_T); the token tiles of one
-// weight tile are adjacent in launch order, so they read it from L2.
+// Persistent: CTA c takes tiles c, c + G, c + 2G, ... of 128 tokens x R
+// neurons; tile q covers token tile q mod mtiles of neuron tile q / mtiles, so
+// the CTAs running together share few weight tiles and read them through L2.
+// Per tile, D[m][c] accumulates in TMEM lane m, column b 2R + c (gate) and
+// b 2R + R + c (up), b alternating between tiles so that one tile's epilogue
+// overlaps the next tile's MMAs; the load ring runs across tile boundaries.
 __global__ void __launch_bounds__(kThreads, 1)
     gu_wide_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmX2,
                    const WideGuParams p)
@@ -569,11 +575,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t *ring = align1024(smem_raw);
     uint64_t *full = reinterpret_cast<uint64_t *>(ring + (size_t)p.stages * p.stage_bytes);
     uint64_t *empty = full + kMaxStages;
-    uint64_t *acc_full = empty + kMaxStages;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_full + 1);
+    uint64_t *acc_full = empty + kMaxStages;   // [2]
+    uint64_t *acc_empty = acc_full + 2;        // [2]
+    uint64_t *mma_done = acc_empty + 2;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mma_done + 1);
     __shared__ int abort_flag, issued_s, consumed_s;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * BM, t = blockIdx.y, R = p.R, S = p.stages;
+    const int R = p.R, S = p.stages, KBh = p.KBh;
     const int wofs = kA * (p.split ? 2 : 1);
 
     if (threadIdx.x == 0) {
@@ -581,13 +589,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
-        mbar_init(acc_full, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], 128);
+        }
+        mbar_init(mma_done, 1);
         abort_flag = 0;
         issued_s = 0;
         consumed_s = 0;
         mbar_init_fence();
     }
-    if (warp == 1) tmem_alloc(tmem_slot, 256);
+    if (warp == 1) tmem_alloc(tmem_slot, p.tmem_cols);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -595,101 +607,137 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp == 0 && lane == 0) {
         const uint32_t load_bytes = (uint32_t)(wofs + 2 * R * kTileBytes);
-        int kb = 0;
-        for (int s = 0, ph = 0; kb < p.KBh; ++kb) {
-            if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
-            uint8_t *st = ring + (size_t)s * p.stage_bytes;
-            mbar_arrive_expect_tx(&full[s], load_bytes);
-            tma_load(st, &tmX, kb * BK, m0, &full[s]);
-            if (p.split) tma_load(st + kA, &tmX2, kb * BK, m0, &full[s]);
-            bulk_load_shared(st + wofs, p.w + (size_t)(t * p.KBh + kb) * 2 * R * BK, (uint32_t)(2 * R * kTileBytes),
-                             &full[s]);
-            if (++s == S) { s = 0; ph ^= 1; }
+        int i = 0, s = 0, ph = 0;
+        bool stop = false;
+        for (int q = blockIdx.x; q < p.tiles && !stop; q += gridDim.x) {
+            const int m0 = (q % p.mtiles) * BM, t = q / p.mtiles;
+            for (int kb = 0; kb < KBh; ++kb, ++i) {
+                if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) {
+                    set_timeout(p.ctl, &abort_flag);
+                    stop = true;
+                    break;
+                }
+                uint8_t *st = ring + (size_t)s * p.stage_bytes;
+                mbar_arrive_expect_tx(&full[s], load_bytes);
+                tma_load(st, &tmX, kb * BK, m0, &full[s]);
+                if (p.split) tma_load(st + kA, &tmX2, kb * BK, m0, &full[s]);
+                bulk_load_shared(st + wofs, p.w + (size_t)(t * KBh + kb) * 2 * R * BK, (uint32_t)(2 * R * kTileBytes),
+                                 &full[s]);
+                if (++s == S) { s = 0; ph ^= 1; }
+            }
         }
-        issued_s = kb;
+        issued_s = i;
     } else if (warp == 1 && lane == 0) {
         const uint32_t idesc = instr_desc(BM, R);
-        int kb = 0;
-        for (int s = 0, ph = 0; kb < p.KBh; ++kb) {
-            if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
+        int i = 0, s = 0, ph = 0, it = 0;
+        bool stop = false;
+        for (int q = blockIdx.x; q < p.tiles && !stop; q += gridDim.x, ++it) {
+            const int buf = it & 1;
+            if (!mbar_wait(&acc_empty[buf], (uint32_t)((it >> 1) & 1) ^ 1u, &abort_flag)) {
+                set_timeout(p.ctl, &abort_flag);
+                break;
+            }
             tc_fence_after();
-            const uint32_t st = smem_addr(ring + (size_t)s * p.stage_bytes);
-            const uint32_t wa = st + wofs;
-#pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk) {
-                const uint32_t acc = (kb | kk) ? 1u : 0u;
-                const uint64_t a = smem_desc(st + kk * 32);
-                const uint64_t g = smem_desc(wa + kk * 32);
-                const uint64_t u = smem_desc(wa + R * kTileBytes + kk * 32);
-                mma_bf16(tmem, a, g, idesc, acc);
-                mma_bf16(tmem + R, a, u, idesc, acc);
-                if (p.split) {
-                    const uint64_t a2 = smem_desc(st + kA + kk * 32);
-                    mma_bf16(tmem, a2, g, idesc, 1u);
-                    mma_bf16(tmem + R, a2, u, idesc, 1u);
+            const uint32_t dg = tmem + (uint32_t)(buf * 2 * R), du = dg + (uint32_t)R;
+            for (int kb = 0; kb < KBh; ++kb, ++i) {
+                if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) {
+                    set_timeout(p.ctl, &abort_flag);
+                    stop = true;
+                    break;
                 }
-            }
-            mma_commit(&empty[s]);
-            if (++s == S) { s = 0; ph ^= 1; }
-        }
-        consumed_s = kb;
-        mma_commit(acc_full);
-    } else if (warp >= 2) {
-        // epilogue: thread = token row of the tile, 16 neurons at a time
-        const bool ok = mbar_wait(acc_full, 0u, &abort_flag);
-        tc_fence_after();
-        const int lb = 32 * (warp & 3);
-        const int m = m0 + lb + lane;
-        const bool row_ok = ok && m < p.M;
-        float thr = INFINITY;
-        if (row_ok) thr = (p.dense_flags && p.dense_flags[m]) ? 0.f : p.t_l;
-        for (int c0 = 0; c0 < R; c0 += 16) {
-            float g[16], u[16];
-            tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)c0, g);
-            tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(R + c0), u);
-            tmem_ld_wait();
-            const int n = t * R + c0;
-            if (!row_ok || n >= p.N) continue;
-            uint32_t hw[8], kw[4] = {0u, 0u, 0u, 0u};
+                tc_fence_after();
+                const uint32_t st = smem_addr(ring + (size_t)s * p.stage_bytes);
+                const uint32_t wa = st + wofs;
 #pragma unroll
-            for (int e = 0; e < 16; e += 2) {
-                const float a0 = g[e] / (1.0f + expf(-g[e]));             // SiLU, Eq. 2
-                const float a1 = g[e + 1] / (1.0f + expf(-g[e + 1]));
-                const bool k0 = fabsf(a0) >= thr, k1 = fabsf(a1) >= thr;   // Eqs. 4-5
-                hw[e / 2] = (uint32_t)bf16_bits(k0 ? a0 * u[e] : 0.f) |
-                            ((uint32_t)bf16_bits(k1 ? a1 * u[e + 1] : 0.f) << 16);
-                kw[e / 4] |= ((k0 ? 1u : 0u) << (8 * (e % 4))) | ((k1 ? 1u : 0u) << (8 * (e % 4) + 8));
-            }
-            uint16_t *hrow = p.hact + (size_t)m * p.ldh + n;
-            uint8_t *krow = p.keep ? p.keep + (size_t)m * p.keep_stride + n : nullptr;
-            if (n + 16 <= p.N) {   // n is a multiple of 16: 32-byte aligned h, 16-byte aligned keep
-                reinterpret_cast<uint4 *>(hrow)[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-                reinterpret_cast<uint4 *>(hrow)[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
-                if (krow) *reinterpret_cast<uint4 *>(krow) = make_uint4(kw[0], kw[1], kw[2], kw[3]);
-            } else {
-#pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    if (n + e < p.N) {
-                        hrow[e] = (uint16_t)(hw[e / 2] >> (16 * (e & 1)));
-                        if (krow) krow[e] = (uint8_t)(kw[e / 4] >> (8 * (e & 3)));
+                for (int kk = 0; kk < BK / 16; ++kk) {
+                    const uint32_t acc = (kb | kk) ? 1u : 0u;
+                    const uint64_t a = smem_desc(st + kk * 32);
+                    const uint64_t g = smem_desc(wa + kk * 32);
+                    const uint64_t u = smem_desc(wa + R * kTileBytes + kk * 32);
+                    mma_bf16(dg, a, g, idesc, acc);
+                    mma_bf16(du, a, u, idesc, acc);
+                    if (p.split) {
+                        const uint64_t a2 = smem_desc(st + kA + kk * 32);
+                        mma_bf16(dg, a2, g, idesc, 1u);
+                        mma_bf16(du, a2, u, idesc, 1u);
                     }
                 }
+                mma_commit(&empty[s]);
+                if (++s == S) { s = 0; ph ^= 1; }
             }
-            if (p.keep_trace) {
-                uint8_t *trow = p.keep_trace + (size_t)m * p.N + n;
-#pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    if (n + e < p.N) trow[e] = (uint8_t)(kw[e / 4] >> (8 * (e & 3)));
-            }
+            mma_commit(&acc_full[buf]);
         }
-        tc_fence_before();
+        consumed_s = i;
+        mma_commit(mma_done);
+    } else if (warp >= 2) {
+        // epilogue: thread = token row of the tile, 16 neurons at a time
+        const int lb = 32 * (warp & 3);
+        int it = 0;
+        for (int q = blockIdx.x; q < p.tiles; q += gridDim.x, ++it) {
+            const int buf = it & 1;
+            const int m = (q % p.mtiles) * BM + lb + lane, t = q / p.mtiles;
+            const bool ok = mbar_wait(&acc_full[buf], (uint32_t)((it >> 1) & 1), &abort_flag);
+            tc_fence_after();
+            const bool row_ok = ok && m < p.M;
+            float thr = INFINITY;
+            if (row_ok) thr = (p.dense_flags && p.dense_flags[m]) ? 0.f : p.t_l;
+            const uint32_t dg = tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * 2 * R);
+            for (int c0 = 0; c0 < R; c0 += 16) {
+                float g[16], u[16];
+                tmem_ld16(dg + (uint32_t)c0, g);
+                tmem_ld16(dg + (uint32_t)(R + c0), u);
+                tmem_ld_wait();
+                const int n = t * R + c0;
+                if (!row_ok || n >= p.N) continue;
+                uint32_t hw[8], kw[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+                for (int e = 0; e < 16; e += 2) {
+                    const float a0 = g[e] / (1.0f + expf(-g[e]));             // SiLU, Eq. 2
+                    const float a1 = g[e + 1] / (1.0f + expf(-g[e + 1]));
+                    const bool k0 = fabsf(a0) >= thr, k1 = fabsf(a1) >= thr;   // Eqs. 4-5
+                    hw[e / 2] = (uint32_t)bf16_bits(k0 ? a0 * u[e] : 0.f) |
+                                ((uint32_t)bf16_bits(k1 ? a1 * u[e + 1] : 0.f) << 16);
+                    kw[e / 4] |= ((k0 ? 1u : 0u) << (8 * (e % 4))) | ((k1 ? 1u : 0u) << (8 * (e % 4) + 8));
+                }
+                uint16_t *hrow = p.hact + (size_t)m * p.ldh + n;
+                uint8_t *krow = p.keep ? p.keep + (size_t)m * p.keep_stride + n : nullptr;
+                if (n + 16 <= p.N) {   // n is a multiple of 16: 32-byte aligned h, 16-byte aligned keep
+                    reinterpret_cast<uint4 *>(hrow)[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+                    reinterpret_cast<uint4 *>(hrow)[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+                    if (krow) *reinterpret_cast<uint4 *>(krow) = make_uint4(kw[0], kw[1], kw[2], kw[3]);
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        if (n + e < p.N) {
+                            hrow[e] = (uint16_t)(hw[e / 2] >> (16 * (e & 1)));
+                            if (krow) krow[e] = (uint8_t)(kw[e / 4] >> (8 * (e & 3)));
+                        }
+                    }
+                }
+                if (p.keep_trace) {
+                    uint8_t *trow = p.keep_trace + (size_t)m * p.N + n;
+#pragma unroll
+                    for (int e = 0; e < 16; ++e)
+                        if (n + e < p.N) trow[e] = (uint8_t)(kw[e / 4] >> (8 * (e & 3)));
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(&acc_empty[buf]);
+            if (!ok) break;
+        }
     }
     __syncthreads();
-    if (abort_flag && threadIdx.x == 0) drain_after_abort(full, S, issued_s, consumed_s, acc_full);
+    if (threadIdx.x == 0) {
+        // the arrival on mma_done must land before this CTA's shared memory is released
+        int never = 0;
+        if (abort_flag)
+            for (int k = consumed_s; k < issued_s; ++k) mbar_wait(&full[k % S], (uint32_t)((k / S) & 1), &never);
+        mbar_wait(mma_done, 0u, &never);
+    }
     __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem, 256);
+        tmem_dealloc(tmem, p.tmem_cols);
     }
 }
 
@@ -890,18 +938,28 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols, 
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Raises the kernel's dynamic shared-memory limit once per device; `configured`
-// is the caller's flag word, one per kernel.
+// The device's opt-in limit of shared memory per CTA.
+int smem_optin()
+{
+    static int by_dev[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    int &n = by_dev[dev & 63];
+    if (n == 0) cudaDeviceGetAttribute(&n, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    return n;
+}
+
+// Raises the kernel's dynamic shared-memory limit on the current device to at
+// least `bytes`; `configured` is the caller's per-device record for this kernel.
 template <typename K>
-cudaError_t set_smem(K kernel, std::atomic<unsigned long long> &configured)
+cudaError_t set_smem(K kernel, size_t bytes, std::atomic<int> (&configured)[64])
 {
     int dev = 0;
     cudaGetDevice(&dev);
-    const unsigned long long bit = 1ull << (dev & 63);
-    if (configured.load() & bit) return cudaSuccess;
-    const int bytes = kSmemBudget + 2048;
-    const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e == cudaSuccess) configured.fetch_or(bit);
+    std::atomic<int> &have = configured[dev & 63];
+    if ((int)bytes <= have.load()) return cudaSuccess;
+    const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess) have.store((int)bytes);
     return e;
 }
 
@@ -943,6 +1001,14 @@ cudaError_t launch_pdl_threads(void (*kernel)(KArgs...), dim3 grid, int threads,
 
 // Dynamic shared memory of a launch: the stage ring, 1 KB of alignment slack and the barriers.
 size_t smem_for(int stages, int stage_bytes) { return (size_t)stages * stage_bytes + 1024 + 256; }
+
+// Ring budget of the prefill kernels: kSmemWide, or less if the device allows
+// less (the opt-in limit covers the kernel's static shared memory as well).
+int wide_budget()
+{
+    const int lim = smem_optin() - 1024 - 256 - 64;
+    return lim < kSmemWide ? lim : kSmemWide;
+}
 
 int stages_for(int stage_bytes, int budget = kSmemBudget)
 {
@@ -1055,6 +1121,10 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
                          int32_t *active_cnt, uint8_t *keep_trace, void *tc_ws, int *ctl, cudaStream_t stream)
 {
     using namespace tc;
+    auto fail = [](cudaError_t err, const char *where) {
+        cuda_fail(err, where);
+        return err;
+    };
     const int H = layer->H, N = layer->N, ldn = layer->ldn, R = layer->tc_R;
     const TcLayout W = tc_layout(H, N, B);
     uint8_t *base = static_cast<uint8_t *>(tc_ws);
@@ -1071,7 +1141,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
     if (split) {
         e = launch_pdl_threads(split_kernel, dim3(B), 256, stream, static_cast<const float *>(x), H,
                                x_mode == kXResidNorm ? norm_w : nullptr, eps, xhi, xlo);
-        if (e != cudaSuccess) return e;
+        if (e != cudaSuccess) return fail(e, "split kernel launch");
     }
 
     if (B <= kMaxSkinny) {
@@ -1079,7 +1149,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         CUtensorMap mX, mX2, mH;
         if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, NT) || !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, NT) ||
             !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, NT))
-            return cudaErrorInvalidValue;
+            return fail(cudaErrorInvalidValue, "tensor map encoding");
         SkinnyGuParams gp{};
         gp.w = layer->gu_blk;
         gp.M = B;
@@ -1109,10 +1179,11 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.stages = stages_for(gp.stage_bytes, kSmemBudget - slack);
         gp.ring_bytes = gp.stages * gp.stage_bytes + slack;
         gp.tmem_cols = tmem_cols_for(2 * NT);
-        static std::atomic<unsigned long long> cfg_gu{0};
-        if ((e = set_smem(gu_skinny_kernel, cfg_gu)) != cudaSuccess) return e;
+        static std::atomic<int> cfg_gu[64];
+        if ((e = set_smem(gu_skinny_kernel, smem_for(1, gp.ring_bytes), cfg_gu)) != cudaSuccess)
+            return fail(e, "shared-memory attribute");
         e = launch_pdl(gu_skinny_kernel, dim3(layer->tc_T), smem_for(1, gp.ring_bytes), stream, mX, mX2, gp);
-        if (e != cudaSuccess) return e;
+        if (e != cudaSuccess) return fail(e, "gate/up kernel launch");
 
         SkinnyDownParams dp{};
         dp.w = layer->wd_blk;
@@ -1127,17 +1198,18 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         dp.stage_bytes = dp.a_bytes + NT * kTileBytes;
         dp.stages = stages_for(dp.stage_bytes);
         dp.tmem_cols = tmem_cols_for(2 * NT);
-        static std::atomic<unsigned long long> cfg_dn{0};
-        if ((e = set_smem(down_skinny_kernel, cfg_dn)) != cudaSuccess) return e;
+        static std::atomic<int> cfg_dn[64];
+        if ((e = set_smem(down_skinny_kernel, smem_for(dp.stages, dp.stage_bytes), cfg_dn)) != cudaSuccess)
+            return fail(e, "shared-memory attribute");
         e = launch_pdl(down_skinny_kernel, dim3(dp.units < sms ? dp.units : sms), smem_for(dp.stages, dp.stage_bytes),
                        stream, mH, dp);
-        if (e != cudaSuccess) return e;
+        if (e != cudaSuccess) return fail(e, "down kernel launch");
     } else {
         CUtensorMap mX, mX2, mH;
         if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, BM) ||
             !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, BM) ||
             !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, BM))
-            return cudaErrorInvalidValue;
+            return fail(cudaErrorInvalidValue, "tensor map encoding");
         const int mtiles = (B + BM - 1) / BM;
 
         WideGuParams gp{};
@@ -1146,6 +1218,9 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.N = N;
         gp.R = R;
         gp.KBh = layer->tc_kbh;
+        gp.mtiles = mtiles;
+        gp.tiles = mtiles * layer->tc_T;
+        gp.tmem_cols = tmem_cols_for(4 * R);
         gp.split = split ? 1 : 0;
         gp.t_l = t_l;
         gp.dense_flags = dense_flags;
@@ -1156,12 +1231,13 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.keep_trace = keep_trace;
         gp.ctl = ctl;
         gp.stage_bytes = BM * kTileBytes * (split ? 2 : 1) + 2 * R * kTileBytes;
-        gp.stages = stages_for(gp.stage_bytes);
-        static std::atomic<unsigned long long> cfg_gu{0};
-        if ((e = set_smem(gu_wide_kernel, cfg_gu)) != cudaSuccess) return e;
-        gu_wide_kernel<<<dim3(mtiles, layer->tc_T), kThreads, smem_for(gp.stages, gp.stage_bytes), stream>>>(
-            mX, mX2, gp);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        gp.stages = stages_for(gp.stage_bytes, wide_budget());
+        static std::atomic<int> cfg_gu[64];
+        if ((e = set_smem(gu_wide_kernel, smem_for(gp.stages, gp.stage_bytes), cfg_gu)) != cudaSuccess)
+            return fail(e, "shared-memory attribute");
+        gu_wide_kernel<<<dim3(gp.tiles < sms ? gp.tiles : sms), kThreads, smem_for(gp.stages, gp.stage_bytes),
+                         stream>>>(mX, mX2, gp);
+        if ((e = cudaGetLastError()) != cudaSuccess) return fail(e, "gate/up kernel launch");
 
         // down projection: 256 output columns per tile when the hidden tiles pair up;
         // split K (neurons) when the tile grid alone leaves SMs idle
@@ -1184,17 +1260,18 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         dp.stages = stages_for(dp.stage_bytes);
         if (splits > 1 && out_mode == kOutY &&
             (e = cudaMemsetAsync(out, 0, (size_t)B * H * sizeof(float), stream)) != cudaSuccess)
-            return e;
-        static std::atomic<unsigned long long> cfg_dn{0};
-        if ((e = set_smem(down_wide_kernel, cfg_dn)) != cudaSuccess) return e;
+            return fail(e, "y clear");
+        static std::atomic<int> cfg_dn[64];
+        if ((e = set_smem(down_wide_kernel, smem_for(dp.stages, dp.stage_bytes), cfg_dn)) != cudaSuccess)
+            return fail(e, "shared-memory attribute");
         down_wide_kernel<<<dim3(mtiles, layer->tc_dt / dp.dtiles, splits), kThreads,
                            smem_for(dp.stages, dp.stage_bytes), stream>>>(mH, dp);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if ((e = cudaGetLastError()) != cudaSuccess) return fail(e, "down kernel launch");
     }
     if (active_idx) {
         e = launch_pdl_threads(keep_list_kernel, dim3(B), 512, stream, static_cast<const uint8_t *>(keep), kstride, N,
                                active_idx, active_cnt);
-        if (e != cudaSuccess) return e;
+        if (e != cudaSuccess) return fail(e, "kept-list kernel launch");
     }
     return cudaSuccess;
 }

@@ -75,6 +75,10 @@ struct FusedParams {
     uint8_t *keep_trace;          // [nb][N] or nullptr
 };
 
+// Records the CUDA error behind a SATS_ECUDA result (per host thread), with a
+// static description of the step that failed; returns SATS_ECUDA.
+sats_status cuda_fail(cudaError_t e, const char *where);
+
 // Number of CTAs the fused kernel runs with on `device` (all co-resident).
 int fused_grid(int nchunks);
 int fused_tokens_per_pass(int H);

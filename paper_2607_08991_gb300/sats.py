@@ -25,7 +25,10 @@ _lib = None
 class SatsError(RuntimeError):
     def __init__(self, status: int, where: str):
         self.status = status
-        super().__init__("%s: %s (status %d)" % (where, status_string(status), status))
+        msg = "%s: %s (status %d)" % (where, status_string(status), status)
+        if status == ECUDA:
+            msg += ": " + lib().sats_last_cuda_error().decode()
+        super().__init__(msg)
 
 
 def lib() -> ctypes.CDLL:
@@ -50,6 +53,7 @@ def lib() -> ctypes.CDLL:
             "sats_sparse_mlp_f32": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_sparse_mlp_fixed_scratch": (I, [P, P, I, F, P, P, P, P]),
             "sats_uses_tensor_cores": (I, [I, I]),
+            "sats_last_cuda_error": (ctypes.c_char_p, []),
             "sats_dense_mlp": (I, [P, P, I, P, P, Z, P]),
             "sats_route": (I, [P, I, P, I, P, P, P, P]),
             "sats_mlp_stack": (I, [P, P, P, I, F, P, P, I, P, I, P, P, Z, P]),
@@ -71,7 +75,7 @@ def exported_symbols() -> Sequence[str]:
     """Every C entry point this binding forwards to."""
     return ("sats_version", "sats_status_string", "sats_layer_create", "sats_layer_destroy", "sats_layer_shape",
             "sats_workspace_bytes", "sats_workspace_init", "sats_sparse_mlp", "sats_sparse_mlp_f32",
-            "sats_sparse_mlp_fixed_scratch", "sats_uses_tensor_cores", "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
+            "sats_sparse_mlp_fixed_scratch", "sats_uses_tensor_cores", "sats_last_cuda_error", "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
             "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_get_error", "sats_get_status_word")
 
 
