@@ -628,7 +628,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         issued_s = i;
     } else if (warp == 1 && lane == 0) {
-        const uint32_t idesc = instr_desc(BM, R);
+        // gate rows and up rows are adjacent in the stage: one MMA with N = 2R writes the gate
+        // accumulator to columns [0, R) and the up accumulator to [R, 2R)
+        const uint32_t idesc = instr_desc(BM, 2 * R);
         int i = 0, s = 0, ph = 0, it = 0;
         bool stop = false;
         for (int q = blockIdx.x; q < p.tiles && !stop; q += gridDim.x, ++it) {
@@ -638,7 +640,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             tc_fence_after();
-            const uint32_t dg = tmem + (uint32_t)(buf * 2 * R), du = dg + (uint32_t)R;
+            const uint32_t d = tmem + (uint32_t)(buf * 2 * R);
             for (int kb = 0; kb < KBh; ++kb, ++i) {
                 if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) {
                     set_timeout(p.ctl, &abort_flag);
@@ -650,17 +652,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t wa = st + wofs;
 #pragma unroll
                 for (int kk = 0; kk < BK / 16; ++kk) {
-                    const uint32_t acc = (kb | kk) ? 1u : 0u;
-                    const uint64_t a = smem_desc(st + kk * 32);
-                    const uint64_t g = smem_desc(wa + kk * 32);
-                    const uint64_t u = smem_desc(wa + R * kTileBytes + kk * 32);
-                    mma_bf16(dg, a, g, idesc, acc);
-                    mma_bf16(du, a, u, idesc, acc);
-                    if (p.split) {
-                        const uint64_t a2 = smem_desc(st + kA + kk * 32);
-                        mma_bf16(dg, a2, g, idesc, 1u);
-                        mma_bf16(du, a2, u, idesc, 1u);
-                    }
+                    const uint64_t w = smem_desc(wa + kk * 32);
+                    mma_bf16(d, smem_desc(st + kk * 32), w, idesc, (kb | kk) ? 1u : 0u);
+                    if (p.split) mma_bf16(d, smem_desc(st + kA + kk * 32), w, idesc, 1u);
                 }
                 mma_commit(&empty[s]);
                 if (++s == S) { s = 0; ph ^= 1; }
