@@ -9,8 +9,9 @@
 //   Y = h W_down                        (second kernel)
 // X is bf16: the caller's bf16 activations, or fp32 activations (optionally
 // RMS-normalised) split into a bf16 high part and a bf16 low part, both fed to
-// the same accumulator, so that the gate values keep ~fp32 accuracy.  h is
-// kept in bf16 between the two GEMMs.
+// the same accumulator, so that the gate values keep ~fp32 accuracy.  h goes
+// to the second GEMM the same way, as a bf16 high part and a bf16 low part
+// (about 16 significant bits), so that errors do not build up along a stack.
 //
 // Two orientations:
 //  - skinny (M <= 256 tokens, bandwidth-bound): the weights are the MMA's A
@@ -250,7 +251,8 @@ struct SkinnyGuParams {
     int split;                    // 1: two B operands (bf16 hi and lo parts of fp32 x)
     float t_l;                    // threshold of sparse-path tokens
     const uint8_t *dense_flags;   // [M] (1 = base path, threshold 0) or nullptr
-    uint16_t *hact;               // [M][ldh] bf16
+    uint16_t *hact;               // [M][ldh] bf16: h rounded to bf16
+    uint16_t *hact_lo;            // [M][ldh] bf16: h minus that rounding
     int ldh;
     uint8_t *keep;                // [M][keep_stride] or nullptr
     int keep_stride;
@@ -377,7 +379,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const float thr = (p.dense_flags && p.dense_flags[j]) ? 0.f : p.t_l;
                     const float a = g[e] / (1.0f + expf(-g[e]));   // SiLU, Eq. 2
                     const bool keep = fabsf(a) >= thr;             // Eqs. 4-5
-                    p.hact[(size_t)j * p.ldh + n] = bf16_bits(keep ? a * u[e] : 0.f);
+                    const float h = keep ? a * u[e] : 0.f;
+                    const uint16_t hb = bf16_bits(h);
+                    p.hact[(size_t)j * p.ldh + n] = hb;
+                    p.hact_lo[(size_t)j * p.ldh + n] = bf16_bits(h - __uint_as_float((uint32_t)hb << 16));
                     if (p.keep) p.keep[(size_t)j * p.keep_stride + n] = keep ? 1 : 0;
                     if (p.keep_trace) p.keep_trace[(size_t)j * p.N + n] = keep ? 1 : 0;
                 }
@@ -407,9 +412,11 @@ struct SkinnyDownParams {
 // CTA c handles units [c U / G, (c+1) U / G) in order; consecutive units of one
 // hidden tile form a segment accumulated in TMEM (two buffers, so that the
 // epilogue of one segment overlaps the MMAs of the next) and added into y.
-// Unit u's weight tile is tile u of wd_blk.
+// Unit u's weight tile is tile u of wd_blk; h arrives as its high and low bf16
+// parts, two MMAs into the same accumulator.
 __global__ void __launch_bounds__(kThreads, 1)
-    down_skinny_kernel(const __grid_constant__ CUtensorMap tmH, const SkinnyDownParams p)
+    down_skinny_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmH2,
+                       const SkinnyDownParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *ring = align1024(smem_raw);
@@ -450,7 +457,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp == 0 && lane == 0) {
         const uint32_t w_bytes = (uint32_t)(BM * kTileBytes);
-        const uint32_t load_bytes = w_bytes + (uint32_t)(NT * kTileBytes);
+        const uint32_t load_bytes = w_bytes + (uint32_t)(2 * NT * kTileBytes);
         const uint64_t policy = l2_policy_evict_first();
         // the weight tiles do not depend on the preceding kernel: start them first
         const int npre = nu < S ? nu : S;
@@ -469,6 +476,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 bulk_load(st, p.w + (size_t)u * BM * BK, w_bytes, &full[s], policy);
             }
             tma_load(st + p.a_bytes, &tmH, (u % KBn) * BK, 0, &full[s]);
+            tma_load(st + p.a_bytes + NT * kTileBytes, &tmH2, (u % KBn) * BK, 0, &full[s]);
             if (++s == S) { s = 0; ph ^= 1; }
         }
         issued_s = i;   // a break happens only before stage i's loads are issued (i >= npre)
@@ -490,9 +498,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 const uint32_t st = smem_addr(ring + (size_t)s * p.stage_bytes);
 #pragma unroll
-                for (int kk = 0; kk < BK / 16; ++kk)
-                    mma_bf16(tmem + (uint32_t)(buf * NT), smem_desc(st + kk * 32), smem_desc(st + p.a_bytes + kk * 32),
-                             idesc, (first && kk == 0) ? 0u : 1u);
+                for (int kk = 0; kk < BK / 16; ++kk) {
+                    const uint64_t w = smem_desc(st + kk * 32);
+                    mma_bf16(tmem + (uint32_t)(buf * NT), w, smem_desc(st + p.a_bytes + kk * 32), idesc,
+                             (first && kk == 0) ? 0u : 1u);
+                    mma_bf16(tmem + (uint32_t)(buf * NT), w, smem_desc(st + p.a_bytes + NT * kTileBytes + kk * 32),
+                             idesc, 1u);
+                }
                 first = false;
                 mma_commit(&empty[s]);
                 if (++s == S) { s = 0; ph ^= 1; }
@@ -550,7 +562,7 @@ struct WideGuParams {
     int split;
     float t_l;
     const uint8_t *dense_flags;
-    uint16_t *hact;
+    uint16_t *hact, *hact_lo;     // h as bf16 high and low parts
     int ldh;
     uint8_t *keep;
     int keep_stride;              // a multiple of 16
@@ -683,27 +695,34 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tmem_ld_wait();
                 const int n = t * R + c0;
                 if (!row_ok || n >= p.N) continue;
-                uint32_t hw[8], kw[4] = {0u, 0u, 0u, 0u};
+                uint32_t hw[8], lw[8], kw[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
                 for (int e = 0; e < 16; e += 2) {
                     const float a0 = g[e] / (1.0f + expf(-g[e]));             // SiLU, Eq. 2
                     const float a1 = g[e + 1] / (1.0f + expf(-g[e + 1]));
                     const bool k0 = fabsf(a0) >= thr, k1 = fabsf(a1) >= thr;   // Eqs. 4-5
-                    hw[e / 2] = (uint32_t)bf16_bits(k0 ? a0 * u[e] : 0.f) |
-                                ((uint32_t)bf16_bits(k1 ? a1 * u[e + 1] : 0.f) << 16);
+                    const float h0 = k0 ? a0 * u[e] : 0.f, h1 = k1 ? a1 * u[e + 1] : 0.f;
+                    const uint16_t b0 = bf16_bits(h0), b1 = bf16_bits(h1);
+                    hw[e / 2] = (uint32_t)b0 | ((uint32_t)b1 << 16);
+                    lw[e / 2] = (uint32_t)bf16_bits(h0 - __uint_as_float((uint32_t)b0 << 16)) |
+                                ((uint32_t)bf16_bits(h1 - __uint_as_float((uint32_t)b1 << 16)) << 16);
                     kw[e / 4] |= ((k0 ? 1u : 0u) << (8 * (e % 4))) | ((k1 ? 1u : 0u) << (8 * (e % 4) + 8));
                 }
                 uint16_t *hrow = p.hact + (size_t)m * p.ldh + n;
+                uint16_t *lrow = p.hact_lo + (size_t)m * p.ldh + n;
                 uint8_t *krow = p.keep ? p.keep + (size_t)m * p.keep_stride + n : nullptr;
                 if (n + 16 <= p.N) {   // n is a multiple of 16: 32-byte aligned h, 16-byte aligned keep
                     reinterpret_cast<uint4 *>(hrow)[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
                     reinterpret_cast<uint4 *>(hrow)[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+                    reinterpret_cast<uint4 *>(lrow)[0] = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+                    reinterpret_cast<uint4 *>(lrow)[1] = make_uint4(lw[4], lw[5], lw[6], lw[7]);
                     if (krow) *reinterpret_cast<uint4 *>(krow) = make_uint4(kw[0], kw[1], kw[2], kw[3]);
                 } else {
 #pragma unroll
                     for (int e = 0; e < 16; ++e) {
                         if (n + e < p.N) {
                             hrow[e] = (uint16_t)(hw[e / 2] >> (16 * (e & 1)));
+                            lrow[e] = (uint16_t)(lw[e / 2] >> (16 * (e & 1)));
                             if (krow) krow[e] = (uint8_t)(kw[e / 4] >> (8 * (e & 3)));
                         }
                     }
@@ -749,9 +768,11 @@ struct WideDownParams {
 };
 
 // One 128-token x (128 dtiles)-column tile of Y = h W_down over one split of
-// the neuron range.  Grid: (ceil(M / 128), tc_dt / dtiles, splits).
+// the neuron range; h arrives as its high and low bf16 parts (two A tiles).
+// Grid: (ceil(M / 128), tc_dt / dtiles, splits).
 __global__ void __launch_bounds__(kThreads, 1)
-    down_wide_kernel(const __grid_constant__ CUtensorMap tmH, const WideDownParams p)
+    down_wide_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmH2,
+                     const WideDownParams p)
 {
     constexpr int kA = BM * kTileBytes;
     extern __shared__ uint8_t smem_raw[];
@@ -785,7 +806,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = *tmem_slot;
 
     if (warp == 0 && lane == 0) {
-        const uint32_t load_bytes = (uint32_t)(kA + BN * kTileBytes);
+        const uint32_t load_bytes = (uint32_t)(2 * kA + BN * kTileBytes);
         int i = 0;
         for (int s = 0, ph = 0; kb0 + i < kb1; ++i) {
             if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
@@ -793,9 +814,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint8_t *st = ring + (size_t)s * p.stage_bytes;
             mbar_arrive_expect_tx(&full[s], load_bytes);
             tma_load(st, &tmH, kb * BK, m0, &full[s]);
+            tma_load(st + kA, &tmH2, kb * BK, m0, &full[s]);
             for (int q = 0; q < p.dtiles; ++q)
-                bulk_load_shared(st + kA + q * kA, p.w + ((size_t)(d0 + q) * p.KBn + kb) * BM * BK, (uint32_t)kA,
-                                 &full[s]);
+                bulk_load_shared(st + 2 * kA + q * kA, p.w + ((size_t)(d0 + q) * p.KBn + kb) * BM * BK,
+                                 (uint32_t)kA, &full[s]);
             if (++s == S) { s = 0; ph ^= 1; }
         }
         issued_s = i;
@@ -807,8 +829,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const uint32_t st = smem_addr(ring + (size_t)s * p.stage_bytes);
 #pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk)
-                mma_bf16(tmem, smem_desc(st + kk * 32), smem_desc(st + kA + kk * 32), idesc, (i | kk) ? 1u : 0u);
+            for (int kk = 0; kk < BK / 16; ++kk) {
+                const uint64_t w = smem_desc(st + 2 * kA + kk * 32);
+                mma_bf16(tmem, smem_desc(st + kk * 32), w, idesc, (i | kk) ? 1u : 0u);
+                mma_bf16(tmem, smem_desc(st + kA + kk * 32), w, idesc, 1u);
+            }
             mma_commit(&empty[s]);
             if (++s == S) { s = 0; ph ^= 1; }
         }
@@ -1080,7 +1105,7 @@ cudaError_t tc_free_layer(sats_layer *l)
 
 namespace {
 struct TcLayout {
-    size_t xhi, xlo, hact, keep, total;
+    size_t xhi, xlo, hact, hact_lo, keep, total;
 };
 
 TcLayout tc_layout(int H, int N, int B)
@@ -1094,6 +1119,8 @@ TcLayout tc_layout(int H, int N, int B)
     L.xlo = off;
     off += al((size_t)B * H * 2);
     L.hact = off;
+    off += al((size_t)B * ldn * 2);
+    L.hact_lo = off;
     off += al((size_t)B * ldn * 2);
     L.keep = off;
     off += al((size_t)B * (((size_t)N + 15) & ~(size_t)15));
@@ -1125,6 +1152,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
     uint16_t *xhi = reinterpret_cast<uint16_t *>(base + W.xhi);
     uint16_t *xlo = reinterpret_cast<uint16_t *>(base + W.xlo);
     uint16_t *hact = reinterpret_cast<uint16_t *>(base + W.hact);
+    uint16_t *hact_lo = reinterpret_cast<uint16_t *>(base + W.hact_lo);
     uint8_t *keep = base + W.keep;
     const int kstride = (N + 15) & ~15;
     const int sms = sm_count();
@@ -1140,9 +1168,9 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
 
     if (B <= kMaxSkinny) {
         const int NT = (B + 15) & ~15;
-        CUtensorMap mX, mX2, mH;
+        CUtensorMap mX, mX2, mH, mH2;
         if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, NT) || !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, NT) ||
-            !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, NT))
+            !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, NT) || !make_map(&mH2, hact_lo, B, N, (uint64_t)ldn * 2, NT))
             return fail(cudaErrorInvalidValue, "tensor map encoding");
         SkinnyGuParams gp{};
         gp.w = layer->gu_blk;
@@ -1155,6 +1183,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.t_l = t_l;
         gp.dense_flags = dense_flags;
         gp.hact = hact;
+        gp.hact_lo = hact_lo;
         gp.ldh = ldn;
         gp.keep = active_idx ? keep : nullptr;
         gp.keep_stride = kstride;
@@ -1189,20 +1218,20 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         dp.out = out;
         dp.ctl = ctl;
         dp.a_bytes = BM * kTileBytes;
-        dp.stage_bytes = dp.a_bytes + NT * kTileBytes;
+        dp.stage_bytes = dp.a_bytes + 2 * NT * kTileBytes;
         dp.stages = stages_for(dp.stage_bytes);
         dp.tmem_cols = tmem_cols_for(2 * NT);
         static std::atomic<int> cfg_dn[64];
         if ((e = set_smem(down_skinny_kernel, smem_for(dp.stages, dp.stage_bytes), cfg_dn)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
         e = launch_pdl(down_skinny_kernel, dim3(dp.units < sms ? dp.units : sms), smem_for(dp.stages, dp.stage_bytes),
-                       stream, mH, dp);
+                       stream, mH, mH2, dp);
         if (e != cudaSuccess) return fail(e, "down kernel launch");
     } else {
-        CUtensorMap mX, mX2, mH;
+        CUtensorMap mX, mX2, mH, mH2;
         if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, BM) ||
             !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, BM) ||
-            !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, BM))
+            !make_map(&mH, hact, B, N, (uint64_t)ldn * 2, BM) || !make_map(&mH2, hact_lo, B, N, (uint64_t)ldn * 2, BM))
             return fail(cudaErrorInvalidValue, "tensor map encoding");
         const int mtiles = (B + BM - 1) / BM;
 
@@ -1219,6 +1248,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.t_l = t_l;
         gp.dense_flags = dense_flags;
         gp.hact = hact;
+        gp.hact_lo = hact_lo;
         gp.ldh = ldn;
         gp.keep = active_idx ? keep : nullptr;
         gp.keep_stride = kstride;
@@ -1250,8 +1280,8 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         dp.add_residual = out_mode == kOutResid ? 1 : 0;
         dp.out = out;
         dp.ctl = ctl;
-        dp.stage_bytes = BM * kTileBytes * (1 + dp.dtiles);
-        dp.stages = stages_for(dp.stage_bytes);
+        dp.stage_bytes = BM * kTileBytes * (2 + dp.dtiles);
+        dp.stages = stages_for(dp.stage_bytes, wide_budget());
         if (splits > 1 && out_mode == kOutY &&
             (e = cudaMemsetAsync(out, 0, (size_t)B * H * sizeof(float), stream)) != cudaSuccess)
             return fail(e, "y clear");
@@ -1259,7 +1289,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         if ((e = set_smem(down_wide_kernel, smem_for(dp.stages, dp.stage_bytes), cfg_dn)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
         down_wide_kernel<<<dim3(mtiles, layer->tc_dt / dp.dtiles, splits), kThreads,
-                           smem_for(dp.stages, dp.stage_bytes), stream>>>(mH, dp);
+                           smem_for(dp.stages, dp.stage_bytes), stream>>>(mH, mH2, dp);
         if ((e = cudaGetLastError()) != cudaSuccess) return fail(e, "down kernel launch");
     }
     if (active_idx) {

@@ -81,6 +81,37 @@ def mlp_weights(H: int, N: int, layer: int = 0, std: float = 0.02, seed: int = S
     )
 
 
+def _seed63(*seed: int) -> int:
+    return int(np.random.SeedSequence(list(seed)).generate_state(1, np.uint64)[0] & np.uint64((1 << 63) - 1))
+
+
+def device_normal_bf16(shape, std: float, *seed: int, device="cuda"):
+    """N(0, std) rounded to bf16 (nearest even), drawn on a CUDA device by torch's
+    seeded Philox generator: a device int16 tensor of bf16 bit patterns.  For
+    the model-sized weights of the full-size workloads, which the host would
+    take minutes to draw; the oracle gets the same values by copying them to
+    the host (`host_bits`)."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(_seed63(*seed))
+    z = torch.randn(shape, generator=g, device=device, dtype=torch.float32)
+    z.mul_(std)
+    return z.to(torch.bfloat16).view(torch.int16)
+
+
+def host_bits(t) -> np.ndarray:
+    """A device int16 tensor of bf16 bit patterns -> uint16 numpy array on the host."""
+    return t.cpu().numpy().view(np.uint16)
+
+
+def mlp_weights_device(H: int, N: int, layer: int = 0, std: float = 0.02, seed: int = SEED_WEIGHTS,
+                       device="cuda"):
+    """The weights of layer `layer` drawn on the device: (Wg [H][N], Wu [H][N], Wd [N][H]) int16 tensors."""
+    return (device_normal_bf16((H, N), std, seed + layer, 10, device=device),
+            device_normal_bf16((H, N), std, seed + layer, 11, device=device),
+            device_normal_bf16((N, H), std, seed + layer, 12, device=device))
+
+
 def activations_bf16(B: int, H: int, seed: int = SEED_X) -> np.ndarray:
     """x ~ N(0, 1) rounded to bf16: [B][H] uint16 bit patterns."""
     return normal_bf16((B, H), 1.0, seed)

@@ -1,0 +1,247 @@
+"""The five workloads at full size against the oracle.
+
+1. small layer, hidden 512 / intermediate 1408, one token, t at the 50th
+   percentile of 64 calibration vectors: every output checked;
+2. Llama-3.1-8B-shaped layer (4096 / 14336), one token, t from 256
+   calibration vectors at 50 / 70 / 90 %: every output checked;
+3. 32 Llama-shaped blocks (RMSNorm -> MLP -> residual), 128 decode tokens one
+   per call, per-layer targets evenly spread over [55 %, 85 %];
+4. 36 Qwen3-8B-shaped blocks (4096 / 12288) with routing over a 151936-entry
+   table (30 % dense), decode batches of 1, 8, 32 and 64 tokens, sparse path
+   at 50 %;
+5. one Llama-shaped block with routing (20 % of a 128256-entry table dense,
+   Zipf(1.1) token ids) at 256 and 2048 tokens per call and 40 / 60 / 80 / 90 %.
+
+For the stacks and the large batches the oracle checks a sample of tokens
+(first, last, and dense- and sparse-routed ones): block by block it takes the
+kernel's keep decisions inside the threshold band (and checks every other
+decision), then the final residual stream is compared.  Thresholds always come
+from the oracle's Eq. 3 on calibration vectors run through the oracle's own
+blocks; the model-sized weights are drawn on the device by the seeded
+generator in paper_2607_08991_gb300/inputs.py and copied to the host for the
+oracle.
+"""
+import concurrent.futures
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_08991_gb300 import inputs
+from tests import _parity as P
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+
+@pytest.fixture(scope="module")
+def sats():
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_08991_gb300 import sats as s
+    return s
+
+
+def _f32(v):
+    return float(np.float32(v))
+
+
+_POOL = concurrent.futures.ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1))
+
+
+def _rows_sparse_mlp(oracle, n, Wg, Wu, Wd, t, keep_hint=None, band_rel=0.0):
+    """oracle.sparse_mlp row by row on a thread pool (the C oracle releases the GIL);
+    the rows are independent, so this is the same computation."""
+    B = n.shape[0]
+    t = np.broadcast_to(np.asarray(t, np.float64), (B,))
+    futs = [_POOL.submit(oracle.sparse_mlp, n[b:b + 1], Wg, Wu, Wd, t[b:b + 1],
+                         None if keep_hint is None else keep_hint[b:b + 1], band_rel) for b in range(B)]
+    parts = [f.result() for f in futs]
+    return (np.concatenate([p[0] for p in parts]), np.concatenate([p[1] for p in parts]),
+            np.concatenate([p[2] for p in parts]), sum(p[3] for p in parts))
+
+
+# ----------------------------------------------------------------------------- single layers
+
+def test_config1_small_layer(sats, oracle):
+    H, N = inputs.SMALL_H, inputs.SMALL_N
+    w = inputs.mlp_weights(H, N)
+    cal = oracle.bf16_to_f64(inputs.activations_bf16(64, H, seed=inputs.SEED_CALIB))
+    t = _f32(oracle.percentile_threshold(oracle.gate_act(cal, w.Wg), 0.5))
+    xb = inputs.activations_bf16(1, H)
+    layer = sats.Layer(P.dev_u16(w.Wg), P.dev_u16(w.Wu), P.dev_u16(w.Wd))
+    ws = sats.Workspace(H, N, 1)
+    y = torch.full((1, H), float("nan"), device="cuda")
+    idx = torch.full((1, N), -1, dtype=torch.int32, device="cuda")
+    cnt = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+    sats.sparse_mlp(layer, P.dev_u16(xb), t, y, ws, idx, cnt)
+    assert sats.get_error(ws) == sats.OK
+    keep_gpu = P.keep_from_lists(idx, cnt, N)
+    y_ref, a_ref, keep_ref, _ = oracle.sparse_mlp(oracle.bf16_to_f64(xb), w.Wg, w.Wu, w.Wd, t,
+                                                 keep_hint=keep_gpu, band_rel=P.BAND_REL)
+    P.assert_keep_match(keep_gpu, keep_ref, a_ref, t)
+    P.assert_close(y.cpu().numpy(), y_ref)
+    layer.close()
+
+
+def test_config2_llama_layer_256_calibration_vectors(sats, oracle):
+    H, N = inputs.LLAMA_H, inputs.LLAMA_N
+    Wg, Wu, Wd = inputs.mlp_weights_device(H, N)
+    hg, hu, hd = (inputs.host_bits(m) for m in (Wg, Wu, Wd))
+    cal = oracle.bf16_to_f64(inputs.activations_bf16(256, H, seed=inputs.SEED_CALIB))
+    a_cal = np.concatenate(list(_POOL.map(lambda c: oracle.gate_act(cal[c:c + 16], hg), range(0, 256, 16))))
+    layer = sats.Layer(Wg, Wu, Wd)
+    ws = sats.Workspace(H, N, 1)
+    xb = inputs.activations_bf16(1, H)
+    x64 = oracle.bf16_to_f64(xb)
+    for k in (0.5, 0.7, 0.9):
+        t = _f32(oracle.percentile_threshold(a_cal, k))
+        y = torch.full((1, H), float("nan"), device="cuda")
+        idx = torch.full((1, N), -1, dtype=torch.int32, device="cuda")
+        cnt = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+        sats.sparse_mlp(layer, P.dev_u16(xb), t, y, ws, idx, cnt)
+        assert sats.get_error(ws) == sats.OK
+        keep_gpu = P.keep_from_lists(idx, cnt, N)
+        y_ref, a_ref, keep_ref, _ = oracle.sparse_mlp(x64, hg, hu, hd, t, keep_hint=keep_gpu, band_rel=P.BAND_REL)
+        P.assert_keep_match(keep_gpu, keep_ref, a_ref, t)
+        P.assert_close(y.cpu().numpy(), y_ref)
+        assert abs((1.0 - keep_gpu.mean()) - k) < 0.05
+    layer.close()
+
+
+# ----------------------------------------------------------------------------- stacks
+
+class _Stack:
+    """L blocks of one shape: device layers, norm gains, and thresholds calibrated by the
+    oracle (Eq. 3) on `n_cal` fp32 calibration vectors carried through the earlier blocks."""
+
+    def __init__(self, sats, oracle, L, H, N, targets, eps, n_cal, seed):
+        self.L, self.H, self.N, self.eps, self.seed = L, H, N, eps, seed
+        self.nw = [inputs.norm_weight(H, layer=l) for l in range(L)]
+        self.layers, self.t = [], []
+        cal = inputs.activations_f32(n_cal, H, seed=inputs.SEED_CALIB).astype(np.float64)
+        for l in range(L):
+            Wg, Wu, Wd = inputs.mlp_weights_device(H, N, layer=l, seed=seed)
+            self.layers.append(sats.Layer(Wg, Wu, Wd))
+            hg, hu, hd = (inputs.host_bits(m) for m in (Wg, Wu, Wd))
+            del Wg, Wu, Wd
+            n = oracle.rmsnorm(cal, self.nw[l], eps)
+            tl = _f32(oracle.percentile_threshold(oracle.gate_act(n, hg), targets[l]))
+            self.t.append(tl)
+            cal = cal + _rows_sparse_mlp(oracle, n, hg, hu, hd, tl)[0]
+
+    def host_weights(self, l):
+        Wg, Wu, Wd = inputs.mlp_weights_device(self.H, self.N, layer=l, seed=self.seed)
+        return tuple(inputs.host_bits(m) for m in (Wg, Wu, Wd))
+
+    def check(self, oracle, x0_rows, dense_rows, trace_rows, x_gpu_rows):
+        """Oracle blocks on the sampled tokens, following the kernel inside the band only."""
+        xs = x0_rows.astype(np.float64).copy()
+        for l in range(self.L):
+            hg, hu, hd = self.host_weights(l)
+            n = oracle.rmsnorm(xs, self.nw[l], self.eps)
+            t = np.where(dense_rows, 0.0, np.float64(self.t[l]))
+            y, a, keep, _ = _rows_sparse_mlp(oracle, n, hg, hu, hd, t, keep_hint=trace_rows[l], band_rel=P.BAND_REL)
+            P.assert_keep_match(trace_rows[l], keep, a, t)
+            xs = xs + y
+        P.assert_close(x_gpu_rows, xs)
+        return xs
+
+    def close(self):
+        for l in self.layers:
+            l.close()
+
+
+def test_config3_llama_stack_128_decode_tokens(sats, oracle):
+    L, H, N, T = inputs.LLAMA_L, inputs.LLAMA_H, inputs.LLAMA_N, 128
+    eps = 1e-5
+    targets = inputs.stack_sparsity_targets(L, 0.55, 0.85)
+    st = _Stack(sats, oracle, L, H, N, targets, eps, n_cal=2, seed=inputs.SEED_WEIGHTS)
+    x0 = inputs.activations_f32(T, H, seed=inputs.SEED_X + 3)
+    ws = sats.Workspace(H, N, 1)
+    nws = [P.dev(w) for w in st.nw]
+    sampled = [0, T - 1]
+    traces = {}
+    x = P.dev(x0.copy())
+    for tok in range(T):          # decode: one token per call through all L blocks
+        tr = torch.full((L, 1, N), 7, dtype=torch.uint8, device="cuda") if tok in sampled else None
+        sats.mlp_stack(st.layers, nws, st.t, eps, x[tok:tok + 1], ws, keep_trace=tr)
+        if tr is not None:
+            traces[tok] = tr
+    assert sats.get_error(ws) == sats.OK
+    xg = x.cpu().numpy()
+    assert np.all(np.isfinite(xg))
+    trace_rows = np.concatenate([traces[t].cpu().numpy() for t in sampled], axis=1)   # [L][rows][N]
+    assert set(np.unique(trace_rows).tolist()) <= {0, 1}
+    st.check(oracle, x0[sampled], np.zeros(len(sampled), bool), trace_rows, xg[sampled])
+    sparsity = 1.0 - trace_rows.mean(axis=(1, 2))
+    assert abs(sparsity.mean() - 0.70) < 0.08          # targets spread over [0.55, 0.85], mean 0.70
+    st.close()
+
+
+def test_config4_qwen_routed_stack(sats, oracle):
+    L, H, N, V = inputs.QWEN_L, inputs.QWEN_H, inputs.QWEN_N, inputs.QWEN_V
+    eps = 1e-6
+    st = _Stack(sats, oracle, L, H, N, [0.5] * L, eps, n_cal=2, seed=inputs.SEED_WEIGHTS + 100)
+    lut = inputs.routing_lut(V, 0.3)
+    assert abs(lut.mean() - 0.3) < 0.01
+    nws = [P.dev(w) for w in st.nw]
+    lut_d = P.dev(lut)
+    for B in (1, 8, 32, 64):
+        x0 = inputs.activations_f32(B, H, seed=inputs.SEED_X + 40 + B)
+        ids = inputs.token_ids_uniform(B, V, seed=inputs.SEED_IDS + B)
+        dense = lut[ids] == 1
+        ws = sats.Workspace(H, N, B)
+        x = P.dev(x0.copy())
+        trace = torch.full((L, B, N), 7, dtype=torch.uint8, device="cuda")
+        sats.mlp_stack(st.layers, nws, st.t, eps, x, ws, token_ids=P.dev(ids), lut=lut_d, keep_trace=trace)
+        assert sats.get_error(ws) == sats.OK
+        tr = trace.cpu().numpy()
+        assert set(np.unique(tr).tolist()) <= {0, 1}
+        assert tr[:, dense].all()                     # base-path tokens keep every neuron in every block
+        # one base-path and one sparse-path token per batch (the only token at B = 1)
+        rows = sorted(({int(np.argmax(dense))} if dense.any() else set())
+                      | ({int(np.argmax(~dense))} if (~dense).any() else set()))
+        xg = x.cpu().numpy()
+        assert np.all(np.isfinite(xg))
+        st.check(oracle, x0[rows], dense[rows], tr[:, rows], xg[rows])
+        sp = 1.0 - tr[:, ~dense].mean() if (~dense).any() else 0.5
+        assert abs(sp - 0.5) < 0.1
+    st.close()
+
+
+def test_config5_llama_prefill_routed(sats, oracle):
+    H, N, V = inputs.LLAMA_H, inputs.LLAMA_N, inputs.LLAMA_V
+    eps = 1e-5
+    Wg, Wu, Wd = inputs.mlp_weights_device(H, N, seed=inputs.SEED_WEIGHTS + 200)
+    hg, hu, hd = (inputs.host_bits(m) for m in (Wg, Wu, Wd))
+    layer = sats.Layer(Wg, Wu, Wd)
+    del Wg, Wu, Wd
+    nw = inputs.norm_weight(H)
+    cal = inputs.activations_f32(8, H, seed=inputs.SEED_CALIB).astype(np.float64)
+    a_cal = oracle.gate_act(oracle.rmsnorm(cal, nw, eps), hg)
+    lut = inputs.routing_lut(V, 0.2, seed=inputs.SEED_LUT + 5)
+    for B in (256, 2048):
+        ids = inputs.token_ids_zipf(B, V, seed=inputs.SEED_IDS + B)
+        dense = lut[ids] == 1
+        x0 = inputs.activations_f32(B, H, seed=inputs.SEED_X + 50 + B)
+        ws = sats.Workspace(H, N, B)
+        rows = sorted({0, B - 1, B // 2} | ({int(np.argmax(dense))} if dense.any() else set())
+                      | ({int(np.argmax(~dense))} if (~dense).any() else set()))
+        for k in (0.4, 0.6, 0.8, 0.9):
+            t = _f32(oracle.percentile_threshold(a_cal, k))
+            x = P.dev(x0.copy())
+            trace = torch.full((1, B, N), 7, dtype=torch.uint8, device="cuda")
+            sats.mlp_stack([layer], [P.dev(nw)], [t], eps, x, ws, token_ids=P.dev(ids), lut=P.dev(lut),
+                           keep_trace=trace)
+            assert sats.get_error(ws) == sats.OK
+            tr = trace.cpu().numpy()
+            assert tr[0][dense].all()
+            n = oracle.rmsnorm(x0[rows].astype(np.float64), nw, eps)
+            tt = np.where(dense[rows], 0.0, np.float64(t))
+            y, a, keep, _ = _rows_sparse_mlp(oracle, n, hg, hu, hd, tt, keep_hint=tr[0][rows], band_rel=P.BAND_REL)
+            P.assert_keep_match(tr[0][rows], keep, a, tt)
+            P.assert_close(x.cpu().numpy()[rows], x0[rows].astype(np.float64) + y)
+            if (~dense).any():
+                assert abs((1.0 - tr[0][~dense].mean()) - k) < 0.08
+    layer.close()
