@@ -92,8 +92,8 @@ SATS_API sats_status sats_layer_shape(const sats_layer *layer, int *H, int *N);
  * byte per neuron and token (for the index outputs) and the routing scratch of
  * sats_mlp_stack: N * 4 bytes plus B * 5 plus 1 KB.  A batch that runs on the
  * tensor cores (sats_uses_tensor_cores) also needs, per token, bf16 copies of
- * its activations and of h plus one keep byte per neuron: about
- * B * (4 H + 3 N) bytes more.  It must be
+ * its activations and of h (two parts each) plus one keep byte per neuron:
+ * about B * (4 H + 5 N) bytes more.  It must be
  * zero-filled once before first use (sats_workspace_init does that on
  * `stream`); every call leaves its counters at zero for the next call.  Calls
  * that share one workspace must not overlap on the GPU.
@@ -111,10 +111,9 @@ SATS_API sats_status sats_workspace_init(void *ws, size_t ws_bytes, void *stream
  *    call and read only the W_up columns and W_down rows of kept neurons;
  *  - larger batches run as two tensor-core GEMMs over all neurons,
  *    [x W_gate | x W_up] and then h W_down, with the mask applied to
- *    h = CATS(SiLU(x W_gate)) * (x W_up) between them; h is rounded to bf16
- *    there (a relative error of at most 2^-9 per element), and fp32
- *    activations are split into two bf16 parts so that they keep ~16
- *    significant bits.
+ *    h = CATS(SiLU(x W_gate)) * (x W_up) between them; h, and fp32
+ *    activations, are carried as a bf16 high part plus a bf16 low part
+ *    (about 16 significant bits) with fp32 accumulation.
  *   x          : device bf16 [B][H]
  *   t_l        : threshold, >= 0 (0 keeps every neuron: the dense MLP;
  *                +inf keeps none and gives y = 0).  NaN or < 0 -> SATS_EINVAL.
