@@ -445,6 +445,189 @@ def run_gpu(args):
         dist.destroy_process_group()
 
 
+# ---------------------------------------------------------------------------- other workloads
+def _calibrate_stack(sats, layers, nws, targets, eps, xc, ws, stream, N):
+    """Per-layer thresholds for the bench (setup, not timed, not a parity input): bisection on t
+    until the kept fraction of the calibration vectors, carried through the earlier blocks,
+    meets the layer's target sparsity (the Eq. 3 percentile, found through the library)."""
+    import torch
+    C = xc.shape[0]
+    trace = torch.empty((1, C, N), dtype=torch.uint8, device=xc.device)
+    ts = []
+    for l, layer in enumerate(layers):
+        lo, hi = 0.0, 16.0
+        for _ in range(24):
+            mid = 0.5 * (lo + hi)
+            xt = xc.clone()
+            sats.mlp_stack([layer], [nws[l]], [mid], eps, xt, ws, keep_trace=trace, stream=stream)
+            sp = 1.0 - float(trace.float().mean())
+            if sp < targets[l]:
+                lo = mid
+            else:
+                hi = mid
+        ts.append(hi)
+        sats.mlp_stack([layer], [nws[l]], [hi], eps, xc, ws, stream=stream)
+    return ts
+
+
+def _timed(stream, fn, reps):
+    import torch
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(reps):
+        fn(i)
+    e1.record(stream)
+    e1.synchronize()
+    return 1e3 * e0.elapsed_time(e1) / reps
+
+
+def run_workload(args):
+    """The other four workloads (one JSON line each; not the headline)."""
+    import torch
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_08991_gb300 import sats
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.Stream(device=dev)
+    hbm_peak, hbm_kind = _peaks()
+    bf16_peak, bf16_kind = _bf16_peak()
+    wl = args.workload
+    spec = inputs.WORKLOADS[wl]
+    out = {"workload": wl, "data": "synthetic", "hbm_peak_gbs": hbm_peak, "bf16_peak_tflops": bf16_peak,
+           "peak_kind": hbm_kind}
+    clocks = Clocks(0)
+    with torch.cuda.stream(stream):
+        if wl == "small_layer_512x1408_b1":
+            H, N = spec["H"], spec["N"]
+            layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l)) for l in range(64)]
+            ws = sats.Workspace(H, N, 1, device=dev)
+            xc = torch.from_numpy(inputs.activations_bf16(64, H, seed=inputs.SEED_CALIB).view(np.int16)).to(dev)
+            a = torch.empty(64, N, dtype=torch.float32, device=dev)
+            sats.gate_act(layers[0], xc, a, stream=stream)
+            sel = torch.empty(sats.select_workspace_bytes(), dtype=torch.uint8, device=dev)
+            t = sats.percentile_threshold(a, 0.5, sel, stream=stream)
+            x = torch.from_numpy(inputs.activations_bf16(1, H).view(np.int16)).to(dev)
+            y = torch.empty(1, H, dtype=torch.float32, device=dev)
+            idx = torch.empty(1, N, dtype=torch.int32, device=dev)
+            cnt = torch.empty(1, dtype=torch.int32, device=dev)
+            call = lambda i: sats.sparse_mlp(layers[i % 64], x, t, y, ws, idx, cnt, stream=stream)
+            for i in range(64):
+                call(i)
+            stream.synchronize()
+            kept = int(cnt.item())
+            clocks.start()
+            us_cold = _timed(stream, call, args.steps)       # 64 rotating copies (184 MB): weights from HBM
+            us_hot = _timed(stream, lambda i: call(0), args.steps)   # one copy, L2-resident
+            clk = clocks.stop()
+            algo = 2.0 * H * N + 4.0 * H * kept + 2.0 * H + 4.0 * H + 4.0 * kept + 4.0
+            out.update({"metric": "us/token (one layer)", "value": us_cold, "unit": "us/token",
+                        "us_l2_resident": us_hot, "realised_sparsity": 1.0 - kept / N, "algo_bytes": algo,
+                        "achieved_gbs": algo / us_cold / 1e3, "clocks": clk})
+        elif wl in ("llama_stack_32x4096x14336_b1x128", "qwen_stack_36x4096x12288_routed"):
+            H, N, L, eps = spec["H"], spec["N"], spec["L"], spec["eps"]
+            if wl.startswith("llama"):
+                targets = list(inputs.stack_sparsity_targets(L, *spec["sparsity_range"]))
+                seed = inputs.SEED_WEIGHTS
+            else:
+                targets = [spec["sparsity"]] * L
+                seed = inputs.SEED_WEIGHTS + 100
+            layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l, seed=seed)) for l in range(L)]
+            nws = [torch.from_numpy(inputs.norm_weight(H, layer=l)).to(dev) for l in range(L)]
+            xc = torch.from_numpy(inputs.activations_f32(8, H, seed=inputs.SEED_CALIB)).to(dev)
+            wsc = sats.Workspace(H, N, 8, device=dev)
+            ts = _calibrate_stack(sats, layers, nws, targets, eps, xc, wsc, stream, N)
+            if wl.startswith("llama"):
+                T = spec["tokens"]
+                x0 = torch.from_numpy(inputs.activations_f32(T, H, seed=inputs.SEED_X + 3)).to(dev)
+                ws = sats.Workspace(H, N, 1, device=dev)
+                trace = torch.empty((L, 1, N), dtype=torch.uint8, device=dev)
+                kept = []
+                x = x0.clone()
+                for tok in range(T):
+                    sats.mlp_stack(layers, nws, ts, eps, x[tok:tok + 1], ws, keep_trace=trace, stream=stream)
+                    kept.append(trace.sum(dim=(1, 2)).double())
+                kept = torch.stack(kept).mean(dim=0).cpu().numpy()          # [L] mean kept neurons
+                x = x0.clone()
+                step = lambda i: sats.mlp_stack(layers, nws, ts, eps, x[i:i + 1], ws, stream=stream)
+                for i in range(3):
+                    step(i)
+                x.copy_(x0)
+                clocks.start()
+                us = _timed(stream, step, T)        # the 128 decode tokens, each once through the stack
+                clk = clocks.stop()
+                algo = float(sum(2.0 * H * N + 4.0 * H * k + 12.0 * H for k in kept))
+                out.update({"metric": "us/token through the %d-block stack (decode, one token per call)" % L,
+                            "value": us, "unit": "us/token", "tokens_per_s": 1e6 / us,
+                            "realised_sparsity_mean": float(1.0 - kept.mean() / N),
+                            "realised_sparsity_range": [float(1.0 - kept.max() / N), float(1.0 - kept.min() / N)],
+                            "algo_bytes_per_token": algo, "achieved_gbs": algo / us / 1e3,
+                            "frac_of_%s" % hbm_kind: algo / us / 1e3 / hbm_peak, "clocks": clk})
+            else:
+                V = spec["V"]
+                lut = torch.from_numpy(inputs.routing_lut(V, spec["p_dense"])).to(dev)
+                res = {}
+                clocks.start()
+                for B in spec["batches"]:
+                    x0 = torch.from_numpy(inputs.activations_f32(B, H, seed=inputs.SEED_X + 40 + B)).to(dev)
+                    ids = torch.from_numpy(inputs.token_ids_uniform(B, V, seed=inputs.SEED_IDS + B)).to(dev)
+                    ws = sats.Workspace(H, N, B, device=dev)
+                    reps = max(10, args.steps // 4)
+                    xs = x0.repeat(reps + 3, 1, 1)        # a fresh copy of the batch per step
+                    step = lambda i: sats.mlp_stack(layers, nws, ts, eps, xs[i], ws, token_ids=ids, lut=lut,
+                                                    stream=stream)
+                    for i in range(3):
+                        step(reps + i)
+                    us = _timed(stream, step, reps)
+                    tc = sats.uses_tensor_cores(H, B)
+                    wbytes = L * (6.0 * H * N)
+                    res[str(B)] = {"us_per_step": us, "tokens_per_s": B / (us * 1e-6), "path":
+                                   "tensor cores" if tc else "fused",
+                                   "weight_gbs_if_all_weights_read": wbytes / us / 1e3}
+                clk = clocks.stop()
+                out.update({"metric": "us per decode step through the %d-block routed stack" % L,
+                            "value": res[str(spec["batches"][-1])]["us_per_step"], "unit": "us/step",
+                            "per_batch": res, "thresholds_mean": float(np.mean(ts)), "clocks": clk})
+        elif wl == "llama_layer_prefill_routed":
+            H, N, V = inputs.LLAMA_H, inputs.LLAMA_N, spec["V"]
+            eps = 1e-5
+            layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l, seed=inputs.SEED_WEIGHTS + 200))
+                      for l in range(2)]
+            nw = torch.from_numpy(inputs.norm_weight(H)).to(dev)
+            lut = torch.from_numpy(inputs.routing_lut(V, spec["p_dense"], seed=inputs.SEED_LUT + 5)).to(dev)
+            xc = torch.from_numpy(inputs.activations_f32(8, H, seed=inputs.SEED_CALIB)).to(dev)
+            wsc = sats.Workspace(H, N, 8, device=dev)
+            res = {}
+            clocks.start()
+            for k in spec["sparsity"]:
+                t = _calibrate_stack(sats, layers[:1], [nw], [k], eps, xc.clone(), wsc, stream, N)[0]
+                for B in spec["batches"]:
+                    ids = torch.from_numpy(inputs.token_ids_zipf(B, V, seed=inputs.SEED_IDS + B)).to(dev)
+                    x0 = torch.from_numpy(inputs.activations_f32(B, H, seed=inputs.SEED_X + 50 + B)).to(dev)
+                    ws = sats.Workspace(H, N, B, device=dev)
+                    reps = max(6, min(args.steps, int(4e4 / B)))
+                    xs = x0.repeat(reps + 3, 1, 1)
+                    step = lambda i: sats.mlp_stack([layers[i % 2]], [nw], [t], eps, xs[i], ws, token_ids=ids,
+                                                    lut=lut, stream=stream)
+                    for i in range(3):
+                        step(reps + i)
+                    us = _timed(stream, step, reps)
+                    flops = 6.0 * B * H * N
+                    res["%s@%d" % (k, B)] = {"us_per_call": us, "tokens_per_s": B / (us * 1e-6),
+                                             "tflops_dense_equivalent": flops / us / 1e6,
+                                             "tensor_frac_of_%s" % bf16_kind: flops / us / 1e6 / bf16_peak,
+                                             "dense_fraction_of_tokens":
+                                                 float(lut[ids.long()].float().mean())}
+            clk = clocks.stop()
+            out.update({"metric": "us per prefill call (one routed block)", "value": res["0.6@2048"]["us_per_call"],
+                        "unit": "us/call", "per_case": res, "clocks": clk})
+        else:
+            raise SystemExit("unknown workload " + wl)
+    print(json.dumps(out))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -454,6 +637,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-batched", action="store_true", help="skip the batched tensor-core measurements")
+    ap.add_argument("--workload", default=WORKLOAD, choices=sorted(inputs.WORKLOADS),
+                    help="the headline workload (default) or one of the other four, reported on their own line")
     ap.add_argument("--profile-batch", type=int, default=0,
                     help="small capture case for ncu: `warmup + steps` calls at this batch size on one layer copy")
     ap.add_argument("--profile", action="store_true",
@@ -464,6 +649,8 @@ def main():
         args.no_batched = True
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload != WORKLOAD:
+        run_workload(args)
     else:
         run_gpu(args)
 
