@@ -67,6 +67,8 @@ def _load():
         lib.oracle_rmsnorm.argtypes = [I, I, P, P, D, P]
         lib.oracle_mlp_stack.argtypes = [I, I, I, I, P, P, P, P, P, D, P, P, I, P, P, D, P]
         lib.oracle_mlp_stack.restype = I64
+        lib.oracle_layer_err.argtypes = [I, I, I, P, P, P, P, I, P, D, P, P]
+        lib.oracle_sats_select.argtypes = [I, I, P, P, P, D, I, D, D, P, P, P]
         _lib = lib
     return _lib
 
@@ -231,3 +233,87 @@ def mlp_stack(x, Wg: Sequence, Wu: Sequence, Wd: Sequence, norm_w: Sequence, t, 
     if nb < 0:
         raise ValueError("token id outside the vocabulary")
     return x, keep, int(nb)
+
+
+def layer_err(x, Wg, Wu, Wd, t, eps: float = 1e-6):
+    """Sec. 3.1, Eq. 6 at each candidate threshold t[k] on the calibration inputs x [C][H]
+    (the block's MLP inputs).  Returns (err [K], sp [K]): the mean relative L2 distortion
+    ||y - y~_t|| / (||y|| + eps) and the mean fraction of neurons with |a| < t."""
+    x = _f64(x)
+    Wg, Wu, Wd = _u16(Wg), _u16(Wu), _u16(Wd)
+    C, H = x.shape
+    N = Wg.shape[1]
+    t = _f64(np.atleast_1d(t))
+    err = np.empty(t.size, dtype=np.float64)
+    sp = np.empty(t.size, dtype=np.float64)
+    _load().oracle_layer_err(C, H, N, _ptr(x), _ptr(Wg), _ptr(Wu), _ptr(Wd), t.size, _ptr(t), float(eps),
+                             _ptr(err), _ptr(sp))
+    return err, sp
+
+
+def sats_select(t, err, sp, s_tar: float, guard: int = -1, guard_t: float = 0.0, guard_sp: float = 0.0):
+    """Sec. 3.1, Eqs. 7-10 over a candidate table t, err, sp of shape [L][K].
+    Returns (b*, T*(b*) [L], S(b*))."""
+    t, err, sp = _f64(t), _f64(err), _f64(sp)
+    L, K = t.shape
+    assert err.shape == (L, K) and sp.shape == (L, K)
+    b = np.zeros(1)
+    S = np.zeros(1)
+    tout = np.empty(L, dtype=np.float64)
+    _load().oracle_sats_select(L, K, _ptr(t), _ptr(err), _ptr(sp), float(s_tar), int(guard), float(guard_t),
+                               float(guard_sp), _ptr(b), _ptr(tout), _ptr(S))
+    return float(b[0]), tout, float(S[0])
+
+
+def sats_calibrate(x_cal, Wg: Sequence, Wu: Sequence, Wd: Sequence, norm_w: Sequence, eps: float, s_tar: float,
+                   K0: int = 20, K1: int = 8, guardrail: bool = True, err_eps: float = 1e-6):
+    """SATS calibration of a stack (Sec. 3.1, Eqs. 3, 6-10, coarse-to-fine; Sec. 4 guardrail),
+    in the paper's order:
+
+    1. the dense stack on the calibration inputs gives each block's MLP inputs
+       n_l = RMSNorm(x_l) w_l, with x_{l+1} = x_l + MLP_l(n_l);
+    2. coarse candidates T_l: Eq. 3 percentiles of |SiLU(n_l W_gate)| at k / K0, k = 1 .. K0-1;
+    3. Err_l(t) and sp_l(t) for every candidate (Eq. 6);
+    4. b* and T*(b*) (Eqs. 7-10); with the guardrail the last block keeps the CATS
+       threshold at s_tar (its Eq. 3 percentile);
+    5. fine candidates: K1 thresholds evenly spaced strictly between the coarse candidates
+       that neighbour t*_l (0 below the first; the largest |a| above the last);
+    6. Eqs. 6-10 again over coarse and fine candidates together.
+
+    Returns dict(t [L], b, S, coarse=(t, err, sp), fine=(t, err, sp) [L][K0-1+K1])."""
+    x = _f64(x_cal).copy()
+    L = len(Wg)
+    inputs_l, amax, guard = [], [], (L - 1 if guardrail else -1)
+    cand = np.zeros((L, K0 - 1))
+    for l in range(L):
+        n = rmsnorm(x, norm_w[l], eps)
+        inputs_l.append(n)
+        a = gate_act(n, Wg[l])
+        amax.append(float(np.abs(a).max()))
+        cand[l] = [percentile_threshold(a, k / K0) for k in range(1, K0)]
+        x = x + dense_mlp(n, Wg[l], Wu[l], Wd[l])
+    err0 = np.zeros_like(cand)
+    sp0 = np.zeros_like(cand)
+    for l in range(L):
+        err0[l], sp0[l] = layer_err(inputs_l[l], Wg[l], Wu[l], Wd[l], cand[l], err_eps)
+    g_t = g_sp = 0.0
+    if guard >= 0:
+        g_t = percentile_threshold(gate_act(inputs_l[guard], Wg[guard]), s_tar)
+        g_sp = float(layer_err(inputs_l[guard], Wg[guard], Wu[guard], Wd[guard], [g_t], err_eps)[1][0])
+    b0, t0, _ = sats_select(cand, err0, sp0, s_tar, guard, g_t, g_sp)
+    fine = np.zeros((L, K1))
+    for l in range(L):
+        below = cand[l][cand[l] < t0[l]]
+        above = cand[l][cand[l] > t0[l]]
+        lo = below.max() if below.size else 0.0
+        hi = above.min() if above.size else amax[l]
+        fine[l] = lo + (hi - lo) * np.arange(1, K1 + 1) / (K1 + 1)
+    err1 = np.zeros_like(fine)
+    sp1 = np.zeros_like(fine)
+    for l in range(L):
+        err1[l], sp1[l] = layer_err(inputs_l[l], Wg[l], Wu[l], Wd[l], fine[l], err_eps)
+    t_all = np.concatenate([cand, fine], axis=1)
+    e_all = np.concatenate([err0, err1], axis=1)
+    s_all = np.concatenate([sp0, sp1], axis=1)
+    b, t, S = sats_select(t_all, e_all, s_all, s_tar, guard, g_t, g_sp)
+    return dict(t=t, b=b, S=S, coarse=(cand, err0, sp0), fine=(t_all, e_all, s_all), guard=(g_t, g_sp))

@@ -24,7 +24,9 @@
  *   oracle_mlp_stack          Sec. 3.2: a token routed to the sparse path uses
  *                             the thresholded MLP in every block, a base token
  *                             uses the dense MLP in every block.
- *   oracle_layer_err ...      Sec. 3.1, Eqs. 6-10 (SATS calibration)
+ *   oracle_layer_err          Sec. 3.1, Eq. 6  Err_l(t) and the sparsity sp_l(t)
+ *                             of one block at candidate thresholds
+ *   oracle_sats_select        Sec. 3.1, Eqs. 7-10 t*_l(b), T*(b), S(b), b*
  *
  * Layouts follow the paper's row-vector convention x W: W_gate and W_up are
  * [H][N] (hidden x intermediate), W_down is [N][H], all row-major bf16 bit
@@ -293,4 +295,96 @@ int64_t oracle_mlp_stack(int L, int B, int H, int N,
     free(y);
     free(keep);
     return in_band;
+}
+
+/* Sec. 3.1, Eq. 6: the local thresholding error of one block at each of K
+ * candidate thresholds t[k], over C calibration inputs x [C][H] (the block's
+ * MLP inputs):
+ *   err[k] = (1/C) sum_c ||y(x_c) - y~_{t_k}(x_c)||_2 / (||y(x_c)||_2 + eps)
+ * with y the dense output (Eq. 1) and y~_t the thresholded output (Eqs. 4-5).
+ * sp[k] = (1/C) sum_c (number of neurons with |a_j| < t_k) / N, the realised
+ * sparsity of the block under t_k that Eq. 9 averages. */
+void oracle_layer_err(int C, int H, int N, const double *x, const uint16_t *Wg, const uint16_t *Wu,
+                      const uint16_t *Wd, int K, const double *t, double eps, double *err, double *sp)
+{
+    double *y = (double *)malloc(sizeof(double) * (size_t)C * H);
+    double *yt = (double *)malloc(sizeof(double) * (size_t)C * H);
+    uint8_t *keep = (uint8_t *)malloc((size_t)C * N);
+    double *tt = (double *)malloc(sizeof(double) * (size_t)(C > 0 ? C : 1));
+    oracle_dense_mlp(C, H, N, x, Wg, Wu, Wd, y);
+    for (int k = 0; k < K; ++k) {
+        for (int c = 0; c < C; ++c) tt[c] = t[k];
+        oracle_sparse_mlp(C, H, N, x, Wg, Wu, Wd, tt, NULL, 0.0, yt, NULL, keep);
+        double e = 0.0, z = 0.0;
+        for (int c = 0; c < C; ++c) {
+            double dd = 0.0, yy = 0.0;
+            for (int i = 0; i < H; ++i) {
+                const double d = y[(size_t)c * H + i] - yt[(size_t)c * H + i];
+                dd += d * d;
+                yy += y[(size_t)c * H + i] * y[(size_t)c * H + i];
+            }
+            e += sqrt(dd) / (sqrt(yy) + eps);
+            int64_t off = 0;
+            for (int j = 0; j < N; ++j) off += keep[(size_t)c * N + j] ? 0 : 1;
+            z += (double)off / (double)N;
+        }
+        err[k] = C > 0 ? e / C : 0.0;
+        sp[k] = C > 0 ? z / C : 0.0;
+    }
+    free(y);
+    free(yt);
+    free(keep);
+    free(tt);
+}
+
+/* Sec. 3.1, Eqs. 7-10 over a table of candidates: t, err, sp are [L][K]
+ * (candidate k of block l with its Eq. 6 error and its sparsity).  Every block
+ * also has the candidate t = 0 (nothing removed: error 0, sparsity 0).
+ *   Eq. 7:  t*_l(b) = max{t in T_l : Err_l(t) <= b}
+ *   Eq. 8:  T*(b) = [t*_1(b), ..., t*_L(b)]
+ *   Eq. 9:  S(b) = (1/L) sum_l sp_l(t*_l(b))
+ *   Eq. 10: b* = argmin_b |S(b) - s_tar|
+ * b ranges over 0 and every error value in the table (S changes only there),
+ * in increasing order; a tie in Eq. 10 goes to the smaller budget.  Block
+ * `guard` (if >= 0) keeps the fixed threshold guard_t with sparsity guard_sp
+ * and takes no part in Eq. 7 (the final-block guardrail of Sec. 4).
+ * Writes b*, T*(b*) and S(b*). */
+void oracle_sats_select(int L, int K, const double *t, const double *err, const double *sp, double s_tar,
+                        int guard, double guard_t, double guard_sp, double *b_out, double *t_out, double *S_out)
+{
+    const int nb = 1 + L * K;
+    double *budgets = (double *)malloc(sizeof(double) * (size_t)nb);
+    budgets[0] = 0.0;
+    for (int i = 0; i < L * K; ++i) budgets[1 + i] = err[i];
+    qsort(budgets, (size_t)nb, sizeof(double), cmp_double);
+    double best_gap = INFINITY, best_b = 0.0, best_S = 0.0;
+    for (int q = 0; q < nb; ++q) {
+        const double b = budgets[q];
+        if (q > 0 && b == budgets[q - 1]) continue;
+        double S = 0.0;
+        for (int l = 0; l < L; ++l) {
+            if (l == guard) { S += guard_sp; continue; }
+            double tl = 0.0, sl = 0.0;            /* the t = 0 candidate */
+            for (int k = 0; k < K; ++k) {
+                const int i = l * K + k;
+                if (err[i] <= b && t[i] > tl) { tl = t[i]; sl = sp[i]; }
+            }
+            S += sl;
+        }
+        S /= L;
+        const double gap = fabs(S - s_tar);
+        if (gap < best_gap) { best_gap = gap; best_b = b; best_S = S; }
+    }
+    for (int l = 0; l < L; ++l) {
+        if (l == guard) { t_out[l] = guard_t; continue; }
+        double tl = 0.0;
+        for (int k = 0; k < K; ++k) {
+            const int i = l * K + k;
+            if (err[i] <= best_b && t[i] > tl) tl = t[i];
+        }
+        t_out[l] = tl;
+    }
+    *b_out = best_b;
+    *S_out = best_S;
+    free(budgets);
 }
