@@ -246,6 +246,66 @@ SATS_API sats_status sats_percentile_threshold(const float *a, int64_t n, double
                                       void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * SATS calibration (Sec. 3.1): choose each block's threshold by its local
+ * distortion instead of a percentile.
+ *
+ * sats_rmsnorm -- out[b] = x[b] / sqrt(mean_i x[b][i]^2 + eps) * w, the
+ *   pre-MLP normalisation of a decoder block.  x, out: device fp32 [B][H];
+ *   w: device fp32 [H].
+ *
+ * sats_gate_act_f32 -- sats_gate_act for fp32 activations x [B][H].
+ *
+ * sats_layer_err -- Eq. 6 for K candidate thresholds t (host fp32 [K], each
+ *   >= 0) on C calibration inputs x (device fp32 [C][H], the block's MLP
+ *   inputs):
+ *     err[k] = (1/C) sum_c ||y(x_c) - y~_{t_k}(x_c)||_2 / (||y(x_c)||_2 + eps)
+ *     sp[k]  = (1/C) sum_c (neurons with |a| < t_k) / N
+ *   y is the dense output (Eq. 1), y~_t the thresholded one (Eqs. 4-5), both
+ *   computed by the library's MLP kernels.  err, sp: host double [K].  ws:
+ *   device workspace of sats_layer_err_workspace_bytes(H, N, C, K) bytes,
+ *   256-byte aligned (no initialisation needed).  Synchronises `stream`.
+ *
+ * sats_sats_select -- Eqs. 7-10 on the host over a candidate table t, err,
+ *   sp (host double [L][K]; every block also has the candidate t = 0 with
+ *   error 0 and sparsity 0):
+ *     t*_l(b) = max{t in T_l : Err_l(t) <= b}             (Eq. 7)
+ *     S(b) = (1/L) sum_l sp_l(t*_l(b))                     (Eqs. 8-9)
+ *     b* = argmin_b |S(b) - s_tar|                         (Eq. 10)
+ *   over b in {0} and every error in the table, ties to the smaller b.  Block
+ *   `guard` (-1 for none) keeps guard_t (sparsity guard_sp) and takes no part
+ *   in Eq. 7.  Writes b*, t_out[L] = T*(b*) and S(b*).
+ *
+ * sats_sats_calibrate -- the whole calibration of an L-block stack, in the
+ *   paper's order: (1) the dense stack on the calibration inputs x_cal
+ *   (device fp32 [C][H]) gives each block's MLP inputs RMSNorm(x_l) w_l;
+ *   (2) coarse candidates: Eq. 3 percentiles of |SiLU(n_l W_gate)| at k/K0,
+ *   k = 1..K0-1; (3) Eq. 6 for each; (4) Eqs. 7-10; (5) K1 fine candidates
+ *   evenly spaced strictly between the coarse candidates that neighbour each
+ *   block's choice (0 below the first, the largest |a| above the last); (6)
+ *   Eqs. 6-10 over coarse and fine candidates together.  With guardrail != 0
+ *   the last block keeps the CATS threshold (the Eq. 3 percentile at s_tar),
+ *   as Sec. 4 does.  Writes t_out (host fp32 [L]), b* and S(b*), and, if all
+ *   three are given, the candidate table (host double [L][K0 - 1 + K1]).
+ *   ws: sats_sats_workspace_bytes(H, N, C, L, K0, K1) bytes, 256-byte aligned.
+ *   Synchronises `stream`.
+ */
+SATS_API sats_status sats_rmsnorm(const float *x, int B, int H, const float *w, float eps, float *out,
+                                  void *stream);
+SATS_API sats_status sats_gate_act_f32(const sats_layer *layer, const float *x, int B, float *a, void *stream);
+SATS_API size_t sats_layer_err_workspace_bytes(int H, int N, int C, int K);
+SATS_API sats_status sats_layer_err(const sats_layer *layer, const float *x, int C, const float *t, int K,
+                                    float eps, double *err, double *sp, void *ws, size_t ws_bytes, void *stream);
+SATS_API sats_status sats_sats_select(const double *t, const double *err, const double *sp, int L, int K,
+                                      double s_tar, int guard, double guard_t, double guard_sp, double *b_out,
+                                      double *t_out, double *S_out);
+SATS_API size_t sats_sats_workspace_bytes(int H, int N, int C, int L, int K0, int K1);
+SATS_API sats_status sats_sats_calibrate(const sats_layer *const *layers, const float *const *norm_w, int L,
+                                         float eps, const float *x_cal, int C, double s_tar, int K0, int K1,
+                                         int guardrail, float err_eps, float *t_out, double *b_out, double *S_out,
+                                         double *table_t, double *table_err, double *table_sp, void *ws,
+                                         size_t ws_bytes, void *stream);
+
+/*
  * sats_get_error -- synchronises `stream`, reads the status word in the
  * workspace, clears it, and returns SATS_OK, SATS_EDEVICE (bad token id) or
  * SATS_ETIMEOUT (a device wait gave up).

@@ -57,10 +57,9 @@ static bool bad_threshold(float t) { return std::isnan(t) || t < 0.0f; }
 // Runs one block over B tokens: on the tensor cores when the batch is larger
 // than one pass of the fused kernel, else the fused kernel in passes of
 // fused_tokens_per_pass(H) tokens.
-static sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B, const float *t_per_pass_l,
-                             const float *norm_w, float eps, const uint8_t *dense_flags, int out_mode, float *out,
-                             int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws,
-                             cudaStream_t stream)
+sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B, const float *t_per_pass_l,
+                      const float *norm_w, float eps, const uint8_t *dense_flags, int out_mode, float *out,
+                      int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws, cudaStream_t stream)
 {
     const int H = layer->H, N = layer->N;
     const WsLayout L = ws_layout(H, N, B);

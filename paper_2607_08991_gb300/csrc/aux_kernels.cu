@@ -113,9 +113,23 @@ __global__ void __launch_bounds__(kRouteThreads) route_kernel(const int32_t *ids
 }
 
 // ------------------------------------------------------------------ calibration
+// 8 consecutive activations of token row xr starting at element 8 v, as floats.
+__device__ __forceinline__ void load_x8(const uint16_t *xr, int v, float (&xf)[8])
+{
+    unpack8(reinterpret_cast<const uint4 *>(xr)[v], xf);
+}
+__device__ __forceinline__ void load_x8(const float *xr, int v, float (&xf)[8])
+{
+    const float4 p = reinterpret_cast<const float4 *>(xr)[2 * v], q = reinterpret_cast<const float4 *>(xr)[2 * v + 1];
+    xf[0] = p.x; xf[1] = p.y; xf[2] = p.z; xf[3] = p.w;
+    xf[4] = q.x; xf[5] = q.y; xf[6] = q.z; xf[7] = q.w;
+}
+
 // a[b][j] = SiLU(x_b . W_gate[:, j]), one warp per neuron row of wg_t, tokens
 // in groups of 8 (weights re-read from L2 per group; calibration only).
-__global__ void gate_act_kernel(const uint16_t *__restrict__ wg_t, int H, int N, const uint16_t *__restrict__ x,
+// X is uint16_t (bf16 activations) or float.
+template <typename X>
+__global__ void gate_act_kernel(const uint16_t *__restrict__ wg_t, int H, int N, const X *__restrict__ x,
                                 int B, float *__restrict__ a)
 {
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -134,7 +148,7 @@ __global__ void gate_act_kernel(const uint16_t *__restrict__ wg_t, int H, int N,
             for (int t = 0; t < 8; ++t) {
                 if (b0 + t < B) {
                     float xf[8];
-                    unpack8(reinterpret_cast<const uint4 *>(x + (size_t)(b0 + t) * H)[v], xf);
+                    load_x8(x + (size_t)(b0 + t) * H, v, xf);
 #pragma unroll
                     for (int e = 0; e < 8; ++e) acc[t] = fmaf(w[e], xf[e], acc[t]);
                 }
@@ -231,7 +245,15 @@ cudaError_t launch_gate_act(const sats_layer *layer, const uint16_t *x, int B, f
 {
     const int threads = 256;
     const int blocks = (layer->N * 32 + threads - 1) / threads;
-    gate_act_kernel<<<blocks, threads, 0, stream>>>(layer->wg_t, layer->H, layer->N, x, B, a);
+    gate_act_kernel<uint16_t><<<blocks, threads, 0, stream>>>(layer->wg_t, layer->H, layer->N, x, B, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gate_act_f32(const sats_layer *layer, const float *x, int B, float *a, cudaStream_t stream)
+{
+    const int threads = 256;
+    const int blocks = (layer->N * 32 + threads - 1) / threads;
+    gate_act_kernel<float><<<blocks, threads, 0, stream>>>(layer->wg_t, layer->H, layer->N, x, B, a);
     return cudaGetLastError();
 }
 

@@ -101,6 +101,13 @@ cudaError_t launch_route(const int32_t *ids, int B, const uint8_t *lut, int V, i
                          int32_t *n_dense, uint8_t *flags, int32_t *status, cudaStream_t stream);
 cudaError_t launch_gate_act(const sats_layer *layer, const uint16_t *x, int B, float *a,
                             cudaStream_t stream);
+cudaError_t launch_gate_act_f32(const sats_layer *layer, const float *x, int B, float *a, cudaStream_t stream);
+
+// One block over B tokens (fused kernel or tensor cores), as the C ABI calls run it
+// (api.cu).  ws: a workspace of ws_layout(H, N, B).total bytes with zeroed control words.
+sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B, const float *t_l,
+                      const float *norm_w, float eps, const uint8_t *dense_flags, int out_mode, float *out,
+                      int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws, cudaStream_t stream);
 size_t select_ws_bytes();
 cudaError_t launch_select(const float *a, int64_t n, int64_t m, void *ws, float *t_dev,
                           cudaStream_t stream);

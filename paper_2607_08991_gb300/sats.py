@@ -60,6 +60,13 @@ def lib() -> ctypes.CDLL:
             "sats_gate_act": (I, [P, P, I, P, P, Z, P]),
             "sats_select_workspace_bytes": (Z, []),
             "sats_percentile_threshold": (I, [P, I64, D, ctypes.POINTER(F), P, Z, P]),
+            "sats_rmsnorm": (I, [P, I, I, P, F, P, P]),
+            "sats_gate_act_f32": (I, [P, P, I, P, P]),
+            "sats_layer_err_workspace_bytes": (Z, [I, I, I, I]),
+            "sats_layer_err": (I, [P, P, I, P, I, F, P, P, P, Z, P]),
+            "sats_sats_select": (I, [P, P, P, I, I, D, I, D, D, P, P, P]),
+            "sats_sats_workspace_bytes": (Z, [I, I, I, I, I, I]),
+            "sats_sats_calibrate": (I, [P, P, I, F, P, I, D, I, I, I, F, P, P, P, P, P, P, P, Z, P]),
             "sats_get_error": (I, [P, Z, P]),
             "sats_get_status_word": (I, [P, P]),
         }
@@ -76,7 +83,9 @@ def exported_symbols() -> Sequence[str]:
     return ("sats_version", "sats_status_string", "sats_layer_create", "sats_layer_destroy", "sats_layer_shape",
             "sats_workspace_bytes", "sats_workspace_init", "sats_sparse_mlp", "sats_sparse_mlp_f32",
             "sats_sparse_mlp_fixed_scratch", "sats_uses_tensor_cores", "sats_last_cuda_error", "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
-            "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_get_error", "sats_get_status_word")
+            "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_rmsnorm", "sats_gate_act_f32",
+            "sats_layer_err_workspace_bytes", "sats_layer_err", "sats_sats_select", "sats_sats_workspace_bytes",
+            "sats_sats_calibrate", "sats_get_error", "sats_get_status_word")
 
 
 def status_string(s: int) -> str:
@@ -231,6 +240,76 @@ def percentile_threshold(a: torch.Tensor, k: float, sel_ws: torch.Tensor,
                                            _ptr(sel_ws, "sel_ws"), sel_ws.numel() * sel_ws.element_size(),
                                            _stream(stream)), "sats_percentile_threshold")
     return float(out.value)
+
+
+def rmsnorm(x: torch.Tensor, w: torch.Tensor, eps: float, out: torch.Tensor,
+            stream: Optional[torch.cuda.Stream] = None):
+    B, H = x.shape
+    _check(lib().sats_rmsnorm(_ptr(x, "x", 4), B, H, _ptr(w, "w", 4), float(eps), _ptr(out, "out", 4),
+                              _stream(stream)), "sats_rmsnorm")
+
+
+def gate_act_f32(layer: Layer, x: torch.Tensor, a: torch.Tensor, stream: Optional[torch.cuda.Stream] = None):
+    _check(lib().sats_gate_act_f32(layer.handle, _ptr(x, "x", 4), x.shape[0], _ptr(a, "a", 4), _stream(stream)),
+           "sats_gate_act_f32")
+
+
+def layer_err(layer: Layer, x: torch.Tensor, t: Sequence[float], eps: float = 1e-6,
+              stream: Optional[torch.cuda.Stream] = None):
+    """Eq. 6 at each candidate threshold on the calibration inputs x (fp32 [C][H]):
+    returns (err, sp) as lists of floats."""
+    C = x.shape[0]
+    K = len(t)
+    n = int(lib().sats_layer_err_workspace_bytes(layer.H, layer.N, C, K))
+    ws = torch.empty(n + 256, dtype=torch.uint8, device=x.device)
+    off = (-ws.data_ptr()) % 256
+    tt = (ctypes.c_float * max(K, 1))(*[float(v) for v in t])
+    err = (ctypes.c_double * max(K, 1))()
+    sp = (ctypes.c_double * max(K, 1))()
+    _check(lib().sats_layer_err(layer.handle, _ptr(x, "x", 4), C, tt, K, float(eps), err, sp,
+                                ctypes.c_void_p(ws.data_ptr() + off), n, _stream(stream)), "sats_layer_err")
+    return list(err)[:K], list(sp)[:K]
+
+
+def sats_select(t, err, sp, s_tar: float, guard: int = -1, guard_t: float = 0.0, guard_sp: float = 0.0):
+    """Eqs. 7-10 over a [L][K] candidate table (host function): returns (b*, T*(b*), S(b*))."""
+    L, K = len(t), len(t[0]) if len(t) else 0
+    flat = lambda m: (ctypes.c_double * max(L * K, 1))(*[float(v) for row in m for v in row])
+    b = ctypes.c_double()
+    S = ctypes.c_double()
+    tout = (ctypes.c_double * L)()
+    _check(lib().sats_sats_select(flat(t), flat(err), flat(sp), L, K, float(s_tar), int(guard), float(guard_t),
+                                  float(guard_sp), ctypes.byref(b), tout, ctypes.byref(S)), "sats_sats_select")
+    return b.value, list(tout), S.value
+
+
+def sats_calibrate(layers: Sequence[Layer], norm_w: Sequence[torch.Tensor], eps: float, x_cal: torch.Tensor,
+                   s_tar: float, K0: int = 20, K1: int = 8, guardrail: bool = True, err_eps: float = 1e-6,
+                   stream: Optional[torch.cuda.Stream] = None):
+    """SATS calibration of a stack (sats_sats_calibrate): returns dict(t, b, S, table=(t, err, sp))."""
+    L = len(layers)
+    C, H = x_cal.shape
+    N = layers[0].N
+    n = int(lib().sats_sats_workspace_bytes(H, N, C, L, K0, K1))
+    if n == 0:
+        raise ValueError("unsupported calibration shape")
+    ws = torch.empty(n + 256, dtype=torch.uint8, device=x_cal.device)
+    off = (-ws.data_ptr()) % 256
+    hs = (ctypes.c_void_p * L)(*[l.handle.value for l in layers])
+    nws = (ctypes.c_void_p * L)(*[_ptr(w, "norm_w", 4).value for w in norm_w])
+    tout = (ctypes.c_float * L)()
+    b = ctypes.c_double()
+    S = ctypes.c_double()
+    Kt = K0 - 1 + K1
+    tt = (ctypes.c_double * (L * Kt))()
+    te = (ctypes.c_double * (L * Kt))()
+    ts = (ctypes.c_double * (L * Kt))()
+    _check(lib().sats_sats_calibrate(hs, nws, L, float(eps), _ptr(x_cal, "x_cal", 4), C, float(s_tar), K0, K1,
+                                     1 if guardrail else 0, float(err_eps), tout, ctypes.byref(b), ctypes.byref(S),
+                                     tt, te, ts, ctypes.c_void_p(ws.data_ptr() + off), n, _stream(stream)),
+           "sats_sats_calibrate")
+    rows = lambda arr: [list(arr[l * Kt:(l + 1) * Kt]) for l in range(L)]
+    return dict(t=list(tout), b=b.value, S=S.value, table=(rows(tt), rows(te), rows(ts)))
 
 
 def get_error(ws: Workspace, stream: Optional[torch.cuda.Stream] = None) -> int:
