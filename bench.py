@@ -623,6 +623,31 @@ def run_workload(args):
             clk = clocks.stop()
             out.update({"metric": "us per prefill call (one routed block)", "value": res["0.6@2048"]["us_per_call"],
                         "unit": "us/call", "per_case": res, "clocks": clk})
+        elif wl == "sats_calibration_llama_32x4096x14336":
+            H, N, L, C = spec["H"], spec["N"], spec["L"], spec["calib"]
+            layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l)) for l in range(L)]
+            nws = [torch.from_numpy(inputs.norm_weight(H, layer=l)).to(dev) for l in range(L)]
+            xc = torch.from_numpy(inputs.activations_f32(C, H, seed=inputs.SEED_CALIB)).to(dev)
+            torch.cuda.synchronize()
+            # one Eq. 6 evaluation for its cost per candidate
+            n0 = torch.empty_like(xc)
+            sats.rmsnorm(xc, nws[0], spec["eps"], n0, stream=stream)
+            sats.layer_err(layers[0], n0, [0.1], stream=stream)
+            t0 = time.perf_counter()
+            sats.layer_err(layers[0], n0, [0.05 * k for k in range(1, 9)], stream=stream)
+            per_cand = (time.perf_counter() - t0) / 8
+            clocks.start()
+            t0 = time.perf_counter()
+            r = sats.sats_calibrate(layers, nws, spec["eps"], xc, spec["target"], K0=spec["K0"], K1=spec["K1"],
+                                    guardrail=True, stream=stream)
+            el = time.perf_counter() - t0
+            clk = clocks.stop()
+            out.update({"metric": "seconds for the SATS calibration of the %d-block stack" % L, "value": el,
+                        "unit": "s", "calibration_vectors": C, "coarse_candidates": spec["K0"] - 1,
+                        "fine_candidates": spec["K1"], "eq6_evaluations": L * (spec["K0"] - 1 + spec["K1"]) + 1,
+                        "seconds_per_eq6_candidate_one_block": per_cand, "target_sparsity": spec["target"],
+                        "realised_S": r["S"], "budget": r["b"], "thresholds": [round(v, 5) for v in r["t"]],
+                        "clocks": clk})
         else:
             raise SystemExit("unknown workload " + wl)
     print(json.dumps(out))
