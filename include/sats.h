@@ -306,6 +306,33 @@ SATS_API sats_status sats_sats_calibrate(const sats_layer *const *layers, const 
                                          size_t ws_bytes, void *stream);
 
 /*
+ * Routing calibration (Sec. 3.2).
+ *
+ * sats_token_scores -- Eqs. 11-12: for n corpus occurrences (ids: device
+ *   int32 [n]; l_base, l_sparse: device fp32 [n], the next-token losses of
+ *   the base and sparse paths), d_i = max(0, l_sparse_i - l_base_i) and
+ *   score[v] = mean of d_i over the occurrences of v (device fp32 [V]); a
+ *   token that never occurs gets +inf (it keeps the base path).  An id
+ *   outside [0, V) returns SATS_EDEVICE.  ws: sats_route_calib_workspace_bytes(V)
+ *   bytes, 256-byte aligned.  Synchronises `stream`.
+ *
+ * sats_route_calibrate -- Eq. 14: tau* = argmin_tau |R(tau) - r_tar|, where
+ *   R(tau) is the fraction of the m held-out occurrences (heldout_ids: device
+ *   int32 [m]) whose score is < tau (routed to the sparse path, Eq. 13); the
+ *   candidates are 0, every score of a token occurring in the held-out split,
+ *   and +inf, and a tie goes to the smaller tau.  Writes tau* and R(tau*)
+ *   (host), and, if lut is given, the routing table lut[v] = score[v] >= tau*
+ *   (device uint8 [V]; 1 = base path), as sats_route and sats_mlp_stack take
+ *   it.  Synchronises `stream`.
+ */
+SATS_API size_t sats_route_calib_workspace_bytes(int V);
+SATS_API sats_status sats_token_scores(const int32_t *ids, const float *l_base, const float *l_sparse, int64_t n,
+                                       int V, float *score, void *ws, size_t ws_bytes, void *stream);
+SATS_API sats_status sats_route_calibrate(const float *score, int V, const int32_t *heldout_ids, int64_t m,
+                                          double r_tar, float *tau_out, double *R_out, uint8_t *lut, void *ws,
+                                          size_t ws_bytes, void *stream);
+
+/*
  * sats_get_error -- synchronises `stream`, reads the status word in the
  * workspace, clears it, and returns SATS_OK, SATS_EDEVICE (bad token id) or
  * SATS_ETIMEOUT (a device wait gave up).

@@ -3,9 +3,11 @@
 This package is TEST INFRASTRUCTURE.  Only ``tests/``, ``__graft_entry__.smoke()``
 and the ``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import
 it.  It shares no code with the CUDA library in ``paper_2607_08991_gb300``:
-the arithmetic lives in ``sats_oracle.c`` (plain C, IEEE double), compiled
-with gcc into ``liboracle.so`` and called through ctypes.  This module only
-marshals numpy arrays.
+the MLP arithmetic (Sec. 2, Eqs. 1-5), Eq. 3, routing (Eq. 13), the stack,
+Eq. 6 and Eqs. 7-10 live in ``sats_oracle.c`` (plain C, IEEE double),
+compiled with gcc into ``liboracle.so`` and called through ctypes; the
+routing calibration (Sec. 3.2, Eqs. 11-14) and the order of the SATS
+coarse-to-fine steps are written out here in numpy (float64).
 
 Paper: "Sensitivity-Aware Thresholding and Token Routing for Activation
 Sparsification in Large Language Models" (arXiv 2607.08991).  Each wrapper
@@ -317,3 +319,44 @@ def sats_calibrate(x_cal, Wg: Sequence, Wu: Sequence, Wd: Sequence, norm_w: Sequ
     s_all = np.concatenate([sp0, sp1], axis=1)
     b, t, S = sats_select(t_all, e_all, s_all, s_tar, guard, g_t, g_sp)
     return dict(t=t, b=b, S=S, coarse=(cand, err0, sp0), fine=(t_all, e_all, s_all), guard=(g_t, g_sp))
+
+
+# ---------------------------------------------------------------- routing calibration (Sec. 3.2)
+
+def token_scores(ids, l_base, l_sparse, V: int) -> np.ndarray:
+    """Sec. 3.2, Eqs. 11-12: d_i = max(0, l_sparse_i - l_base_i) for every corpus occurrence i,
+    and s(x) = the mean of d_i over I_x = {i : x_i = x}.  A token with no occurrence has no
+    estimate; it gets +inf (the base path under Eq. 13 for every tau).  Raises on an id outside [0, V)."""
+    ids = np.asarray(ids, dtype=np.int64)
+    if ids.size and (ids.min() < 0 or ids.max() >= V):
+        raise ValueError("token id outside the vocabulary")
+    d = np.maximum(0.0, np.asarray(l_sparse, np.float64) - np.asarray(l_base, np.float64))   # Eq. 11
+    total = np.bincount(ids, weights=d, minlength=V)
+    count = np.bincount(ids, minlength=V)
+    s = np.full(V, np.inf)
+    seen = count > 0
+    s[seen] = total[seen] / count[seen]                                                      # Eq. 12
+    return s
+
+
+def routed_fraction(score, heldout_ids, tau) -> float:
+    """R(tau): the fraction of held-out occurrences routed to the sparse path, score < tau (Eq. 13)."""
+    s = np.asarray(score, np.float64)[np.asarray(heldout_ids, np.int64)]
+    return float(np.mean(s < tau)) if s.size else 0.0
+
+
+def route_threshold(score, heldout_ids, r_tar: float):
+    """Sec. 3.2, Eq. 14: tau* = argmin_tau |R(tau) - r_tar| over the candidates 0, every score of a
+    token occurring in the held-out split, and +inf (R only changes at those values); a tie goes to
+    the smaller tau.  Returns (tau*, R(tau*))."""
+    s = np.sort(np.asarray(score, np.float64)[np.asarray(heldout_ids, np.int64)])
+    cands = np.unique(np.concatenate([[0.0], s[np.isfinite(s)], [np.inf]]))
+    R = np.searchsorted(s, cands, side="left") / max(s.size, 1)
+    gaps = np.abs(R - r_tar)
+    k = int(np.argmin(gaps))          # first minimum: the smallest tau among ties
+    return float(cands[k]), float(R[k])
+
+
+def route_lut(score, tau: float) -> np.ndarray:
+    """Eq. 13 as a table: 1 (base path) where score >= tau, 0 (sparse path) where score < tau."""
+    return (np.asarray(score, np.float64) >= tau).astype(np.uint8)

@@ -400,3 +400,177 @@ sats_status sats_sats_calibrate(const sats_layer *const *layers, const float *co
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------- routing calibration (Sec. 3.2)
+namespace sats {
+namespace {
+
+// Eqs. 11-12, the sums: for every occurrence, d = max(0, l_sparse - l_base) into the token's total.
+__global__ void score_accum_kernel(const int32_t *__restrict__ ids, const float *__restrict__ lb,
+                                   const float *__restrict__ ls, int64_t n, int V, double *__restrict__ total,
+                                   unsigned *__restrict__ count, int32_t *__restrict__ status)
+{
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const int id = ids[i];
+        if (id < 0 || id >= V) {
+            atomicOr(status, kStatusBadToken);
+            continue;
+        }
+        atomicAdd(total + id, (double)fmaxf(0.0f, ls[i] - lb[i]));
+        atomicAdd(count + id, 1u);
+    }
+}
+
+// Eq. 12, the means; +inf for a token that never occurs (it keeps the base path).
+__global__ void score_final_kernel(const double *__restrict__ total, const unsigned *__restrict__ count, int V,
+                                   float *__restrict__ score)
+{
+    const int v = blockIdx.x * blockDim.x + threadIdx.x;
+    if (v < V) score[v] = count[v] ? (float)(total[v] / count[v]) : INFINITY;
+}
+
+__global__ void freq_kernel(const int32_t *__restrict__ ids, int64_t m, int V, unsigned *__restrict__ freq,
+                            int32_t *__restrict__ status)
+{
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < m; i += (int64_t)gridDim.x * blockDim.x) {
+        const int id = ids[i];
+        if (id < 0 || id >= V) {
+            atomicOr(status, kStatusBadToken);
+            continue;
+        }
+        atomicAdd(freq + id, 1u);
+    }
+}
+
+// Eq. 13 as a table: 1 (base path) where score >= tau, 0 (sparse path) where score < tau.
+__global__ void lut_kernel(const float *__restrict__ score, int V, float tau, uint8_t *__restrict__ lut)
+{
+    const int v = blockIdx.x * blockDim.x + threadIdx.x;
+    if (v < V) lut[v] = score[v] < tau ? 0 : 1;
+}
+
+struct ScoreLayout {
+    size_t status, total, count, total_bytes;
+};
+
+ScoreLayout score_layout(int V)
+{
+    ScoreLayout S{};
+    size_t off = 0;
+    S.status = off;
+    off += 256;
+    S.total = off;
+    off += al256((size_t)V * sizeof(double));
+    S.count = off;
+    off += al256((size_t)V * sizeof(unsigned));
+    S.total_bytes = off;
+    return S;
+}
+
+sats_status read_status_word(int32_t *word, cudaStream_t st)
+{
+    int32_t v = 0;
+    cudaError_t e = cudaMemcpyAsync(&v, word, sizeof v, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "status read");
+    return (v & kStatusBadToken) ? SATS_EDEVICE : SATS_OK;
+}
+
+int grid_for(int64_t n)
+{
+    const int64_t g = (n + 255) / 256;
+    return (int)(g < 4096 ? (g > 0 ? g : 1) : 4096);
+}
+
+}  // namespace
+}  // namespace sats
+
+extern "C" {
+
+size_t sats_route_calib_workspace_bytes(int V)
+{
+    if (V < 1) return 0;
+    return score_layout(V).total_bytes;
+}
+
+sats_status sats_token_scores(const int32_t *ids, const float *l_base, const float *l_sparse, int64_t n, int V,
+                              float *score, void *ws, size_t ws_bytes, void *stream)
+{
+    if (V < 1 || n < 0 || !score || !ws || (n > 0 && (!ids || !l_base || !l_sparse))) return SATS_EINVAL;
+    const ScoreLayout S = score_layout(V);
+    if (ws_bytes < S.total_bytes || (reinterpret_cast<uintptr_t>(ws) & 255u)) return ws_bytes < S.total_bytes ? SATS_ENOSPACE : SATS_EINVAL;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    char *base = static_cast<char *>(ws);
+    int32_t *status = reinterpret_cast<int32_t *>(base + S.status);
+    double *total = reinterpret_cast<double *>(base + S.total);
+    unsigned *count = reinterpret_cast<unsigned *>(base + S.count);
+    cudaError_t e = cudaMemsetAsync(ws, 0, S.total_bytes, st);
+    if (e != cudaSuccess) return cuda_fail(e, "score workspace clear");
+    if (n > 0) score_accum_kernel<<<grid_for(n), 256, 0, st>>>(ids, l_base, l_sparse, n, V, total, count, status);
+    score_final_kernel<<<(V + 255) / 256, 256, 0, st>>>(total, count, V, score);
+    if ((e = cudaGetLastError()) != cudaSuccess) return cuda_fail(e, "score kernel launch");
+    return read_status_word(status, st);
+}
+
+sats_status sats_route_calibrate(const float *score, int V, const int32_t *heldout_ids, int64_t m, double r_tar,
+                                 float *tau_out, double *R_out, uint8_t *lut, void *ws, size_t ws_bytes, void *stream)
+{
+    if (V < 1 || m < 0 || !score || !tau_out || !ws || std::isnan(r_tar) || (m > 0 && !heldout_ids)) return SATS_EINVAL;
+    const ScoreLayout S = score_layout(V);
+    if (ws_bytes < S.total_bytes || (reinterpret_cast<uintptr_t>(ws) & 255u)) return ws_bytes < S.total_bytes ? SATS_ENOSPACE : SATS_EINVAL;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    char *base = static_cast<char *>(ws);
+    int32_t *status = reinterpret_cast<int32_t *>(base + S.status);
+    unsigned *freq = reinterpret_cast<unsigned *>(base + S.count);
+    cudaError_t e = cudaMemsetAsync(status, 0, 256, st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(freq, 0, (size_t)V * sizeof(unsigned), st);
+    if (e != cudaSuccess) return cuda_fail(e, "held-out count clear");
+    if (m > 0) freq_kernel<<<grid_for(m), 256, 0, st>>>(heldout_ids, m, V, freq, status);
+    if ((e = cudaGetLastError()) != cudaSuccess) return cuda_fail(e, "held-out count kernel launch");
+    sats_status s = read_status_word(status, st);
+    if (s != SATS_OK) return s;
+    // Eq. 14 on the host over the V scores: R(tau) = (held-out occurrences with score < tau) / m
+    std::vector<float> sc((size_t)V);
+    std::vector<unsigned> fr((size_t)V);
+    e = cudaMemcpyAsync(sc.data(), score, sc.size() * sizeof(float), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(fr.data(), freq, fr.size() * sizeof(unsigned), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "score read-back");
+    std::vector<std::pair<float, unsigned>> occ;
+    for (int v = 0; v < V; ++v)
+        if (fr[(size_t)v]) occ.emplace_back(sc[(size_t)v], fr[(size_t)v]);
+    std::sort(occ.begin(), occ.end());
+    // candidates in increasing order: 0, each distinct finite held-out score, +inf; below(tau) is the
+    // number of held-out occurrences whose score is < tau
+    const double M = m > 0 ? (double)m : 1.0;
+    double best_gap = INFINITY, best_R = 0.0;
+    float best_tau = 0.0f;
+    auto consider = [&](float tau, uint64_t below) {
+        const double R = (double)below / M;
+        const double gap = std::fabs(R - r_tar);
+        if (gap < best_gap) {
+            best_gap = gap;
+            best_tau = tau;
+            best_R = R;
+        }
+    };
+    uint64_t below = 0;
+    size_t i = 0;
+    while (i < occ.size() && occ[i].first < 0.0f) below += occ[i++].second;   // (scores are >= 0)
+    consider(0.0f, below);
+    while (i < occ.size() && std::isfinite(occ[i].first)) {
+        const float v = occ[i].first;
+        if (v > 0.0f) consider(v, below);   // R(v) counts the scores strictly below v
+        while (i < occ.size() && occ[i].first == v) below += occ[i++].second;
+    }
+    consider(INFINITY, below);
+    *tau_out = best_tau;
+    if (R_out) *R_out = best_R;
+    if (lut) {
+        lut_kernel<<<(V + 255) / 256, 256, 0, st>>>(score, V, best_tau, lut);
+        if ((e = cudaGetLastError()) != cudaSuccess) return cuda_fail(e, "table kernel launch");
+    }
+    return SATS_OK;
+}
+
+}  // extern "C"

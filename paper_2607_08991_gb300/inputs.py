@@ -145,6 +145,20 @@ def token_ids_zipf(B: int, V: int, s: float = 1.1, seed: int = SEED_IDS) -> np.n
     return np.minimum(np.searchsorted(cdf, u, side="right"), V - 1).astype(np.int32)
 
 
+def routing_corpus(n: int, V: int, seed: int = SEED_IDS + 100, s: float = 1.1):
+    """A synthetic stand-in for the routing calibration corpus of Sec. 3.2: n token
+    occurrences with Zipf(s) ids over V, a base-path loss l_base ~ N(3, 1), and a
+    sparse-path loss l_sparse = l_base + r(x) + N(0, 0.05), where r(v) ~ Exp(0.1) is a
+    per-token risk (so the excess damage depends on the token, as the method assumes).
+    Returns (ids int32 [n], l_base fp32 [n], l_sparse fp32 [n])."""
+    ids = token_ids_zipf(n, V, s=s, seed=seed)
+    g = _rng(seed, 1)
+    risk = g.exponential(0.1, size=V).astype(np.float32)
+    l_base = (3.0 + g.standard_normal(n)).astype(np.float32)
+    l_sparse = (l_base + risk[ids] + 0.05 * g.standard_normal(n)).astype(np.float32)
+    return ids, l_base, l_sparse
+
+
 def stack_sparsity_targets(L: int, lo: float, hi: float, seed: int = SEED_SHUFFLE) -> np.ndarray:
     """L evenly spaced targets in [lo, hi] (mean (lo+hi)/2), assigned to layers by a seeded shuffle."""
     base = lo + (hi - lo) * (np.arange(L) + 0.5) / L

@@ -67,6 +67,9 @@ def lib() -> ctypes.CDLL:
             "sats_sats_select": (I, [P, P, P, I, I, D, I, D, D, P, P, P]),
             "sats_sats_workspace_bytes": (Z, [I, I, I, I, I, I]),
             "sats_sats_calibrate": (I, [P, P, I, F, P, I, D, I, I, I, F, P, P, P, P, P, P, P, Z, P]),
+            "sats_route_calib_workspace_bytes": (Z, [I]),
+            "sats_token_scores": (I, [P, P, P, I64, I, P, P, Z, P]),
+            "sats_route_calibrate": (I, [P, I, P, I64, D, ctypes.POINTER(F), ctypes.POINTER(D), P, P, Z, P]),
             "sats_get_error": (I, [P, Z, P]),
             "sats_get_status_word": (I, [P, P]),
         }
@@ -85,7 +88,8 @@ def exported_symbols() -> Sequence[str]:
             "sats_sparse_mlp_fixed_scratch", "sats_uses_tensor_cores", "sats_last_cuda_error", "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
             "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_rmsnorm", "sats_gate_act_f32",
             "sats_layer_err_workspace_bytes", "sats_layer_err", "sats_sats_select", "sats_sats_workspace_bytes",
-            "sats_sats_calibrate", "sats_get_error", "sats_get_status_word")
+            "sats_sats_calibrate", "sats_route_calib_workspace_bytes", "sats_token_scores", "sats_route_calibrate",
+            "sats_get_error", "sats_get_status_word")
 
 
 def status_string(s: int) -> str:
@@ -310,6 +314,37 @@ def sats_calibrate(layers: Sequence[Layer], norm_w: Sequence[torch.Tensor], eps:
            "sats_sats_calibrate")
     rows = lambda arr: [list(arr[l * Kt:(l + 1) * Kt]) for l in range(L)]
     return dict(t=list(tout), b=b.value, S=S.value, table=(rows(tt), rows(te), rows(ts)))
+
+
+def _calib_ws(V: int, device):
+    n = int(lib().sats_route_calib_workspace_bytes(V))
+    ws = torch.empty(n + 256, dtype=torch.uint8, device=device)
+    return ws, ctypes.c_void_p(ws.data_ptr() + (-ws.data_ptr()) % 256), n
+
+
+def token_scores(ids: torch.Tensor, l_base: torch.Tensor, l_sparse: torch.Tensor, V: int,
+                 stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    """Eqs. 11-12: per-token mean excess damage (device fp32 [V]; +inf for unseen tokens)."""
+    score = torch.empty(V, dtype=torch.float32, device=ids.device)
+    keep, ws, n = _calib_ws(V, ids.device)
+    _check(lib().sats_token_scores(_ptr(ids, "ids", 4), _ptr(l_base, "l_base", 4), _ptr(l_sparse, "l_sparse", 4),
+                                   ids.numel(), V, _ptr(score, "score", 4), ws, n, _stream(stream)),
+           "sats_token_scores")
+    return score
+
+
+def route_calibrate(score: torch.Tensor, heldout_ids: torch.Tensor, r_tar: float,
+                    stream: Optional[torch.cuda.Stream] = None):
+    """Eq. 14: returns (tau*, R(tau*), lut) with lut the device uint8 routing table (1 = base path)."""
+    V = score.numel()
+    lut = torch.empty(V, dtype=torch.uint8, device=score.device)
+    keep, ws, n = _calib_ws(V, score.device)
+    tau = ctypes.c_float()
+    R = ctypes.c_double()
+    _check(lib().sats_route_calibrate(_ptr(score, "score", 4), V, _ptr(heldout_ids, "heldout_ids", 4),
+                                      heldout_ids.numel(), float(r_tar), ctypes.byref(tau), ctypes.byref(R),
+                                      _ptr(lut, "lut", 1), ws, n, _stream(stream)), "sats_route_calibrate")
+    return tau.value, R.value, lut
 
 
 def get_error(ws: Workspace, stream: Optional[torch.cuda.Stream] = None) -> int:
