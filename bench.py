@@ -648,6 +648,28 @@ def run_workload(args):
                         "seconds_per_eq6_candidate_one_block": per_cand, "target_sparsity": spec["target"],
                         "realised_S": r["S"], "budget": r["b"], "thresholds": [round(v, 5) for v in r["t"]],
                         "clocks": clk})
+        elif wl == "route_calibration_qwen_v151936":
+            V = spec["V"]
+            ids, lb, ls = inputs.routing_corpus(spec["corpus"], V)
+            held = inputs.token_ids_zipf(spec["heldout"], V, seed=inputs.SEED_IDS + 200)
+            ids_d, lb_d, ls_d = (torch.from_numpy(a).to(dev) for a in (ids, lb, ls))
+            held_d = torch.from_numpy(held).to(dev)
+            sats.token_scores(ids_d, lb_d, ls_d, V, stream=stream)      # warm-up
+            clocks.start()
+            t0 = time.perf_counter()
+            score = sats.token_scores(ids_d, lb_d, ls_d, V, stream=stream)
+            t_scores = time.perf_counter() - t0
+            res = {}
+            for r_tar in spec["targets"]:
+                t0 = time.perf_counter()
+                tau, R, lut = sats.route_calibrate(score, held_d, r_tar, stream=stream)
+                res[str(r_tar)] = {"tau": tau, "R": R, "seconds": time.perf_counter() - t0,
+                                   "dense_fraction_of_vocab": float(lut.float().mean())}
+            clk = clocks.stop()
+            out.update({"metric": "seconds for the token scores of the routing corpus (Eqs. 11-12)",
+                        "value": t_scores, "unit": "s", "corpus_occurrences": spec["corpus"],
+                        "heldout_occurrences": spec["heldout"], "occurrences_per_s": spec["corpus"] / t_scores,
+                        "per_target": res, "clocks": clk})
         else:
             raise SystemExit("unknown workload " + wl)
     print(json.dumps(out))

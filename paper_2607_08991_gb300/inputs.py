@@ -175,6 +175,9 @@ WORKLOADS: Dict[str, dict] = {
                                            p_dense=0.3, sparsity=0.5, eps=1e-6),
     "llama_layer_prefill_routed": dict(H=LLAMA_H, N=LLAMA_N, V=LLAMA_V, batches=[256, 2048], zipf_s=1.1,
                                        p_dense=0.2, sparsity=[0.4, 0.6, 0.8, 0.9]),
+    # routing calibration (Sec. 3.2) over the Qwen3-8B-shaped vocabulary
+    "route_calibration_qwen_v151936": dict(V=QWEN_V, corpus=4_000_000, heldout=1_000_000,
+                                           targets=[0.25, 0.5, 0.75]),
     # SATS calibration (Sec. 3.1) of the 32-block Llama-shaped stack
     "sats_calibration_llama_32x4096x14336": dict(H=LLAMA_H, N=LLAMA_N, L=LLAMA_L, calib=64, K0=20, K1=8,
                                                   target=0.5, eps=1e-5),
