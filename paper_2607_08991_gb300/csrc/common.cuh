@@ -112,6 +112,13 @@ __device__ __forceinline__ void bulk_load_shared(void *dst, const void *src, uin
                  : "memory");
 }
 
+// Starts bringing `bytes` (a multiple of 16) at a 16-byte aligned global
+// address into L2; no completion to wait for.
+__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 // Barrier among `count` threads (a multiple of 32) on hardware barrier `id`.
 __device__ __forceinline__ void named_barrier(int id, int count)
 {

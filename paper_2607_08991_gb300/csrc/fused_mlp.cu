@@ -63,6 +63,7 @@ constexpr int kUdSlotBytes = kUdRingBytes / kUdSlots;      // 32 KB
 constexpr int kBufs = 4;                                   // list buffers (gate lookahead, chunks)
 constexpr int kPoolChunksPerCta = 3;                       // chunks of each range left to the shared pool
 constexpr int kMaxUdRows = 8;                              // W_ud rows per stage (small H)
+constexpr uint32_t kL2PrefetchBytes = 128 * 1024;          // gate rows brought into L2 before the previous call ends
 
 enum StageKind { kRows = 0, kEnd = 1 };
 
@@ -231,6 +232,23 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
     const int own = max(0, (nb1 - nb0 + kChunk - 1) / kChunk - kPoolChunksPerCta);
     int next_k = -1;   // a claimed, not yet used pool chunk
     bool waited = false;   // the workspace's pool counter is used only after the previous grid ended
+    {
+        // The weights do not depend on the previous call: while it finishes (its tail
+        // leaves HBM mostly idle), start moving the rows this CTA streams first, past
+        // what the gate ring holds, into L2.
+        const size_t first = (size_t)kGateStages * rows_per_stage;
+        const size_t own_rows = (size_t)min(nb1 - nb0, own * kChunk);
+        if (own_rows > first) {
+            const char *src = reinterpret_cast<const char *>(p.wg_t + (size_t)(nb0 + first) * H);
+            size_t left = min((size_t)kL2PrefetchBytes, (own_rows - first) * row_bytes);
+            for (size_t off = 0; left > 0;) {
+                const uint32_t nbytes = (uint32_t)min(left, (size_t)65536);
+                bulk_prefetch_l2(src + off, nbytes);
+                off += nbytes;
+                left -= nbytes;
+            }
+        }
+    }
     if (own == 0) {
         grid_dependency_wait();
         waited = true;
