@@ -50,7 +50,7 @@ typedef enum {
     SATS_EINVAL = 1,    /* null pointer, negative size, NaN or negative threshold, bad k */
     SATS_ESHAPE = 2,    /* H not a multiple of 8, H or N out of range */
     SATS_ECUDA = 3,     /* a CUDA runtime call failed (launch, copy, allocation) */
-    SATS_EDEVICE = 4,   /* a kernel reported bad input (token id outside [0, V)) */
+    SATS_EDEVICE = 4,   /* a kernel reported bad input (token id outside [0, V)) or an internal fault */
     SATS_ETIMEOUT = 5,  /* a bounded device-side wait gave up */
     SATS_ENOSPACE = 6   /* workspace smaller than sats_workspace_bytes() */
 } sats_status;
@@ -88,9 +88,9 @@ SATS_API sats_status sats_layer_shape(const sats_layer *layer, int *H, int *N);
 /*
  * Workspace.  Every compute call takes a device workspace `ws` of at least
  * sats_workspace_bytes(H, N, B) bytes (B = the largest batch the caller will
- * pass).  It holds scheduling counters, the device status word, one keep
- * byte per neuron and token (for the index outputs) and the routing scratch of
- * sats_mlp_stack: N * 4 bytes plus B * 5 plus 1 KB.  A batch that runs on the
+ * pass).  It holds scheduling counters, the device status word, one 64-bit
+ * word per 8 neurons (kept counts and prefixes for the index outputs) and the
+ * routing scratch of sats_mlp_stack: N bytes plus B * 5 plus 1 KB.  A batch that runs on the
  * tensor cores (sats_uses_tensor_cores) also needs, per token, bf16 copies of
  * its activations and of h (two parts each) plus one keep byte per neuron:
  * about B * (4 H + 5 N) bytes more.  It must be
@@ -138,12 +138,12 @@ SATS_API sats_status sats_sparse_mlp(const sats_layer *layer, const void *x, int
  * device allocator at all.
  *
  * Arguments, results and errors are those of sats_sparse_mlp.  Instead of a
- * workspace the call uses one 1 MiB array in the library's device memory; every
- * GPU that loads the library holds this array until the process exits.  A
- * shape whose workspace (sats_workspace_bytes(H, N, B)) exceeds 1 MiB is
- * rejected with SATS_ENOSPACE; with four keep bytes per neuron that admits
- * N up to about 260,000.  The call allocates nothing: before its kernel it
- * clears the array's control words with cudaMemsetAsync on `stream`.
+ * workspace the call uses one 256 KiB array in the library's device memory;
+ * every GPU that loads the library holds this array until the process exits.
+ * A shape whose workspace (sats_workspace_bytes(H, N, B)) exceeds 256 KiB is
+ * rejected with SATS_ENOSPACE; with one 64-bit word per 8 neurons that admits
+ * N up to about 259,000 for B <= 2.  The call allocates nothing: before its
+ * kernel it clears the array's control words with cudaMemsetAsync on `stream`.
  *
  * The first call on each device looks up the array's device address
  * (cudaGetSymbolAddress); make that first call before any stream capture.

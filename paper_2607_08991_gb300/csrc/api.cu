@@ -22,8 +22,8 @@ WsLayout ws_layout(int H, int N, int B)
     size_t off = 0;
     L.ctl = off;
     off += align256(kCtlInts * sizeof(int));
-    L.keep = off;   // one keep byte per neuron and token of a pass, rows padded to 16 bytes
-    off += align256((size_t)kMaxTokensPerPass * (((size_t)N + 15) & ~(size_t)15));
+    L.flags = off;   // one 64-bit word per chunk of kChunk neurons, then one per CTA of the fused grid
+    off += align256(((size_t)nchunks_of(N) + kMaxGrid) * sizeof(uint64_t));
     L.route_perm = off;
     off += align256((size_t)(B > 0 ? B : 1) * sizeof(int32_t));
     L.route_flags = off;
@@ -35,6 +35,12 @@ WsLayout ws_layout(int H, int N, int B)
 }
 
 static bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+cudaError_t clear_fused_state(void *ws, int H, int N, int B, cudaStream_t stream)
+{
+    // the fused kernel clears the chunk flags itself; its counters must start at zero
+    return cudaMemsetAsync(ws, 0, ws_layout(H, N, B).flags, stream);
+}
 
 static thread_local cudaError_t g_last_cuda = cudaSuccess;
 static thread_local const char *g_last_where = nullptr;
@@ -89,7 +95,7 @@ sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B,
         p.out_mode = out_mode;
         p.out = out + (size_t)b0 * H;
         p.ctl = reinterpret_cast<int *>(base + L.ctl);
-        p.keep_tmp = reinterpret_cast<uint8_t *>(base + L.keep);
+        p.flags = reinterpret_cast<uint64_t *>(base + L.flags);
         p.active_idx = active_idx ? active_idx + (size_t)b0 * N : nullptr;
         p.active_cnt = active_cnt ? active_cnt + b0 : nullptr;
         p.keep_trace = keep_trace ? keep_trace + (size_t)b0 * N : nullptr;
@@ -126,7 +132,7 @@ static sats_status sparse_common(const sats_layer *layer, int x_mode, const void
 // device memory, present on every GPU that loads the library until the
 // process exits.  Host code cannot use the symbol itself as a device address;
 // the address is looked up per device with cudaGetSymbolAddress.
-constexpr size_t kFixedScratchBytes = (size_t)1 << 20;   // 1 MiB
+constexpr size_t kFixedScratchBytes = (size_t)1 << 18;   // 256 KiB
 static __device__ __align__(256) unsigned char g_fixed_scratch[kFixedScratchBytes];
 
 static std::mutex g_fixed_scratch_mu;
@@ -253,7 +259,7 @@ sats_status sats_sparse_mlp_fixed_scratch(const sats_layer *layer, const void *x
     if (!ws) return cuda_fail(cudaErrorInvalidSymbol, "fixed scratch lookup");
     // the array keeps the previous call's contents: the control words
     // (scheduling counters, status) must start at zero
-    const cudaError_t ez = cudaMemsetAsync(ws, 0, kCtlInts * sizeof(int), static_cast<cudaStream_t>(stream));
+    const cudaError_t ez = clear_fused_state(ws, layer->H, layer->N, B, static_cast<cudaStream_t>(stream));
     if (ez != cudaSuccess) return cuda_fail(ez, "fixed scratch clear");
     return sparse_common(layer, kXBf16, x, B, t_l, y, active_idx, active_cnt, ws, kFixedScratchBytes, stream);
 }
@@ -365,7 +371,7 @@ static sats_status read_status(int32_t *word, cudaStream_t st)
     if (e == cudaSuccess && v != 0) e = cudaMemset(word, 0, sizeof v);
     if (e != cudaSuccess) return cuda_fail(e, "status read");
     if (v & kStatusTimeout) return SATS_ETIMEOUT;
-    if (v & kStatusBadToken) return SATS_EDEVICE;
+    if (v & (kStatusBadToken | kStatusInternal)) return SATS_EDEVICE;
     return SATS_OK;
 }
 

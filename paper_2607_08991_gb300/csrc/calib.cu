@@ -173,7 +173,7 @@ sats_status sats_layer_err(const sats_layer *layer, const float *x, int C, const
     float *yd = reinterpret_cast<float *>(base + W.yd), *yk = reinterpret_cast<float *>(base + W.yk);
     int32_t *idx = reinterpret_cast<int32_t *>(base + W.idx), *cnt = reinterpret_cast<int32_t *>(base + W.cnt);
     double *acc = reinterpret_cast<double *>(base + W.acc);
-    cudaError_t e = cudaMemsetAsync(mlp, 0, kCtlInts * sizeof(int), st);
+    cudaError_t e = clear_fused_state(mlp, H, N, C, st);
     if (e == cudaSuccess) e = cudaMemsetAsync(acc, 0, (size_t)2 * K * sizeof(double), st);
     if (e != cudaSuccess) return cuda_fail(e, "layer error workspace clear");
     const float zero = 0.0f;
@@ -298,7 +298,7 @@ sats_status sats_sats_calibrate(const sats_layer *const *layers, const float *co
 
     // 1-2: the dense stack gives each block's MLP inputs; coarse candidates from |SiLU(n W_gate)|
     cudaError_t e = cudaMemcpyAsync(x, x_cal, (size_t)C * H * sizeof(float), cudaMemcpyDeviceToDevice, st);
-    if (e == cudaSuccess) e = cudaMemsetAsync(mlp, 0, kCtlInts * sizeof(int), st);
+    if (e == cudaSuccess) e = clear_fused_state(mlp, H, N, C, st);
     if (e != cudaSuccess) return cuda_fail(e, "calibration set-up");
     std::vector<double> tc((size_t)L * Kc), amax((size_t)L), errc((size_t)L * Kc), spc((size_t)L * Kc);
     double g_t = 0.0, g_sp = 0.0;

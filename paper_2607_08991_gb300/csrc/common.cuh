@@ -15,6 +15,7 @@ namespace sats {
 // Bits of the device status word (workspace control block or caller's word).
 constexpr int kStatusBadToken = 1;   // a token id outside [0, V)
 constexpr int kStatusTimeout = 2;    // a bounded wait gave up
+constexpr int kStatusInternal = 4;   // an index-list position out of range (a kernel defect; the store is skipped)
 
 // Upper bound of every device-side wait before it reports kStatusTimeout.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;   // 2 s
@@ -142,6 +143,20 @@ __device__ __forceinline__ int ld_acquire_gpu(const int *p)
     int v;
     asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
+}
+
+// Relaxed (no ordering) 64-bit accesses at GPU scope, for words that carry
+// their whole payload.
+__device__ __forceinline__ uint64_t ld_relaxed_gpu_u64(const uint64_t *p)
+{
+    uint64_t v;
+    asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void st_relaxed_gpu_u64(uint64_t *p, uint64_t v)
+{
+    asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
 __device__ __forceinline__ void st_release_gpu(int *p, int v)

@@ -10,23 +10,29 @@
 // contiguous bytes.  A neuron no token keeps costs no HBM traffic beyond its
 // gate row.
 //
-// One CTA per SM, 576 threads in four roles, two shared-memory rings fed by
+// One CTA per SM, 608 threads in five roles, two shared-memory rings fed by
 // cp.async.bulk copies that complete on per-stage mbarriers:
-//   * gate producer (one thread): walks the first part of the CTA's contiguous
-//     range of N / G neurons in chunks of 8, then claims chunks from a shared
-//     pool (the last few chunks of every CTA's range) until it is empty, so
-//     that faster SMs take more of the tail; a chunk is started only when one
-//     of four list buffers is free.  Streams gate rows into the gate ring
-//     (5 x 16 KB).
+//   * gate producer (one thread): works through chunks of 8 neurons: first the
+//     CTA's three fixed chunks (c, c + G, c + 2G, which it may stream before the
+//     previous call has finished), then chunks claimed in increasing order from
+//     one counter, so that faster SMs take more of them; a chunk is started only
+//     when one of four list buffers is free.  Streams gate rows into the gate
+//     ring (5 x 16 KB).
 //   * 8 gate warps: thread t owns the 16-byte vectors t, t + 256, ... of every
 //     gate row and keeps the matching activations in registers as float pairs;
 //     dot products use paired FP32 FMAs (fma.rn.f32x2), two rows at a time
 //     with a transposed warp reduction; per-warp partials go to the chunk's
 //     list buffer, then each warp arrives on the buffer's barrier.
 //   * list producer (one warp, lane = row): sums the partials of a chunk,
-//     applies SiLU (Eq. 2) and the mask (Eqs. 4-5) per token, writes the
-//     optional index outputs, frees the buffer, and streams the W_ud rows of
-//     the kept neurons into the W_ud ring (4 slots of 32 KB).
+//     applies SiLU (Eq. 2) and the mask (Eqs. 4-5) per token, publishes the
+//     chunk's kept counts, frees the buffer, and streams the W_ud rows of the
+//     kept neurons into the W_ud ring (4 slots of 32 KB).
+//   * index warp: turns each chunk's kept rows into its entries of the
+//     ascending index lists.  A chunk's place in the list is the number of
+//     neurons kept in all earlier chunks, found by a decoupled look-back over
+//     the chunks' flag words (each holds the chunk's own counts, then the
+//     inclusive prefix once known), so the lists are complete as soon as every
+//     chunk's gate work is done.
 //   * 8 up/down warps: thread t owns vectors t, t + 256, ... of the up and
 //     down halves of each W_ud row and keeps its y columns in registers.  The
 //     up dot products of a stage are reduced across these warps through a
@@ -36,9 +42,9 @@
 // other.  After its stream each CTA adds its y partial into the output with
 // vector reductions in L2 (red.global.add.v4.f32); a counter guarantees that
 // every CTA has read its activations (the residual stream, which the output
-// may alias) and zeroed its slice of y before any CTA adds.  When the
-// kept-index lists are requested, every chunk writes one keep byte per neuron
-// and token, and the last CTA to finish turns them into the ascending lists.
+// may alias), zeroed its slice of y and cleared its slice of the chunk flags
+// before any CTA adds or touches a flag.  The last CTA to finish resets the
+// counters.
 // Every wait is bounded in time; a wait that gives up sets the status word.
 #include <cmath>
 
@@ -54,16 +60,43 @@ constexpr int kGateThreads = kGateWarps * 32;        // 256
 constexpr int kUdThreads = kUdWarps * 32;            // 256
 constexpr int kGateProducerWarp = kGateWarps + kUdWarps;   // 16
 constexpr int kListWarp = kGateProducerWarp + 1;           // 17
-constexpr int kThreads = (kListWarp + 1) * 32;             // 576
+constexpr int kIndexWarp = kListWarp + 1;                  // 18
+constexpr int kThreads = (kIndexWarp + 1) * 32;            // 608
 constexpr int kGateStageBytes = 16384;
 constexpr int kGateStages = 5;
 constexpr int kUdRingBytes = 131072;
 constexpr int kUdSlots = 4;
 constexpr int kUdSlotBytes = kUdRingBytes / kUdSlots;      // 32 KB
 constexpr int kBufs = 4;                                   // list buffers (gate lookahead, chunks)
-constexpr int kPoolChunksPerCta = 3;                       // chunks of each range left to the shared pool
+constexpr int kStaticChunks = 3;                           // fixed chunks per CTA before the claimed ones
+constexpr int kPendingChunks = 16;                        // chunk words held back until every CTA has cleared its flags
 constexpr int kMaxUdRows = 8;                              // W_ud rows per stage (small H)
 constexpr uint32_t kL2PrefetchBytes = 128 * 1024;          // gate rows brought into L2 before the previous call ends
+
+// Index-list words (the flags region: nchunks chunk words, then one slice word
+// per CTA; CTA c's slice is chunks [c per, (c + 1) per), per = ceil(nchunks / G)).
+// Chunk word: [63:62] status (0: not yet published this call, kChunkKept:
+// published), [8b + 7:8b] the rows of the chunk kept for token b.  Slice word:
+// [63:62] status (0, kFlagAgg: the slice's own kept counts, kFlagInc: the kept
+// counts of slices 0..c), [61:31] token 1's count, [30:0] token 0's count.
+// Every CTA clears its chunk words and its slice word before it passes its
+// prologue, and the words are written and read only after every CTA has passed
+// it.  A word holds its whole payload, so the accesses are relaxed; a word only
+// moves from 0 to its final value (slice words through kFlagAgg), and every
+// writer of a slice's kFlagInc writes the same value (the prefix is unique).
+constexpr uint64_t kChunkKept = 1ull << 62;
+constexpr uint64_t kFlagAgg = 1ull << 62;
+constexpr uint64_t kFlagInc = 2ull << 62;
+constexpr uint64_t kFlagPayload = (1ull << 62) - 1ull;   // payloads add field by field (sums stay below 2^31)
+constexpr int kLookWords = kMaxGrid / 32;                 // slice words per lane: one look-back step covers the grid
+
+__device__ __forceinline__ uint64_t make_flag(uint64_t status, uint32_t v0, uint32_t v1)
+{
+    return status | ((uint64_t)(v1 & 0x7FFFFFFFu) << 31) | (uint64_t)(v0 & 0x7FFFFFFFu);
+}
+__device__ __forceinline__ uint32_t flag_value(uint64_t f, int b) { return (uint32_t)(f >> (31 * b)) & 0x7FFFFFFFu; }
+__device__ __forceinline__ uint32_t flag_state(uint64_t f) { return (uint32_t)(f >> 62); }
+__device__ __forceinline__ uint32_t chunk_rows(uint64_t f, int b) { return (uint32_t)(f >> (8 * b)) & 0xFFu; }
 
 enum StageKind { kRows = 0, kEnd = 1 };
 
@@ -93,9 +126,10 @@ struct Shared {
     int chunkq[kBufs];          // first neuron of the chunk in a buffer (-1: no more work)
     int chunkrows[kBufs];
     int gissued[kGateStages], uissued[kUdSlots];
-    float thr[BT];
+    float thr[BT];              // per-token threshold, written and read by the list producer
     float red[kGateWarps + kUdWarps][BT];
-    int warp_sums[kThreads / 32];
+    uint64_t pend_word[kPendingChunks];   // chunk words not yet published (list producer)
+    int pend_chunk[kPendingChunks];
     int abort;
 };
 
@@ -222,78 +256,63 @@ template <int BT>
 __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *gring)
 {
     const uint64_t pol = l2_policy_evict_first();
-    const int H = p.H, N = p.N;
+    const int H = p.H, N = p.N, G = gridDim.x, nch = p.nchunks;
     const uint32_t row_bytes = (uint32_t)H * 2u;
     const int rows_per_stage = min(kChunk, kGateStageBytes / (int)row_bytes);
-    // this CTA's contiguous neuron range [nb0, nb1): N / gridDim neurons, +-1;
-    // its first `own` chunks are this CTA's, the rest go to the shared pool
-    const int nb0 = (int)((long long)blockIdx.x * N / gridDim.x);
-    const int nb1 = (int)((long long)(blockIdx.x + 1) * N / gridDim.x);
-    const int own = max(0, (nb1 - nb0 + kChunk - 1) / kChunk - kPoolChunksPerCta);
-    int next_k = -1;   // a claimed, not yet used pool chunk
-    bool waited = false;   // the workspace's pool counter is used only after the previous grid ended
+    // chunk k holds neurons [8k, 8k + 8); chunks c + s G (s < kStaticChunks) are this
+    // CTA's; the others, from kStaticChunks * G on, are claimed in increasing order
+    const int nstatic = kStaticChunks * G;
+    auto static_chunk = [&](int s) { return (int)blockIdx.x + s * G; };
     {
         // The weights do not depend on the previous call: while it finishes (its tail
-        // leaves HBM mostly idle), start moving the rows this CTA streams first, past
-        // what the gate ring holds, into L2.
-        const size_t first = (size_t)kGateStages * rows_per_stage;
-        const size_t own_rows = (size_t)min(nb1 - nb0, own * kChunk);
-        if (own_rows > first) {
-            const char *src = reinterpret_cast<const char *>(p.wg_t + (size_t)(nb0 + first) * H);
-            size_t left = min((size_t)kL2PrefetchBytes, (own_rows - first) * row_bytes);
-            for (size_t off = 0; left > 0;) {
-                const uint32_t nbytes = (uint32_t)min(left, (size_t)65536);
+        // leaves HBM mostly idle), start moving this CTA's fixed chunks past the first
+        // (which the gate ring takes) into L2.
+        size_t left = kL2PrefetchBytes;
+        for (int s = 1; s < kStaticChunks && left > 0; ++s) {
+            const int k = static_chunk(s);
+            if (k >= nch) break;
+            const int n0 = k * kChunk;
+            const char *src = reinterpret_cast<const char *>(p.wg_t + (size_t)n0 * H);
+            size_t bytes = min(left, (size_t)min(kChunk, N - n0) * row_bytes);
+            left -= bytes;
+            for (size_t off = 0; bytes > 0;) {
+                const uint32_t nbytes = (uint32_t)min(bytes, (size_t)65536);
                 bulk_prefetch_l2(src + off, nbytes);
                 off += nbytes;
-                left -= nbytes;
+                bytes -= nbytes;
             }
         }
     }
-    if (own == 0) {
-        grid_dependency_wait();
-        waited = true;
-        next_k = atomicAdd(p.ctl + kCtlPool, 1);
-    }
+    int next_k = -1;       // a claimed chunk not yet started
+    bool waited = false;   // the claim counter belongs to the previous call until that call has ended
+    auto claim = [&]() {
+        if (!waited) {
+            grid_dependency_wait();
+            waited = true;
+        }
+        return nstatic + atomicAdd(p.ctl + kCtlChunk, 1);
+    };
     uint32_t stage = 0, phase = 0;
     bool ok = true;
     for (int seq = 0;; ++seq) {
         const int buf = seq % kBufs;
         // the buffer's previous list has been formed (first kBufs uses pass)
         if (!mbar_wait(&S.bfree[buf], ((uint32_t)(seq / kBufs) & 1u) ^ 1u, &S.abort)) { ok = false; break; }
-        int n0 = -1, end = 0;
-        if (seq < own) {
-            n0 = nb0 + seq * kChunk;
-            end = nb1;
-            // claim the first pool chunk while the own chunks still stream
-            if (seq + 1 == own && next_k < 0) {
-                if (!waited) { grid_dependency_wait(); waited = true; }
-                next_k = atomicAdd(p.ctl + kCtlPool, 1);
-            }
+        const bool fixed = seq < kStaticChunks && static_chunk(seq) < nch;
+        int k;
+        if (fixed) {
+            k = static_chunk(seq);
         } else {
-            // pool chunk k: chunk (own_c + k % P) of CTA k / P's range; the
-            // next claim is issued before this chunk's rows are streamed
-            for (;;) {
-                const int k = next_k >= 0 ? next_k : atomicAdd(p.ctl + kCtlPool, 1);
-                next_k = -1;
-                if (k >= (int)gridDim.x * kPoolChunksPerCta) break;
-                const int c = k / kPoolChunksPerCta, j = k % kPoolChunksPerCta;
-                const int c0 = (int)((long long)c * N / gridDim.x), c1 = (int)((long long)(c + 1) * N / gridDim.x);
-                const int cown = max(0, (c1 - c0 + kChunk - 1) / kChunk - kPoolChunksPerCta);
-                const int m0 = c0 + (cown + j) * kChunk;
-                if (m0 < c1) {
-                    n0 = m0;
-                    end = c1;
-                    next_k = atomicAdd(p.ctl + kCtlPool, 1);
-                    break;
-                }
-            }
+            k = next_k >= 0 ? next_k : claim();
+            next_k = -1;
         }
+        const int n0 = k < nch ? k * kChunk : -1;
         if (n0 < 0) {
             S.chunkq[buf] = -1;                                   // end of work for the list producer
             for (int w = 0; w < kGateWarps; ++w) mbar_arrive(&S.gsync[buf]);
             break;
         }
-        const int rows = min(kChunk, end - n0);
+        const int rows = min(kChunk, N - n0);
         S.chunkq[buf] = n0;
         S.chunkrows[buf] = rows;
         for (int r0 = 0; r0 < rows; r0 += rows_per_stage) {
@@ -312,6 +331,9 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
             if (++stage == kGateStages) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
+        // the next chunk is a claimed one: claim it while this chunk's rows stream
+        const bool next_fixed = seq + 1 < kStaticChunks && static_chunk(seq + 1) < nch;
+        if (!next_fixed) next_k = claim();
     }
     if (ok && mbar_wait(&S.gempty[stage], phase ^ 1u, &S.abort)) {
         S.gdesc[stage].kind = kEnd;
@@ -389,31 +411,25 @@ __device__ void gate_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *g
     }
 }
 
-// Row stride of the keep bytes (16-byte aligned rows, so they load as uint4).
-__device__ __forceinline__ int keep_stride(int N) { return (N + 15) & ~15; }
-
-// The 16 keep bytes of block q with the bytes of neurons >= N cleared: the
-// padding at the end of a row is never written and holds stale data.
-__device__ __forceinline__ uint4 keep_block(const uint4 *row, int q, int N)
+// Waits (bounded) until every CTA has passed its prologue.
+__device__ bool wait_prologues(int *ctl)
 {
-    uint4 v = __ldcg(row + q);
-    const int valid = N - 16 * q;
-    if (valid < 16) {
-        uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const int c = min(4, max(0, valid - 4 * j));
-            w[j] &= c == 4 ? 0xffffffffu : ((1u << (8 * c)) - 1u);
+    const unsigned long long t0 = global_ns();
+    while (ld_acquire_gpu(ctl + kCtlPrologue) < (int)gridDim.x) {
+        if (global_ns() - t0 > kWaitLimitNs) {
+            flag_status(ctl, kStatusTimeout);
+            return false;
         }
-        v = make_uint4(w[0], w[1], w[2], w[3]);
+        __nanosleep(64);
     }
-    return v;
+    return true;
 }
 
 // ------------------------------------------------------------------ list producer
 // Lane r = row r of the chunk: sums the gate partials across the gate warps,
-// SiLU (Eq. 2), CATS mask (Eqs. 4-5) per token, index outputs.  Returns the
-// union of rows kept by any token, with each lane's a values and keep bits.
+// SiLU (Eq. 2), CATS mask (Eqs. 4-5) per token, keep trace.  Returns the
+// union of rows kept by any token, with each lane's a values and the kept rows
+// per token.
 template <int BT>
 __device__ uint32_t chunk_keep(const FusedParams &p, Shared<BT> &S, int buf, int n0, int rows, int lane,
                                float (&a)[BT], uint32_t (&bal)[BT])
@@ -436,9 +452,7 @@ __device__ uint32_t chunk_keep(const FusedParams &p, Shared<BT> &S, int buf, int
 #pragma unroll
         for (int b = 0; b < BT; ++b) {
             if (b >= p.nb) break;
-            const uint8_t k = (uint8_t)((bal[b] >> lane) & 1u);
-            if (p.active_idx) p.keep_tmp[(size_t)b * keep_stride(p.N) + n0 + lane] = k;
-            if (p.keep_trace) p.keep_trace[(size_t)b * p.N + n0 + lane] = k;
+            if (p.keep_trace) p.keep_trace[(size_t)b * p.N + n0 + lane] = (uint8_t)((bal[b] >> lane) & 1u);
         }
     }
     return uni;
@@ -454,6 +468,13 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
     const uint32_t lt = (1u << lane) - 1u;
     uint32_t stage = 0, phase = 0;
     grid_dependency_wait();   // the workspace and y belong to the previous launch until it ends
+    if (lane < BT) {
+        // per-token threshold (0: the token takes the dense path); only this warp reads it
+        float t = INFINITY;
+        if (lane < p.nb) t = (p.dense_flags && p.dense_flags[lane]) ? 0.f : p.t_l;
+        S.thr[lane] = t;
+    }
+    __syncwarp();
     if (p.out_mode == kOutY) {
         // zero this CTA's slice of y; every CTA adds into y only after all
         // CTAs have passed their prologue (kCtlPrologue)
@@ -463,14 +484,44 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         for (int q = blockIdx.x * per + lane; q < q1; q += 32)
             reinterpret_cast<float4 *>(p.out)[q] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
+    if (p.active_idx) {
+        // clear this CTA's chunk words and slice word (read and written only after every prologue)
+        const int per = (p.nchunks + gridDim.x - 1) / gridDim.x;
+        const int j1 = min(p.nchunks, (int)(blockIdx.x + 1) * per);
+        for (int j = blockIdx.x * per + lane; j < j1; j += 32) p.flags[j] = 0ull;
+        if (lane == 0) p.flags[p.nchunks + blockIdx.x] = 0ull;
+    }
+    __threadfence();
     bool ok = mbar_wait(&S.xloaded, 0u, &S.abort);
     __syncwarp();
     if (ok && lane == 0) {
-        // this CTA has read its activations and zeroed its slice of y
+        // this CTA has read its activations, zeroed its slice of y and cleared its flags
         __threadfence();
         atomicAdd(p.ctl + kCtlPrologue, 1);
     }
     __syncwarp();
+    // Lane 0 publishes each chunk's word once every CTA has cleared its words;
+    // words of chunks finished before that wait in shared memory (and the warp
+    // waits for the prologues once kPendingChunks of them are held).
+    bool flags_open = false;
+    int npend = 0;
+    auto publish = [&](int k, uint64_t w, bool must) -> bool {
+        if (!flags_open) flags_open = ld_acquire_gpu(p.ctl + kCtlPrologue) >= (int)gridDim.x;
+        if (!flags_open && (must || npend == kPendingChunks)) {
+            flags_open = wait_prologues(p.ctl);
+            if (!flags_open) return false;
+        }
+        if (!flags_open) {
+            S.pend_chunk[npend] = k;
+            S.pend_word[npend] = w;
+            ++npend;
+            return true;
+        }
+        for (int i = 0; i < npend; ++i) st_relaxed_gpu_u64(p.flags + S.pend_chunk[i], S.pend_word[i]);
+        npend = 0;
+        if (k >= 0) st_relaxed_gpu_u64(p.flags + k, w);
+        return true;
+    };
     for (int seq = 0; ok; ++seq) {
         const int buf = seq % kBufs;
         if (!mbar_wait(&S.gsync[buf], (uint32_t)(seq / kBufs) & 1u, &S.abort)) { ok = false; break; }
@@ -483,6 +534,17 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         const uint32_t uni = chunk_keep<BT>(p, S, buf, n0, rows, lane, a, bal);
         __syncwarp();
         if (lane == 0) mbar_arrive(&S.bfree[buf]);   // partials read: the gate producer may refill the buffer
+        if (p.active_idx) {
+            int good = 1;
+            if (lane == 0) {
+                uint64_t w = kChunkKept;
+#pragma unroll
+                for (int b = 0; b < BT; ++b)
+                    if (b < p.nb) w |= (uint64_t)(bal[b] & 0xFFu) << (8 * b);
+                good = publish(n0 / kChunk, w, false) ? 1 : 0;
+            }
+            if (!__shfl_sync(0xffffffffu, good, 0)) { ok = false; break; }
+        }
         const int cnt = __popc(uni);
         const int pos = __popc(uni & lt);
         const bool mine = (uni >> lane) & 1u;
@@ -512,6 +574,11 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         }
         if (!ok) break;
     }
+    if (ok && p.active_idx) {
+        int good = 1;
+        if (lane == 0 && npend > 0) good = publish(-1, 0ull, true) ? 1 : 0;
+        ok = __shfl_sync(0xffffffffu, good, 0) != 0;
+    }
     if (ok && mbar_wait(&S.uempty[stage], phase ^ 1u, &S.abort)) {
         if (lane == 0) {
             S.udesc[stage].kind = kEnd;
@@ -522,6 +589,161 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         flag_status(p.ctl, kStatusTimeout);
     }
     __syncwarp();
+}
+
+
+// ------------------------------------------------------------------ index warp
+// Lane 0 waits (bounded, with backoff, one load at a time so that the words'
+// L2 lines are not flooded) until word w is published; warp-uniform result.
+template <int BT>
+__device__ __forceinline__ bool wait_word(const uint64_t *w, Shared<BT> &S, unsigned long long t0, int lane)
+{
+    int good = 1;
+    if (lane == 0) {
+        uint32_t ns = 64;
+        while (flag_state(ld_relaxed_gpu_u64(w)) == 0u) {
+            if (global_ns() - t0 > kWaitLimitNs || *(volatile int *)&S.abort) {
+                good = 0;
+                break;
+            }
+            __nanosleep(ns);
+            ns = min(ns * 2u, 512u);
+        }
+    }
+    return __shfl_sync(0xffffffffu, good, 0) != 0;
+}
+
+// The ascending per-token index lists, one slice of chunks per CTA.  The
+// entries of a chunk start at the number of neurons kept in all earlier chunks:
+//   1. the slice's kept counts, summed once each of its chunk words is published
+//      (slices are contiguous in chunk order, and chunks are taken in increasing
+//      order, so slices complete in about that order during the call);
+//   2. the slice's prefix, by a decoupled look-back over the slice words of
+//      the CTAs before it in one step (kMaxGrid words, kLookWords per lane): the
+//      counts of the slices after the nearest published prefix; it publishes its
+//      own prefix and those of the slices it summed;
+//   3. each chunk's entries, from a warp scan of the chunks' counts.
+template <int BT>
+__device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
+{
+    static_assert(BT <= 2, "slice words carry two tokens' counts");
+    if (!p.active_idx) return;
+    const int N = p.N, nch = p.nchunks, c = blockIdx.x;
+    const int per = (nch + gridDim.x - 1) / gridDim.x;
+    const int k0 = c * per, k1 = min(nch, k0 + per);
+    if (k0 >= k1) return;   // no chunks: only slices after the last chunk are empty
+    // the control words and index words belong to the previous call until it has ended
+    grid_dependency_wait();
+    int go = 1;
+    if (lane == 0) go = wait_prologues(p.ctl) ? 1 : 0;   // every word is cleared for this call
+    if (!__shfl_sync(0xffffffffu, go, 0)) {
+        if (lane == 0) S.abort = 1;
+        return;
+    }
+    const unsigned long long t0 = global_ns();
+    uint64_t *sw = p.flags + nch;   // slice words
+    bool ok = true;
+    // 1.
+    uint64_t own = 0;
+    for (int base = k0; base < k1 && ok; base += 32) {
+        const int k = base + lane;
+        uint64_t f;
+        for (;;) {
+            f = k < k1 ? ld_relaxed_gpu_u64(p.flags + k) : kChunkKept;
+            const uint32_t missing = __ballot_sync(0xffffffffu, flag_state(f) == 0u);
+            if (!missing) break;
+            if (!wait_word<BT>(p.flags + base + __ffs(missing) - 1, S, t0, lane)) { ok = false; break; }
+        }
+        if (k < k1) own += make_flag(0, __popc(chunk_rows(f, 0)), BT > 1 ? __popc(chunk_rows(f, 1)) : 0u);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) own += __shfl_xor_sync(0xffffffffu, own, o);
+    // 2.
+    uint64_t excl = 0;
+    if (ok && lane == 0) st_relaxed_gpu_u64(sw + c, (c == 0 ? kFlagInc : kFlagAgg) | own);
+    if (ok && c > 0) {
+        for (;;) {
+            // slice c-1-d for d = 32 i + lane
+            uint64_t f[kLookWords];
+#pragma unroll
+            for (int i = 0; i < kLookWords; ++i) {
+                const int j = c - 1 - (32 * i + lane);
+                f[i] = j >= 0 ? ld_relaxed_gpu_u64(sw + j) : kFlagInc;   // before slice 0: 0
+            }
+            int first = 32 * kLookWords, missing = 32 * kLookWords;
+#pragma unroll
+            for (int i = kLookWords - 1; i >= 0; --i) {
+                const uint32_t inc = __ballot_sync(0xffffffffu, flag_state(f[i]) == 2u);
+                const uint32_t unready = __ballot_sync(0xffffffffu, flag_state(f[i]) == 0u);
+                if (inc) first = 32 * i + __ffs(inc) - 1;
+                if (unready) missing = 32 * i + __ffs(unready) - 1;
+            }
+            // first <= c always (the words before slice 0 read as prefix 0)
+            if (missing < first) {
+                if (!wait_word<BT>(sw + (c - 1 - missing), S, t0, lane)) { ok = false; break; }
+                continue;
+            }
+            uint64_t part = 0;
+#pragma unroll
+            for (int i = 0; i < kLookWords; ++i)
+                if (32 * i + lane <= first) part += f[i] & kFlagPayload;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+            excl = part;
+            if (lane == 0) st_relaxed_gpu_u64(sw + c, kFlagInc | (excl + own));
+            // slice c-1-d (d < first) ends at excl minus the slices after it
+            uint64_t after = 0;
+#pragma unroll
+            for (int i = 0; i < kLookWords; ++i) {
+                const int d = 32 * i + lane;
+                const uint64_t v = d < first ? (f[i] & kFlagPayload) : 0ull;
+                uint64_t incl = v;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const uint64_t t = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += t;
+                }
+                if (d < first) st_relaxed_gpu_u64(sw + (c - 1 - d), kFlagInc | (excl - (after + incl - v)));
+                after += __shfl_sync(0xffffffffu, incl, 31);
+            }
+            break;
+        }
+    }
+    if (!ok) {
+        if (lane == 0) {
+            S.abort = 1;
+            flag_status(p.ctl, kStatusTimeout);
+        }
+        return;
+    }
+    // 3.
+    uint32_t run[2] = {flag_value(excl, 0), flag_value(excl, 1)};
+    for (int base = k0; base < k1; base += 32) {
+        const int k = base + lane;
+        const uint64_t f = k < k1 ? ld_relaxed_gpu_u64(p.flags + k) : 0ull;
+#pragma unroll
+        for (int b = 0; b < BT; ++b) {
+            uint32_t m = k < k1 ? chunk_rows(f, b) : 0u;
+            const uint32_t cnt = (uint32_t)__popc(m);
+            uint32_t pre = cnt;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t t = __shfl_up_sync(0xffffffffu, pre, o);
+                if (lane >= o) pre += t;
+            }
+            uint32_t pos = run[b > 0 ? 1 : 0] + pre - cnt;
+            for (; m; m &= m - 1u, ++pos) {
+                if (pos < (uint32_t)N) p.active_idx[(size_t)b * N + pos] = k * kChunk + __ffs(m) - 1;
+                else flag_status(p.ctl, kStatusInternal);
+            }
+            run[b > 0 ? 1 : 0] += __shfl_sync(0xffffffffu, pre, 31);
+        }
+    }
+    if (k1 == nch && lane == 0 && p.active_cnt) {
+#pragma unroll
+        for (int b = 0; b < BT; ++b)
+            if (b < p.nb) p.active_cnt[b] = (int)run[b > 0 ? 1 : 0];
+    }
 }
 
 // ------------------------------------------------------------------ up/down warps
@@ -664,86 +886,6 @@ __device__ void drain_copies(Shared<BT> &S)
         if (S.uissued[s] > 0) (void)mbar_wait(&S.ufull[s], (uint32_t)(S.uissued[s] - 1), &never);
 }
 
-// ------------------------------------------------------------------ tail
-// Waits (bounded) until every CTA has passed its prologue.
-__device__ bool wait_prologues(int *ctl)
-{
-    const unsigned long long t0 = global_ns();
-    while (ld_acquire_gpu(ctl + kCtlPrologue) < (int)gridDim.x) {
-        if (global_ns() - t0 > kWaitLimitNs) {
-            flag_status(ctl, kStatusTimeout);
-            return false;
-        }
-        __nanosleep(64);
-    }
-    return true;
-}
-
-// The ascending per-token kept lists from the keep bytes of all chunks; run by
-// the last CTA to finish, when every chunk's bytes are in memory.
-template <int BT>
-__device__ void compact_indices(const FusedParams &p, Shared<BT> &S, int *stage_buf, int stage_cap)
-{
-    constexpr int kMaxBlocksPerThread = 8;                  // 16 keep bytes per block
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int N = p.N;
-    const int nblk = keep_stride(N) / 16;
-    const int bpt = (nblk + kThreads - 1) / kThreads;       // contiguous blocks per thread
-    const int q0 = tid * bpt;
-    for (int b = 0; b < p.nb; ++b) {
-        const uint4 *kb = reinterpret_cast<const uint4 *>(p.keep_tmp + (size_t)b * keep_stride(N));
-        // one pass of independent 16-byte loads for the common sizes, then a loop
-        uint4 blk[kMaxBlocksPerThread];
-        int cnt = 0;
-#pragma unroll
-        for (int i = 0; i < kMaxBlocksPerThread; ++i) {
-            blk[i] = (i < bpt && q0 + i < nblk) ? keep_block(kb, q0 + i, N) : make_uint4(0u, 0u, 0u, 0u);
-        }
-#pragma unroll
-        for (int i = 0; i < kMaxBlocksPerThread; ++i)
-            cnt += __popc(blk[i].x) + __popc(blk[i].y) + __popc(blk[i].z) + __popc(blk[i].w);   // bytes are 0 or 1
-        for (int i = kMaxBlocksPerThread; i < bpt && q0 + i < nblk; ++i) {
-            const uint4 v = keep_block(kb, q0 + i, N);
-            cnt += __popc(v.x) + __popc(v.y) + __popc(v.z) + __popc(v.w);
-        }
-        // block-wide exclusive scan of the counts
-        int incl = cnt;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int v = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += v;
-        }
-        if (lane == 31) S.warp_sums[warp] = incl;
-        __syncthreads();
-        int base = 0, total = 0;
-        for (int w = 0; w < kThreads / 32; ++w) {
-            if (w < warp) base += S.warp_sums[w];
-            total += S.warp_sums[w];
-        }
-        int pos = base + incl - cnt;
-        // the list is assembled in shared memory (the idle rings) and then
-        // written with coalesced stores; a list too long for it goes straight out
-        const bool staged = total <= stage_cap;
-        int32_t *dst = p.active_idx + (size_t)b * N;
-        int32_t *out = staged ? stage_buf : dst;
-        for (int i = 0; i < bpt && q0 + i < nblk; ++i) {
-            const uint4 v = i < kMaxBlocksPerThread ? blk[i] : keep_block(kb, q0 + i, N);
-            const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
-            const int nbase = (q0 + i) * 16;
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-#pragma unroll
-                for (int e = 0; e < 4; ++e)
-                    if ((w4[j] >> (8 * e)) & 0xffu) out[pos++] = nbase + 4 * j + e;
-        }
-        if (tid == 0 && p.active_cnt) p.active_cnt[b] = total;
-        __syncthreads();
-        if (staged) {
-            for (int i = tid; i < total; i += kThreads) dst[i] = stage_buf[i];
-            __syncthreads();
-        }
-    }
-}
 
 template <int BT, int VPT>
 __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParams p)
@@ -776,11 +918,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
         S.abort = 0;
         mbar_init_fence();
     }
-    if (tid < BT) {
-        float t = INFINITY;
-        if (tid < p.nb) t = (p.dense_flags && p.dense_flags[tid]) ? 0.f : p.t_l;
-        S.thr[tid] = t;
-    }
     __syncthreads();
     // the next launch in the stream may start its weight stream on SMs this
     // grid frees; it waits for this grid's end before touching x, y or the workspace
@@ -794,8 +931,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
     } else if (warp == kGateProducerWarp) {
         if (lane == 0) gate_producer<BT>(p, S, gring);
         __syncwarp();
-    } else {
+    } else if (warp == kListWarp) {
         list_producer<BT>(p, S, uring, lane);
+    } else {
+        index_warp<BT>(p, S, lane);
     }
     __syncthreads();
     if (tid == 0 && S.abort) drain_copies<BT>(S);
@@ -832,17 +971,12 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
         __threadfence();
     }
     __syncthreads();
-    if (last_s) {
-        // every other CTA has added its y, written its keep bytes and is past
-        // its wait on kCtlPrologue
-        if (p.active_idx && !S.abort)
-            compact_indices<BT>(p, S, reinterpret_cast<int *>(smem),
-                                (kGateStages * kGateStageBytes + kUdRingBytes) / (int)sizeof(int));
-        if (tid == 0) {
-            atomicExch(p.ctl + kCtlPrologue, 0);
-            atomicExch(p.ctl + kCtlPool, 0);
-            atomicExch(p.ctl + kCtlDone, 0);
-        }
+    if (last_s && tid == 0) {
+        // every other CTA has added its y, finished its claims and index lists
+        // and is past its waits on kCtlPrologue
+        atomicExch(p.ctl + kCtlPrologue, 0);
+        atomicExch(p.ctl + kCtlChunk, 0);
+        atomicExch(p.ctl + kCtlDone, 0);
     }
 }
 

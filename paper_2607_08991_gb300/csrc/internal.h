@@ -36,20 +36,26 @@ constexpr int kMaxN = 1 << 20;
 
 // Control block at the start of the workspace (ints).
 enum {
-    kCtlChunk = 0,      // reserved
-    kCtlBarCount = 1,   // grid barrier arrivals, reset to 0 by the last arrival
-    kCtlBarGen = 2,     // grid barrier generation
+    kCtlChunk = 0,      // next dynamically claimed chunk of the fused kernel (reset by the last CTA)
+    kCtlBarCount = 1,   // reserved
+    kCtlBarGen = 2,     // reserved
     kCtlStatus = 3,     // device status word (kStatus* bits)
     kCtlNDense = 4,     // route output of the stack driver
     kCtlPrologue = 5,   // CTAs that have read their activations (reset by the last CTA)
     kCtlDone = 6,       // CTAs that have added their partial y (reset by the last CTA)
-    kCtlPool = 7,       // next chunk of the shared tail pool (reset by the last CTA)
+    kCtlReserved7 = 7,  // reserved
     kCtlInts = 64
 };
 
+// Workspace regions.  flags: the fused kernel's index-list words, one 64-bit
+// word per chunk of kChunk neurons (its kept rows) and one per CTA (its slice's
+// kept counts and prefix), cleared by the kernel itself at the start of each call.
 struct WsLayout {
-    size_t ctl, keep, route_perm, route_flags, tc, total;
+    size_t ctl, flags, route_perm, route_flags, tc, total;
 };
+
+// Zeroes the control words of a workspace (the fused kernel's counters and status).
+cudaError_t clear_fused_state(void *ws, int H, int N, int B, cudaStream_t stream);
 WsLayout ws_layout(int H, int N, int B);
 
 enum XMode { kXBf16 = 0, kXF32 = 1, kXResidNorm = 2 };
@@ -69,7 +75,7 @@ struct FusedParams {
     int out_mode;
     float *out;                   // kOutY: y [nb][H]; kOutResid: residual [nb][H] (+=)
     int *ctl;                     // workspace control block
-    uint8_t *keep_tmp;            // [kMaxTokensPerPass][N]: keep byte per neuron (index output only)
+    uint64_t *flags;              // [nchunks + kMaxGrid]: index-list words (index output only)
     int32_t *active_idx;          // [nb][N] or nullptr
     int32_t *active_cnt;          // [nb] or nullptr
     uint8_t *keep_trace;          // [nb][N] or nullptr

@@ -55,7 +55,7 @@ def test_fixed_scratch_matches_workspace_entry(sats, oracle, H, N, B, k):
 
 
 def test_fixed_scratch_refuses_shapes_beyond_its_limit(sats):
-    H, N = 8, 300000            # four keep bytes per neuron: 1.2 MB > 1 MiB
+    H, N = 8, 300000            # one flag byte per neuron: 300 KB > 256 KiB
     z = torch.zeros(H, N, dtype=torch.int16, device="cuda")
     layer = sats.Layer(z, z, torch.zeros(N, H, dtype=torch.int16, device="cuda"))
     x = torch.zeros(1, H, dtype=torch.int16, device="cuda")
