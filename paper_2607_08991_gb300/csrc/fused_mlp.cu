@@ -131,6 +131,8 @@ struct Shared {
     uint64_t pend_word[kPendingChunks];   // chunk words not yet published (list producer)
     int pend_chunk[kPendingChunks];
     int abort;
+    int seen;                   // the list producer has seen every CTA past its prologue
+    int quiet;                  // roles past their last use of the counters (list producer, index warp)
 };
 
 template <int BT>
@@ -425,6 +427,24 @@ __device__ bool wait_prologues(int *ctl)
     return true;
 }
 
+// Called once by the list producer and once by the index warp (one thread
+// each), when each has made its last use of the control counters (the gate
+// producer's claims precede the list producer's end).  The second call counts
+// the CTA done; the last CTA counted resets the counters for the next call,
+// which uses them only after this grid has ended.
+template <int BT>
+__device__ void counters_released(const FusedParams &p, Shared<BT> &S)
+{
+    uint32_t prior;
+    asm volatile("atom.acq_rel.cta.shared.add.u32 %0, [%1], 1;" : "=r"(prior) : "r"(smem_addr(&S.quiet)) : "memory");
+    if (prior != 1u) return;
+    if (atom_add_acq_rel_gpu(p.ctl + kCtlDone, 1) == (int)gridDim.x - 1) {
+        atomicExch(p.ctl + kCtlPrologue, 0);
+        atomicExch(p.ctl + kCtlChunk, 0);
+        atomicExch(p.ctl + kCtlDone, 0);
+    }
+}
+
 // ------------------------------------------------------------------ list producer
 // Lane r = row r of the chunk: sums the gate partials across the gate warps,
 // SiLU (Eq. 2), CATS mask (Eqs. 4-5) per token, keep trace.  Returns the
@@ -534,7 +554,9 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         const uint32_t uni = chunk_keep<BT>(p, S, buf, n0, rows, lane, a, bal);
         __syncwarp();
         if (lane == 0) mbar_arrive(&S.bfree[buf]);   // partials read: the gate producer may refill the buffer
-        if (p.active_idx) {
+        if (!p.active_idx) {
+            if (lane == 0 && !flags_open) flags_open = ld_acquire_gpu(p.ctl + kCtlPrologue) >= (int)gridDim.x;
+        } else {
             int good = 1;
             if (lane == 0) {
                 uint64_t w = kChunkKept;
@@ -588,9 +610,14 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         S.abort = 1;
         flag_status(p.ctl, kStatusTimeout);
     }
+    if (lane == 0) {
+        // the CTA adds into y only after every CTA has read its activations
+        if (!flags_open && !*(volatile int *)&S.abort) flags_open = wait_prologues(p.ctl);
+        S.seen = flags_open ? 1 : 0;
+        counters_released<BT>(p, S);
+    }
     __syncwarp();
 }
-
 
 // ------------------------------------------------------------------ index warp
 // Lane 0 waits (bounded, with backoff, one load at a time so that the words'
@@ -613,6 +640,26 @@ __device__ __forceinline__ bool wait_word(const uint64_t *w, Shared<BT> &S, unsi
     return __shfl_sync(0xffffffffu, good, 0) != 0;
 }
 
+// Each lane whose `need` is set waits (bounded, with backoff) until its word is
+// published; warp-uniform result.
+template <int BT>
+__device__ __forceinline__ bool wait_words(const uint64_t *w, bool need, Shared<BT> &S, unsigned long long t0)
+{
+    int good = 1;
+    if (need) {
+        uint32_t ns = 64;
+        while (flag_state(ld_relaxed_gpu_u64(w)) == 0u) {
+            if (global_ns() - t0 > kWaitLimitNs || *(volatile int *)&S.abort) {
+                good = 0;
+                break;
+            }
+            __nanosleep(ns);
+            ns = min(ns * 2u, 512u);
+        }
+    }
+    return __all_sync(0xffffffffu, good) != 0;
+}
+
 // The ascending per-token index lists, one slice of chunks per CTA.  The
 // entries of a chunk start at the number of neurons kept in all earlier chunks:
 //   1. the slice's kept counts, summed once each of its chunk words is published
@@ -627,15 +674,19 @@ template <int BT>
 __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
 {
     static_assert(BT <= 2, "slice words carry two tokens' counts");
-    if (!p.active_idx) return;
     const int N = p.N, nch = p.nchunks, c = blockIdx.x;
     const int per = (nch + gridDim.x - 1) / gridDim.x;
     const int k0 = c * per, k1 = min(nch, k0 + per);
-    if (k0 >= k1) return;   // no chunks: only slices after the last chunk are empty
     // the control words and index words belong to the previous call until it has ended
     grid_dependency_wait();
+    // no lists, or no chunks (only slices after the last chunk are empty)
+    const bool work = p.active_idx != nullptr && k0 < k1;
     int go = 1;
-    if (lane == 0) go = wait_prologues(p.ctl) ? 1 : 0;   // every word is cleared for this call
+    if (lane == 0) {
+        if (work) go = wait_prologues(p.ctl) ? 1 : 0;   // every word is cleared for this call
+        counters_released<BT>(p, S);                   // the index warp's only counter read is above
+    }
+    if (!work) return;
     if (!__shfl_sync(0xffffffffu, go, 0)) {
         if (lane == 0) S.abort = 1;
         return;
@@ -644,7 +695,7 @@ __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
     uint64_t *sw = p.flags + nch;   // slice words
     bool ok = true;
     // 1.
-    uint64_t own = 0;
+    uint64_t own = 0, f_first = 0;   // f_first: the words of the slice's first 32 chunks, kept for step 3
     for (int base = k0; base < k1 && ok; base += 32) {
         const int k = base + lane;
         uint64_t f;
@@ -654,6 +705,7 @@ __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
             if (!missing) break;
             if (!wait_word<BT>(p.flags + base + __ffs(missing) - 1, S, t0, lane)) { ok = false; break; }
         }
+        if (base == k0) f_first = f;
         if (k < k1) own += make_flag(0, __popc(chunk_rows(f, 0)), BT > 1 ? __popc(chunk_rows(f, 1)) : 0u);
     }
 #pragma unroll
@@ -678,9 +730,16 @@ __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
                 if (inc) first = 32 * i + __ffs(inc) - 1;
                 if (unready) missing = 32 * i + __ffs(unready) - 1;
             }
-            // first <= c always (the words before slice 0 read as prefix 0)
+            // first <= c always (the words before slice 0 read as prefix 0); wait for
+            // every unpublished word before the nearest prefix at once, then read again
             if (missing < first) {
-                if (!wait_word<BT>(sw + (c - 1 - missing), S, t0, lane)) { ok = false; break; }
+                bool wait_ok = true;
+#pragma unroll
+                for (int i = 0; i < kLookWords; ++i) {
+                    const int d = 32 * i + lane;
+                    wait_ok = wait_words<BT>(sw + (c - 1 - d), d < first && flag_state(f[i]) == 0u, S, t0) && wait_ok;
+                }
+                if (!wait_ok) { ok = false; break; }
                 continue;
             }
             uint64_t part = 0;
@@ -720,7 +779,7 @@ __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
     uint32_t run[2] = {flag_value(excl, 0), flag_value(excl, 1)};
     for (int base = k0; base < k1; base += 32) {
         const int k = base + lane;
-        const uint64_t f = k < k1 ? ld_relaxed_gpu_u64(p.flags + k) : 0ull;
+        const uint64_t f = k >= k1 ? 0ull : (base == k0 ? f_first : ld_relaxed_gpu_u64(p.flags + k));
 #pragma unroll
         for (int b = 0; b < BT; ++b) {
             uint32_t m = k < k1 ? chunk_rows(f, b) : 0u;
@@ -916,6 +975,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
         mbar_init(&S.gbar, kGateWarps);
         mbar_init(&S.ubar, kUdWarps);
         S.abort = 0;
+        S.seen = 0;
+        S.quiet = 0;
         mbar_init_fence();
     }
     __syncthreads();
@@ -939,12 +1000,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
     __syncthreads();
     if (tid == 0 && S.abort) drain_copies<BT>(S);
 
-    // add this CTA's partial y into the output, once every CTA has read its
-    // activations (and zeroed its slice of y)
-    __shared__ int go_s;
-    if (tid == 0) go_s = wait_prologues(p.ctl) ? 1 : 0;
-    __syncthreads();
-    if (go_s && warp >= kGateWarps && warp < kGateProducerWarp) {
+    // add this CTA's partial y into the output: the list producer has seen every
+    // CTA past its prologue (every CTA has read its activations and zeroed its slice of y)
+    if (S.seen && warp >= kGateWarps && warp < kGateProducerWarp) {
         const int t = tid - kGateThreads;
         const int HV = p.H >> 3;
 #pragma unroll
@@ -962,21 +1020,6 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
                 }
             }
         }
-    }
-    __syncthreads();
-    __shared__ int last_s;
-    if (tid == 0) {
-        __threadfence();
-        last_s = atomicAdd(p.ctl + kCtlDone, 1) == (int)gridDim.x - 1;
-        __threadfence();
-    }
-    __syncthreads();
-    if (last_s && tid == 0) {
-        // every other CTA has added its y, finished its claims and index lists
-        // and is past its waits on kCtlPrologue
-        atomicExch(p.ctl + kCtlPrologue, 0);
-        atomicExch(p.ctl + kCtlChunk, 0);
-        atomicExch(p.ctl + kCtlDone, 0);
     }
 }
 

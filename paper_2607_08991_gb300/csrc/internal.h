@@ -42,7 +42,7 @@ enum {
     kCtlStatus = 3,     // device status word (kStatus* bits)
     kCtlNDense = 4,     // route output of the stack driver
     kCtlPrologue = 5,   // CTAs that have read their activations (reset by the last CTA)
-    kCtlDone = 6,       // CTAs that have added their partial y (reset by the last CTA)
+    kCtlDone = 6,       // CTAs past their last use of the counters (reset by the last CTA)
     kCtlReserved7 = 7,  // reserved
     kCtlInts = 64
 };
