@@ -177,6 +177,28 @@ SATS_API sats_status sats_sparse_mlp_f32(const sats_layer *layer, const float *x
                                 void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * sats_sparse_mlp_union, sats_sparse_mlp_union_f32 -- sats_sparse_mlp for a
+ * batch of 3 to 8 tokens (H <= 4096), computed over the union of the tokens'
+ * kept neurons: the gate runs over all neurons on the tensor cores; then only
+ * neurons some token keeps have their W_up column and W_down row read, once for
+ * the whole batch (Sec. 2, Eqs. 1-5 per token: each token still keeps exactly
+ * its own neurons, so the result equals sats_sparse_mlp's).  This reads
+ * 2HN (1 + 2 |U| / N) bytes instead of 6HN, |U| the union size, which pays
+ * when the tokens' kept sets overlap strongly; for independent kept sets at
+ * these batch sizes the default path of sats_sparse_mlp is faster.
+ * Arguments, results and errors are those of sats_sparse_mlp (x bf16) and
+ * sats_sparse_mlp_f32 (x fp32, carried as bf16 high and low parts), with a
+ * workspace of sats_workspace_bytes(H, N, B); B outside [3, 8] or H > 4096
+ * returns SATS_ESHAPE.
+ */
+SATS_API sats_status sats_sparse_mlp_union(const sats_layer *layer, const void *x, int B, float t_l, float *y,
+                                           int32_t *active_idx, int32_t *active_cnt, void *ws, size_t ws_bytes,
+                                           void *stream);
+SATS_API sats_status sats_sparse_mlp_union_f32(const sats_layer *layer, const float *x, int B, float t_l,
+                                               float *y, int32_t *active_idx, int32_t *active_cnt, void *ws,
+                                               size_t ws_bytes, void *stream);
+
+/*
  * sats_dense_mlp -- the base gated MLP of Sec. 2, Eq. 1 (every neuron kept):
  *   x : device bf16 [B][H];  y : device fp32 [B][H].
  */

@@ -280,6 +280,36 @@ sats_status sats_sparse_mlp_f32(const sats_layer *layer, const float *x, int B, 
     return sparse_common(layer, kXF32, x, B, t_l, y, active_idx, active_cnt, ws, ws_bytes, stream);
 }
 
+static sats_status union_common(const sats_layer *layer, int x_mode, const void *x, int B, float t_l, float *y,
+                                int32_t *active_idx, int32_t *active_cnt, void *ws, size_t ws_bytes, void *stream)
+{
+    sats_status s = check_layer(layer, ws, ws_bytes, B);
+    if (s != SATS_OK) return s;
+    if (bad_threshold(t_l)) return SATS_EINVAL;
+    if ((active_idx == nullptr) != (active_cnt == nullptr)) return SATS_EINVAL;
+    if (B < 3 || !union_path_ok(layer->H, B)) return SATS_ESHAPE;
+    if (!x || !y || !aligned16(x) || !aligned16(y)) return SATS_EINVAL;
+    const WsLayout L = ws_layout(layer->H, layer->N, B);
+    char *base = static_cast<char *>(ws);
+    const cudaError_t e = run_tc_layer(layer, x_mode, x, B, t_l, nullptr, 0.f, nullptr, kOutY, y, active_idx,
+                                       active_cnt, nullptr, base + L.tc, reinterpret_cast<int *>(base + L.ctl),
+                                       static_cast<cudaStream_t>(stream), true);
+    return e == cudaSuccess ? SATS_OK : SATS_ECUDA;   // run_tc_layer recorded the failing step
+}
+
+sats_status sats_sparse_mlp_union(const sats_layer *layer, const void *x, int B, float t_l, float *y,
+                                  int32_t *active_idx, int32_t *active_cnt, void *ws, size_t ws_bytes, void *stream)
+{
+    return union_common(layer, kXBf16, x, B, t_l, y, active_idx, active_cnt, ws, ws_bytes, stream);
+}
+
+sats_status sats_sparse_mlp_union_f32(const sats_layer *layer, const float *x, int B, float t_l, float *y,
+                                      int32_t *active_idx, int32_t *active_cnt, void *ws, size_t ws_bytes,
+                                      void *stream)
+{
+    return union_common(layer, kXF32, x, B, t_l, y, active_idx, active_cnt, ws, ws_bytes, stream);
+}
+
 sats_status sats_dense_mlp(const sats_layer *layer, const void *x, int B, float *y, void *ws, size_t ws_bytes,
                            void *stream)
 {

@@ -28,135 +28,11 @@
 // the TMEM allocation and lane 0 issues the MMAs, warps 2-5 run the epilogue
 // (warp w reads TMEM lanes 32 (w mod 4) .. 32 (w mod 4) + 31).  Every wait is
 // bounded in time and sets the status word when it gives up.
-#include <cuda.h>
-#include <cuda_bf16.h>
-#include <cudaTypedefs.h>
-
-#include <atomic>
-#include <cmath>
-#include <mutex>
-#include <utility>
-
-#include "common.cuh"
-#include "internal.h"
+#include "tc_common.cuh"
 
 namespace sats {
 namespace tc {
 namespace {
-
-constexpr int BM = 128;              // MMA M: rows of the A operand
-constexpr int BK = 64;               // K per TMA box: one 128-byte swizzle row of bf16
-constexpr int kThreads = 192;
-constexpr int kSmemBudget = 196608;  // stage ring (one CTA per SM)
-constexpr int kSmemWide = 225280;    // stage ring of the persistent prefill kernels, at most
-constexpr int kMaxStages = 8;
-constexpr int kMaxSkinny = 256;      // largest batch on the skinny orientation (MMA N <= 256)
-constexpr int kTileBytes = BK * 2;   // bytes of one tile row
-
-// ---------------------------------------------------------------------- device helpers
-// Shared-memory matrix descriptor of a K-major bf16 tile written by TMA with
-// 128-byte swizzle: rows of 128 bytes, 8-row atoms 1024 bytes apart.
-__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr)
-{
-    uint64_t d = 0;
-    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);     // start address
-    d |= (uint64_t)(16u >> 4) << 16;               // leading byte offset (unused for swizzled K-major)
-    d |= (uint64_t)(1024u >> 4) << 32;             // stride byte offset: one 8-row atom
-    d |= (uint64_t)1 << 46;                        // descriptor version of this architecture
-    d |= (uint64_t)2 << 61;                        // 128-byte swizzle
-    return d;
-}
-
-// Instruction descriptor of kind::f16: bf16 A and B (K-major), fp32 D, M x N.
-__host__ __device__ constexpr uint32_t instr_desc(int M, int N)
-{
-    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
-}
-
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc)
-{
-    asm volatile(
-        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
-        ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(acc)
-        : "memory");
-}
-
-// The mbarrier receives one arrival when all previously issued MMAs are done.
-__device__ __forceinline__ void mma_commit(uint64_t *bar)
-{
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
-                 ::"r"(smem_addr(bar)) : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-
-__device__ __forceinline__ void tmem_alloc(uint32_t *slot, uint32_t ncols)
-{
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(slot)), "r"(ncols)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols)
-{
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
-}
-
-// 16 consecutive fp32 columns of this warp's 32 TMEM lanes (one row per thread).
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16])
-{
-    uint32_t r[16];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr)
-        : "memory");
-#pragma unroll
-    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-
-// Error path only (a role gave up waiting): before the CTA releases its TMEM
-// and exits, wait -- again bounded -- for the tile loads still in flight
-// (stages issued but never consumed) and for the MMAs already issued.
-__device__ void drain_after_abort(uint64_t *full, int stages, int issued, int consumed, uint64_t *acc_full)
-{
-    int never = 0;
-    for (int k = consumed; k < issued; ++k)
-        mbar_wait(&full[k % stages], (uint32_t)((k / stages) & 1), &never);
-    mbar_wait(acc_full, 0u, &never);
-}
-
-// One 2D TMA tile load: inner coordinate c0 (elements, a multiple of 64), row c1.
-__device__ __forceinline__ void tma_load(void *dst, const CUtensorMap *map, int c0, int c1, uint64_t *bar)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
-        ::"r"(smem_addr(dst)), "l"(map), "r"(c0), "r"(c1), "r"(smem_addr(bar))
-        : "memory");
-}
-
-__device__ __forceinline__ uint16_t bf16_bits(float v)
-{
-    const __nv_bfloat16 h = __float2bfloat16_rn(v);
-    return *reinterpret_cast<const uint16_t *>(&h);
-}
-
-__device__ __forceinline__ uint8_t *align1024(uint8_t *p)
-{
-    return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(p) + 1023) & ~(uintptr_t)1023);
-}
-
-
-__device__ __forceinline__ void set_timeout(int *ctl, volatile int *abort_flag)
-{
-    *abort_flag = 1;
-    atomicOr(ctl + kCtlStatus, kStatusTimeout);
-}
 
 // ---------------------------------------------------------------------- activations
 // Row m of X (fp32, optionally RMS-normalised with gain w) -> bf16 hi + lo.
@@ -260,13 +136,18 @@ struct SkinnyGuParams {
     int *ctl;
     float *zero;                  // y [M][H] to clear for the down projection's additions, or nullptr
     int zero_count;               // M H (a multiple of 8)
+    // gate-only mode (the union path): no up tile; the epilogue writes a_keep and the union flags
+    int gate_only;
+    float *a_keep;                // [M][ldh] fp32: keep ? SiLU(g) : 0
+    uint8_t *uflag;               // [N]: 1 if any token keeps the neuron
     int stages, stage_bytes, a_bytes, x_bytes;
     int ring_bytes;               // stages * stage_bytes + room for the last up tile's 128-row read
     uint32_t tmem_cols;
 };
 
 // One tile of R neurons (gate and up) against all M tokens: D[r][j] in TMEM
-// lane r, column j (gate) and NT + j (up).  Grid: tc_T CTAs.
+// lane r, column j (gate) and NT + j (up).  Grid: tc_T CTAs.  In gate-only mode
+// only the gate rows are read and multiplied.
 __global__ void __launch_bounds__(kThreads, 1)
     gu_skinny_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmX2,
                      const SkinnyGuParams p)
@@ -300,7 +181,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     grid_launch_dependents();   // the down projection may start prefetching its weights
 
     if (warp == 0 && lane == 0) {
-        const uint32_t w_bytes = (uint32_t)(2 * R * kTileBytes);
+        const uint32_t w_bytes = (uint32_t)((p.gate_only ? 1 : 2) * R * kTileBytes);
         const uint32_t load_bytes = w_bytes + (uint32_t)(p.x_bytes * (p.split ? 2 : 1));
         const uint64_t policy = l2_policy_evict_first();   // each weight tile is read by this CTA only
         // the weight tiles do not depend on the preceding kernel: start them before waiting for it
@@ -339,11 +220,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint64_t au = smem_desc(st + R * kTileBytes + kk * 32);
                 const uint64_t b = smem_desc(xa + kk * 32);
                 mma_bf16(tmem, ag, b, idesc, acc);
-                mma_bf16(tmem + NT, au, b, idesc, acc);
+                if (!p.gate_only) mma_bf16(tmem + NT, au, b, idesc, acc);
                 if (p.split) {
                     const uint64_t b2 = smem_desc(xa + p.x_bytes + kk * 32);
                     mma_bf16(tmem, ag, b2, idesc, 1u);
-                    mma_bf16(tmem + NT, au, b2, idesc, 1u);
+                    if (!p.gate_only) mma_bf16(tmem + NT, au, b2, idesc, 1u);
                 }
             }
             mma_commit(&empty[s]);
@@ -366,9 +247,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int lb = 32 * (warp & 3);
         const int r = lb + lane, n = t * R + r;
         const bool row_ok = ok && r < R && n < p.N;
+        bool any = false;   // gate-only mode: some token keeps neuron n
         for (int c0 = 0; c0 < NT; c0 += 16) {
             float g[16], u[16];
             tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)c0, g);
+            if (p.gate_only) {
+                tmem_ld_wait();
+                if (!row_ok) continue;
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const int j = c0 + e;
+                    if (j < p.M) {
+                        const float a = g[e] / (1.0f + expf(-g[e]));   // SiLU, Eq. 2
+                        const bool keep = fabsf(a) >= p.t_l;            // Eqs. 4-5
+                        any = any || keep;
+                        p.a_keep[(size_t)j * p.ldh + n] = keep ? a : 0.f;
+                        if (p.keep) p.keep[(size_t)j * p.keep_stride + n] = keep ? 1 : 0;
+                        if (p.keep_trace) p.keep_trace[(size_t)j * p.N + n] = keep ? 1 : 0;
+                    }
+                }
+                continue;
+            }
             tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(NT + c0), u);
             tmem_ld_wait();
             if (!row_ok) continue;
@@ -388,6 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
+        if (p.gate_only && row_ok) p.uflag[n] = any ? 1 : 0;
         tc_fence_before();
     }
     __syncthreads();
@@ -925,150 +825,6 @@ __global__ void __launch_bounds__(512) keep_list_kernel(const uint8_t *__restric
 }
 
 
-// ---------------------------------------------------------------------- host
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
-{
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-    });
-    return fn;
-}
-
-// bf16 matrix [rows][cols] with the given row stride (a multiple of 16 bytes),
-// read in boxes of box_rows x 64 with 128-byte swizzle.
-bool make_map(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols, uint64_t row_stride_bytes,
-              uint32_t box_rows)
-{
-    auto fn = encode_fn();
-    if (!fn) return false;
-    const cuuint64_t dims[2] = {cols, rows};
-    const cuuint64_t strides[1] = {row_stride_bytes};
-    const cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
-    const cuuint32_t es[2] = {1, 1};
-    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-// The device's opt-in limit of shared memory per CTA.
-int smem_optin()
-{
-    static int by_dev[64] = {0};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    int &n = by_dev[dev & 63];
-    if (n == 0) cudaDeviceGetAttribute(&n, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-    return n;
-}
-
-// Raises the kernel's dynamic shared-memory limit on the current device to at
-// least `bytes`; `configured` is the caller's per-device record for this kernel.
-template <typename K>
-cudaError_t set_smem(K kernel, size_t bytes, std::atomic<int> (&configured)[64])
-{
-    int dev = 0;
-    cudaGetDevice(&dev);
-    std::atomic<int> &have = configured[dev & 63];
-    if ((int)bytes <= have.load()) return cudaSuccess;
-    const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-    if (e == cudaSuccess) have.store((int)bytes);
-    return e;
-}
-
-// Launch with programmatic dependent launch: the kernel may start while the
-// preceding kernel in the stream finishes; it calls griddepcontrol.wait before
-// touching anything that kernel produces.
-template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, size_t smem, cudaStream_t stream, Args &&...args)
-{
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = grid;
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
-}
-
-// As launch_pdl, for the small kernels (no dynamic shared memory, `threads` per CTA).
-template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl_threads(void (*kernel)(KArgs...), dim3 grid, int threads, cudaStream_t stream, Args &&...args)
-{
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = grid;
-    cfg.blockDim = dim3(threads);
-    cfg.dynamicSmemBytes = 0;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
-}
-
-// Dynamic shared memory of a launch: the stage ring, 1 KB of alignment slack and the barriers.
-size_t smem_for(int stages, int stage_bytes) { return (size_t)stages * stage_bytes + 1024 + 256; }
-
-// Ring budget of the prefill kernels: kSmemWide, or less if the device allows
-// less (the opt-in limit covers the kernel's static shared memory as well).
-int wide_budget()
-{
-    const int lim = smem_optin() - 1024 - 256 - 64;
-    return lim < kSmemWide ? lim : kSmemWide;
-}
-
-int stages_for(int stage_bytes, int budget = kSmemBudget)
-{
-    const int s = budget / stage_bytes;
-    return s > kMaxStages ? kMaxStages : s;
-}
-
-uint32_t tmem_cols_for(int cols)
-{
-    uint32_t c = 32;
-    while ((int)c < cols) c <<= 1;
-    return c;
-}
-
-int sm_count()
-{
-    static int by_dev[64] = {0};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    int &n = by_dev[dev & 63];
-    if (n == 0) cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    return n > 0 ? n : 1;
-}
-
-// Neurons per tile: the multiple of 16 (<= 128) that minimises waves x rows,
-// so that the neuron tiles cover the SMs in about one wave.
-int choose_rows(int N, int sms)
-{
-    int best = 16;
-    long long best_cost = -1;
-    for (int R = 16; R <= BM; R += 16) {
-        const long long tiles = (N + R - 1) / R;
-        const long long cost = ((tiles + sms - 1) / sms) * R;
-        if (best_cost < 0 || cost <= best_cost) {
-            best_cost = cost;
-            best = R;
-        }
-    }
-    return best;
-}
-
 }  // namespace
 }  // namespace tc
 
@@ -1104,8 +860,14 @@ cudaError_t tc_free_layer(sats_layer *l)
 }
 
 namespace {
+// The dynamic shared-memory limit set for gu_skinny_kernel on each device (both
+// of its modes raise it through this one record, so neither lowers it under the other).
+std::atomic<int> cfg_gu_skinny[64];
+
 struct TcLayout {
-    size_t xhi, xlo, hact, hact_lo, keep, total;
+    size_t xhi, xlo, hact, hact_lo, keep;
+    size_t a_keep, u, uflag, ulist, ucount;   // the union path (batches up to kMaxUnion)
+    size_t total;
 };
 
 TcLayout tc_layout(int H, int N, int B)
@@ -1124,6 +886,18 @@ TcLayout tc_layout(int H, int N, int B)
     off += al((size_t)B * ldn * 2);
     L.keep = off;
     off += al((size_t)B * (((size_t)N + 15) & ~(size_t)15));
+    if (B <= tc::kMaxUnion) {
+        L.a_keep = off;
+        off += al((size_t)B * ldn * 4);
+        L.u = off;
+        off += al((size_t)B * ldn * 4);
+        L.uflag = off;   // padded to 16 bytes (read as 16-byte vectors)
+        off += al(((size_t)N + 15) & ~(size_t)15);
+        L.ulist = off;
+        off += al((size_t)N * 4);
+        L.ucount = off;
+        off += al(4);
+    }
     L.total = off;
     return L;
 }
@@ -1139,7 +913,8 @@ size_t tc_workspace_bytes(int H, int N, int B) { return tc_layout(H, N, B).total
 //   out: y [B][H] (kOutY) or the residual (kOutResid, += y).
 cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int B, float t_l, const float *norm_w,
                          float eps, const uint8_t *dense_flags, int out_mode, float *out, int32_t *active_idx,
-                         int32_t *active_cnt, uint8_t *keep_trace, void *tc_ws, int *ctl, cudaStream_t stream)
+                         int32_t *active_cnt, uint8_t *keep_trace, void *tc_ws, int *ctl, cudaStream_t stream,
+                         bool union_path)
 {
     using namespace tc;
     auto fail = [](cudaError_t err, const char *where) {
@@ -1166,7 +941,54 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         if (e != cudaSuccess) return fail(e, "split kernel launch");
     }
 
-    if (B <= kMaxSkinny) {
+    if (union_path) {   // the caller has checked union_path_ok(H, B) and that no token is on the base path
+        // union path: gate on the tensor cores, then up and down for the union of the kept neurons
+        const int NT = (B + 15) & ~15;
+        CUtensorMap mX, mX2;
+        if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, NT) || !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, NT))
+            return fail(cudaErrorInvalidValue, "tensor map encoding");
+        float *a_keep = reinterpret_cast<float *>(base + W.a_keep);
+        float *u = reinterpret_cast<float *>(base + W.u);
+        uint8_t *uflag = base + W.uflag;
+        int32_t *ulist = reinterpret_cast<int32_t *>(base + W.ulist);
+        int32_t *ucount = reinterpret_cast<int32_t *>(base + W.ucount);
+        SkinnyGuParams gp{};
+        gp.w = layer->gu_blk;
+        gp.M = B;
+        gp.N = N;
+        gp.R = R;
+        gp.KBh = layer->tc_kbh;
+        gp.NT = NT;
+        gp.split = split ? 1 : 0;
+        gp.t_l = t_l;
+        gp.ldh = ldn;
+        gp.keep = active_idx ? keep : nullptr;
+        gp.keep_stride = kstride;
+        gp.keep_trace = keep_trace;
+        gp.ctl = ctl;
+        gp.zero = out_mode == kOutY ? out : nullptr;   // the down projection adds into y
+        gp.zero_count = B * H;
+        gp.gate_only = 1;
+        gp.a_keep = a_keep;
+        gp.uflag = uflag;
+        // stage: the gate rows, then the token tile(s); the gate MMA reads 128 rows from the
+        // stage start (rows R..127 of D are not used), so the ring ends with room for that read
+        gp.a_bytes = R * kTileBytes;
+        gp.x_bytes = NT * kTileBytes;
+        gp.stage_bytes = gp.a_bytes + gp.x_bytes * (split ? 2 : 1);
+        const int over = BM * kTileBytes - gp.stage_bytes;
+        const int slack = over > 0 ? ((over + 1023) & ~1023) : 0;
+        gp.stages = stages_for(gp.stage_bytes, kSmemBudget - slack);
+        gp.ring_bytes = gp.stages * gp.stage_bytes + slack;
+        gp.tmem_cols = tmem_cols_for(NT);
+        if ((e = set_smem(gu_skinny_kernel, smem_for(1, gp.ring_bytes), cfg_gu_skinny)) != cudaSuccess)
+            return fail(e, "shared-memory attribute");
+        e = launch_pdl(gu_skinny_kernel, dim3(layer->tc_T), smem_for(1, gp.ring_bytes), stream, mX, mX2, gp);
+        if (e != cudaSuccess) return fail(e, "gate kernel launch");
+        e = launch_union_tail(layer, B, xa, split ? xlo : nullptr, uflag, ulist, ucount, a_keep, ldn, u, ldn, out, ctl,
+                              stream);
+        if (e != cudaSuccess) return fail(e, "union kernels launch");
+    } else if (B <= kMaxSkinny) {
         const int NT = (B + 15) & ~15;
         CUtensorMap mX, mX2, mH, mH2;
         if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, NT) || !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, NT) ||
@@ -1202,8 +1024,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.stages = stages_for(gp.stage_bytes, kSmemBudget - slack);
         gp.ring_bytes = gp.stages * gp.stage_bytes + slack;
         gp.tmem_cols = tmem_cols_for(2 * NT);
-        static std::atomic<int> cfg_gu[64];
-        if ((e = set_smem(gu_skinny_kernel, smem_for(1, gp.ring_bytes), cfg_gu)) != cudaSuccess)
+        if ((e = set_smem(gu_skinny_kernel, smem_for(1, gp.ring_bytes), cfg_gu_skinny)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
         e = launch_pdl(gu_skinny_kernel, dim3(layer->tc_T), smem_for(1, gp.ring_bytes), stream, mX, mX2, gp);
         if (e != cudaSuccess) return fail(e, "gate/up kernel launch");

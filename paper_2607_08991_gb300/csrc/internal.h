@@ -100,9 +100,16 @@ cudaError_t tc_pack_layer(sats_layer *layer, cudaStream_t stream);
 cudaError_t tc_free_layer(sats_layer *layer);
 bool use_tc_path(int H, int B);
 size_t tc_workspace_bytes(int H, int N, int B);
+// union_mlp.cu: whether a batch may take the union path (B <= 8 sparse-path
+// tokens, H <= 4096), and its list, up and down kernels after the gate-only kernel.
+bool union_path_ok(int H, int B);
+cudaError_t launch_union_tail(const sats_layer *layer, int B, const uint16_t *xa, const uint16_t *xlo,
+                              const uint8_t *uflag, int32_t *ulist, int32_t *ucount, const float *a_keep, int lda,
+                              float *u, int ldu, float *out, int *ctl, cudaStream_t stream);
 cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int B, float t_l, const float *norm_w,
                          float eps, const uint8_t *dense_flags, int out_mode, float *out, int32_t *active_idx,
-                         int32_t *active_cnt, uint8_t *keep_trace, void *tc_ws, int *ctl, cudaStream_t stream);
+                         int32_t *active_cnt, uint8_t *keep_trace, void *tc_ws, int *ctl, cudaStream_t stream,
+                         bool union_path = false);
 cudaError_t launch_route(const int32_t *ids, int B, const uint8_t *lut, int V, int32_t *perm,
                          int32_t *n_dense, uint8_t *flags, int32_t *status, cudaStream_t stream);
 cudaError_t launch_gate_act(const sats_layer *layer, const uint16_t *x, int B, float *a,

@@ -52,6 +52,8 @@ def lib() -> ctypes.CDLL:
             "sats_sparse_mlp": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_sparse_mlp_f32": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_sparse_mlp_fixed_scratch": (I, [P, P, I, F, P, P, P, P]),
+            "sats_sparse_mlp_union": (I, [P, P, I, F, P, P, P, P, Z, P]),
+            "sats_sparse_mlp_union_f32": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_uses_tensor_cores": (I, [I, I]),
             "sats_last_cuda_error": (ctypes.c_char_p, []),
             "sats_dense_mlp": (I, [P, P, I, P, P, Z, P]),
@@ -85,7 +87,9 @@ def exported_symbols() -> Sequence[str]:
     """Every C entry point this binding forwards to."""
     return ("sats_version", "sats_status_string", "sats_layer_create", "sats_layer_destroy", "sats_layer_shape",
             "sats_workspace_bytes", "sats_workspace_init", "sats_sparse_mlp", "sats_sparse_mlp_f32",
-            "sats_sparse_mlp_fixed_scratch", "sats_uses_tensor_cores", "sats_last_cuda_error", "sats_dense_mlp", "sats_route", "sats_mlp_stack", "sats_gate_act",
+            "sats_sparse_mlp_fixed_scratch", "sats_sparse_mlp_union", "sats_sparse_mlp_union_f32",
+            "sats_uses_tensor_cores", "sats_last_cuda_error", "sats_dense_mlp", "sats_route", "sats_mlp_stack",
+            "sats_gate_act",
             "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_rmsnorm", "sats_gate_act_f32",
             "sats_layer_err_workspace_bytes", "sats_layer_err", "sats_sats_select", "sats_sats_workspace_bytes",
             "sats_sats_calibrate", "sats_route_calib_workspace_bytes", "sats_token_scores", "sats_route_calibrate",
@@ -182,10 +186,25 @@ def sparse_mlp_f32(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor, w
                                      ws.ptr, ws.nbytes, _stream(stream)), "sats_sparse_mlp_f32")
 
 
+def sparse_mlp_union(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor, ws: Workspace,
+                     active_idx: Optional[torch.Tensor] = None, active_cnt: Optional[torch.Tensor] = None,
+                     stream: Optional[torch.cuda.Stream] = None):
+    """sats_sparse_mlp over the union of the batch's kept neurons (x bf16 or fp32; 3 <= B <= 8)."""
+    B = x.shape[0]
+    if x.dtype == torch.float32:
+        _check(lib().sats_sparse_mlp_union_f32(layer.handle, _ptr(x, "x", 4), B, float(t_l), _ptr(y, "y", 4),
+                                               _ptr(active_idx, "active_idx", 4), _ptr(active_cnt, "active_cnt", 4),
+                                               ws.ptr, ws.nbytes, _stream(stream)), "sats_sparse_mlp_union_f32")
+    else:
+        _check(lib().sats_sparse_mlp_union(layer.handle, _ptr(x, "x", 2), B, float(t_l), _ptr(y, "y", 4),
+                                           _ptr(active_idx, "active_idx", 4), _ptr(active_cnt, "active_cnt", 4),
+                                           ws.ptr, ws.nbytes, _stream(stream)), "sats_sparse_mlp_union")
+
+
 def sparse_mlp_fixed_scratch(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor,
                              active_idx: Optional[torch.Tensor] = None, active_cnt: Optional[torch.Tensor] = None,
                              stream: Optional[torch.cuda.Stream] = None):
-    """sats_sparse_mlp without a workspace (the library's fixed 1 MiB device scratch)."""
+    """sats_sparse_mlp without a workspace (the library's fixed 256 KiB device scratch)."""
     B = x.shape[0]
     _check(lib().sats_sparse_mlp_fixed_scratch(layer.handle, _ptr(x, "x", 2), B, float(t_l), _ptr(y, "y", 4),
                                                _ptr(active_idx, "active_idx", 4), _ptr(active_cnt, "active_cnt", 4),
