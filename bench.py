@@ -623,6 +623,55 @@ def run_workload(args):
             clk = clocks.stop()
             out.update({"metric": "us per prefill call (one routed block)", "value": res["0.6@2048"]["us_per_call"],
                         "unit": "us/call", "per_case": res, "clocks": clk})
+        elif wl == "union_batch_llama_4096x14336":
+            # the union path (sats_sparse_mlp_union) against the default batched path on
+            # the same calls: independent tokens (rho = 0) and strongly correlated ones
+            H, N = spec["H"], spec["N"]
+            layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l)) for l in range(LAYER_COPIES)]
+            xc = torch.from_numpy(inputs.activations_bf16(spec["calib"], H, seed=inputs.SEED_CALIB).view(np.int16)).to(dev)
+            a = torch.empty(spec["calib"], N, dtype=torch.float32, device=dev)
+            sats.gate_act(layers[0], xc, a, stream=stream)
+            sel = torch.empty(sats.select_workspace_bytes(), dtype=torch.uint8, device=dev)
+            ts = {k: sats.percentile_threshold(a, k, sel, stream=stream) for k in spec["sparsity"]}
+            del a
+            res = {}
+            clocks.start()
+            for rho in spec["rho"]:
+                for B in spec["batches"]:
+                    ws = sats.Workspace(H, N, B, device=dev)
+                    xb = (inputs.activations_bf16(B, H, seed=inputs.SEED_X + B) if rho == 0.0 else
+                          inputs.activations_correlated_bf16(B, H, rho, seed=inputs.SEED_X + B))
+                    x = torch.from_numpy(xb.view(np.int16)).to(dev)
+                    y = torch.empty(B, H, dtype=torch.float32, device=dev)
+                    idx = torch.empty(B, N, dtype=torch.int32, device=dev)
+                    cnt = torch.empty(B, dtype=torch.int32, device=dev)
+                    for k, t in ts.items():
+                        sats.sparse_mlp_union(layers[0], x, t, y, ws, idx, cnt, stream=stream)
+                        stream.synchronize()
+                        c = cnt.cpu().numpy()
+                        keep = np.zeros((B, N), bool)
+                        ii = idx.cpu().numpy()
+                        for m in range(B):
+                            keep[m, ii[m, :c[m]]] = True
+                        U = int(keep.any(axis=0).sum())
+                        runs = {}
+                        for name, fn in (("union", sats.sparse_mlp_union), ("default", sats.sparse_mlp)):
+                            call = lambda i, fn=fn: fn(layers[i % LAYER_COPIES], x, t, y, ws, stream=stream)
+                            for i in range(args.warmup + 3):
+                                call(i)
+                            runs[name] = _timed(stream, call, max(args.steps // 4, 20))
+                        algo_union = 2.0 * H * N + 4.0 * H * U + 2.0 * B * H + 4.0 * B * H
+                        res["rho%.1f_B%d_s%.1f" % (rho, B, k)] = {
+                            "union_fraction": U / N, "mean_sparsity": 1.0 - float(c.mean()) / N,
+                            "us_union": runs["union"], "us_default": runs["default"],
+                            "union_bytes": algo_union, "union_gbs": algo_union / runs["union"] / 1e3,
+                            "default_gbs_all_weights": 6.0 * H * N / runs["default"] / 1e3}
+                    del ws
+            clk = clocks.stop()
+            out.update({"metric": "us per call, union path vs default batched path", "unit": "us/call",
+                        "value": min(v["us_union"] for v in res.values()), "per_case": res,
+                        "input": "x ~ N(0,1) per token (rho 0) or rho z_0 + sqrt(1-rho^2) z_m (rho 0.9), bf16",
+                        "clocks": clk})
         elif wl == "sats_calibration_llama_32x4096x14336":
             H, N, L, C = spec["H"], spec["N"], spec["L"], spec["calib"]
             layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l)) for l in range(L)]

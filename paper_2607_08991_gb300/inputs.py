@@ -117,6 +117,16 @@ def activations_bf16(B: int, H: int, seed: int = SEED_X) -> np.ndarray:
     return normal_bf16((B, H), 1.0, seed)
 
 
+def activations_correlated_bf16(B: int, H: int, rho: float, seed: int = SEED_X) -> np.ndarray:
+    """x_m = rho z_0 + sqrt(1 - rho^2) z_m with z ~ N(0, 1) i.i.d. (so every x_m is
+    N(0, 1) and any two tokens correlate with coefficient rho^2 elementwise),
+    rounded to bf16: [B][H] uint16 bit patterns.  A stand-in for batches whose
+    tokens share most of their kept neurons."""
+    z = _rng(seed, 2).standard_normal(size=(B + 1, H))
+    x = rho * z[0] + np.sqrt(1.0 - rho * rho) * z[1:]
+    return to_bf16_bits(x.astype(np.float32))
+
+
 def activations_f32(B: int, H: int, seed: int = SEED_X) -> np.ndarray:
     return _rng(seed, 1).standard_normal(size=(B, H), dtype=np.float32)
 
@@ -178,6 +188,9 @@ WORKLOADS: Dict[str, dict] = {
     # routing calibration (Sec. 3.2) over the Qwen3-8B-shaped vocabulary
     "route_calibration_qwen_v151936": dict(V=QWEN_V, corpus=4_000_000, heldout=1_000_000,
                                            targets=[0.25, 0.5, 0.75]),
+    # batched decode on the union of the kept neurons, independent and correlated tokens
+    "union_batch_llama_4096x14336": dict(H=LLAMA_H, N=LLAMA_N, batches=[3, 4, 8], sparsity=[0.7, 0.9],
+                                         rho=[0.0, 0.9], calib=256),
     # SATS calibration (Sec. 3.1) of the 32-block Llama-shaped stack
     "sats_calibration_llama_32x4096x14336": dict(H=LLAMA_H, N=LLAMA_N, L=LLAMA_L, calib=64, K0=20, K1=8,
                                                   target=0.5, eps=1e-5),
