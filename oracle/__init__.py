@@ -61,6 +61,8 @@ def _load():
         lib.oracle_masked_mlp.argtypes = [I, I, I, P, P, P, P, P, P]
         lib.oracle_sparse_mlp.argtypes = [I, I, I, P, P, P, P, P, P, D, P, P, P]
         lib.oracle_sparse_mlp.restype = I64
+        lib.oracle_sparse_mlp_lora.argtypes = [I, I, I, I, P, P, P, P, P, P, P, P, P, P, D, P, P, D, P, P, P]
+        lib.oracle_sparse_mlp_lora.restype = I64
         lib.oracle_dense_mlp.argtypes = [I, I, I, P, P, P, P, P]
         lib.oracle_percentile_threshold.argtypes = [P, I64, D]
         lib.oracle_percentile_threshold.restype = D
@@ -164,6 +166,30 @@ def sparse_mlp(x, Wg, Wu, Wd, t, keep_hint=None, band_rel: float = 0.0):
     keep = np.empty((B, N), dtype=np.uint8)
     nb = _load().oracle_sparse_mlp(B, H, N, _ptr(x), _ptr(Wg), _ptr(Wu), _ptr(Wd), _ptr(tt),
                                    _ptr(hint), float(band_rel), _ptr(y), _ptr(a), _ptr(keep))
+    return y, a, keep, int(nb)
+
+
+def sparse_mlp_lora(x, Wg, Wu, Wd, lora, scale: float, t, keep_hint=None, band_rel: float = 0.0):
+    """Sec. 4 (fine-tuned routing): the sparse path on LoRA-adapted projections
+    W + scale A B, the low-rank terms applied factor by factor (Sec. 2, Eqs. 1-5
+    otherwise).  lora = (Ag [H][r], Bg [r][N], Au [H][r], Bu [r][N], Ad [N][r],
+    Bd [r][H]) as bf16 bit patterns.  Returns (y, a, keep, in_band) as sparse_mlp."""
+    x = _f64(x)
+    Wg, Wu, Wd = _u16(Wg), _u16(Wu), _u16(Wd)
+    Ag, Bg, Au, Bu, Ad, Bd = (_u16(m) for m in lora)
+    B, H = x.shape
+    N = Wg.shape[1]
+    r = Ag.shape[1]
+    assert Ag.shape == (H, r) and Au.shape == (H, r) and Bg.shape == (r, N) and Bu.shape == (r, N)
+    assert Ad.shape == (N, r) and Bd.shape == (r, H)
+    tt = _f64(np.broadcast_to(np.asarray(t, dtype=np.float64), (B,)))
+    hint = None if keep_hint is None else np.ascontiguousarray(keep_hint, dtype=np.uint8)
+    y = np.empty((B, H), dtype=np.float64)
+    a = np.empty((B, N), dtype=np.float64)
+    keep = np.empty((B, N), dtype=np.uint8)
+    nb = _load().oracle_sparse_mlp_lora(B, H, N, r, _ptr(x), _ptr(Wg), _ptr(Wu), _ptr(Wd), _ptr(Ag), _ptr(Bg),
+                                        _ptr(Au), _ptr(Bu), _ptr(Ad), _ptr(Bd), float(scale), _ptr(tt),
+                                        _ptr(hint), float(band_rel), _ptr(y), _ptr(a), _ptr(keep))
     return y, a, keep, int(nb)
 
 

@@ -27,6 +27,9 @@
  *   oracle_layer_err          Sec. 3.1, Eq. 6  Err_l(t) and the sparsity sp_l(t)
  *                             of one block at candidate thresholds
  *   oracle_sats_select        Sec. 3.1, Eqs. 7-10 t*_l(b), T*(b), S(b), b*
+ *   oracle_sparse_mlp_lora    Sec. 4 (fine-tuned routing): the sparse path on
+ *                             LoRA-adapted weights W + scale A B, the low-rank
+ *                             terms applied without forming W + scale A B
  *
  * Layouts follow the paper's row-vector convention x W: W_gate and W_up are
  * [H][N] (hidden x intermediate), W_down is [N][H], all row-major bf16 bit
@@ -156,6 +159,76 @@ int64_t oracle_sparse_mlp(int B, int H, int N, const double *x, const uint16_t *
     if (keep_out) memcpy(keep_out, keep, (size_t)B * N);
     free(a);
     free(keep);
+    return in_band;
+}
+
+/* Sec. 4, fine-tuned models: the sparse path runs the thresholded MLP of Sec. 2
+ * (Eqs. 1-5) on LoRA-adapted projections W + scale A B (A: [in][r], B: [r][out]),
+ * with the low-rank products taken factor by factor:
+ *   g = x W_gate + scale (x A_g) B_g,   a = SiLU(g),   keep = |a| >= t  (Eqs. 1-5)
+ *   u = x W_up   + scale (x A_u) B_u,   h = keep ? a u : 0
+ *   y = h W_down + scale (h A_d) B_d
+ * A_g, A_u [H][r]; B_g, B_u [r][N]; A_d [N][r]; B_d [r][H]; bf16 bit patterns.
+ * keep_hint / band_rel as for oracle_sparse_mlp.  Returns the in-band count. */
+int64_t oracle_sparse_mlp_lora(int B, int H, int N, int r, const double *x, const uint16_t *Wg,
+                               const uint16_t *Wu, const uint16_t *Wd, const uint16_t *Ag,
+                               const uint16_t *Bg, const uint16_t *Au, const uint16_t *Bu,
+                               const uint16_t *Ad, const uint16_t *Bd, double scale, const double *t,
+                               const uint8_t *keep_hint, double band_rel,
+                               double *y, double *a_out, uint8_t *keep_out)
+{
+    double *a = (double *)malloc(sizeof(double) * (size_t)B * N);
+    double *u = (double *)malloc(sizeof(double) * (size_t)B * N);
+    uint8_t *keep = (uint8_t *)malloc((size_t)B * N);
+    double *zg = (double *)malloc(sizeof(double) * (size_t)r);
+    double *zu = (double *)malloc(sizeof(double) * (size_t)r);
+    double *w = (double *)malloc(sizeof(double) * (size_t)r);
+    for (int b = 0; b < B; ++b) {
+        const double *xb = x + (size_t)b * H;
+        for (int q = 0; q < r; ++q) {   /* x A_g, x A_u */
+            zg[q] = 0.0;
+            zu[q] = 0.0;
+            for (int k = 0; k < H; ++k) {
+                zg[q] += xb[k] * bf16_value(Ag[(size_t)k * r + q]);
+                zu[q] += xb[k] * bf16_value(Au[(size_t)k * r + q]);
+            }
+        }
+        for (int j = 0; j < N; ++j) {
+            double g = 0.0, v = 0.0, lg = 0.0, lu = 0.0;
+            for (int k = 0; k < H; ++k) {
+                g += xb[k] * bf16_value(Wg[(size_t)k * N + j]);
+                v += xb[k] * bf16_value(Wu[(size_t)k * N + j]);
+            }
+            for (int q = 0; q < r; ++q) {
+                lg += zg[q] * bf16_value(Bg[(size_t)q * N + j]);
+                lu += zu[q] * bf16_value(Bu[(size_t)q * N + j]);
+            }
+            a[(size_t)b * N + j] = oracle_silu(g + scale * lg);
+            u[(size_t)b * N + j] = v + scale * lu;
+        }
+    }
+    const int64_t in_band = oracle_cats_mask(B, N, a, t, keep_hint, band_rel, keep);
+    for (int b = 0; b < B; ++b) {
+        double *yb = y + (size_t)b * H;
+        for (int i = 0; i < H; ++i) yb[i] = 0.0;
+        for (int q = 0; q < r; ++q) w[q] = 0.0;
+        for (int j = 0; j < N; ++j) {
+            const size_t bj = (size_t)b * N + j;
+            const double h = keep[bj] ? a[bj] * u[bj] : 0.0;
+            for (int i = 0; i < H; ++i) yb[i] += h * bf16_value(Wd[(size_t)j * H + i]);
+            for (int q = 0; q < r; ++q) w[q] += h * bf16_value(Ad[(size_t)j * r + q]);   /* h A_d */
+        }
+        for (int q = 0; q < r; ++q)
+            for (int i = 0; i < H; ++i) yb[i] += scale * w[q] * bf16_value(Bd[(size_t)q * H + i]);
+    }
+    if (a_out) memcpy(a_out, a, sizeof(double) * (size_t)B * N);
+    if (keep_out) memcpy(keep_out, keep, (size_t)B * N);
+    free(a);
+    free(u);
+    free(keep);
+    free(zg);
+    free(zu);
+    free(w);
     return in_band;
 }
 

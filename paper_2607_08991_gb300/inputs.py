@@ -112,6 +112,17 @@ def mlp_weights_device(H: int, N: int, layer: int = 0, std: float = 0.02, seed: 
             device_normal_bf16((N, H), std, seed + layer, 12, device=device))
 
 
+def lora_adapter(H: int, N: int, r: int, std_a: float = 0.02, std_b: float = 0.02, seed: int = 7000,
+                 layer: int = 0):
+    """A synthetic LoRA adapter of rank r for one MLP block (the trained adapters are not
+    available): (Ag [H][r], Bg [r][N], Au [H][r], Bu [r][N], Ad [N][r], Bd [r][H]), every
+    factor N(0, std) rounded to bf16 (bit patterns).  Unlike LoRA's zero-initialised B,
+    both factors are non-zero so that every low-rank term is exercised."""
+    return (normal_bf16((H, r), std_a, seed + layer, 20), normal_bf16((r, N), std_b, seed + layer, 21),
+            normal_bf16((H, r), std_a, seed + layer, 22), normal_bf16((r, N), std_b, seed + layer, 23),
+            normal_bf16((N, r), std_a, seed + layer, 24), normal_bf16((r, H), std_b, seed + layer, 25))
+
+
 def activations_bf16(B: int, H: int, seed: int = SEED_X) -> np.ndarray:
     """x ~ N(0, 1) rounded to bf16: [B][H] uint16 bit patterns."""
     return normal_bf16((B, H), 1.0, seed)
