@@ -57,6 +57,7 @@ typedef enum {
 
 /* Opaque handle of one MLP block; owns its repacked device weights. */
 typedef struct sats_layer sats_layer;
+typedef struct sats_lora sats_lora;
 
 /* Library version, (major << 16) | minor. */
 SATS_API int sats_version(void);
@@ -88,9 +89,10 @@ SATS_API sats_status sats_layer_shape(const sats_layer *layer, int *H, int *N);
 /*
  * Workspace.  Every compute call takes a device workspace `ws` of at least
  * sats_workspace_bytes(H, N, B) bytes (B = the largest batch the caller will
- * pass).  It holds scheduling counters, the device status word, one 64-bit
- * word per 8 neurons (kept counts and prefixes for the index outputs) and the
- * routing scratch of sats_mlp_stack: N bytes plus B * 5 plus 1 KB.  A batch that runs on the
+ * pass).  It holds scheduling counters, the device status word, the LoRA
+ * path's partial sums (16 KB), one 64-bit word per 8 neurons (kept counts and
+ * prefixes for the index outputs) and the routing scratch of sats_mlp_stack:
+ * N bytes plus B * 5 plus about 19 KB.  A batch that runs on the
  * tensor cores (sats_uses_tensor_cores) also needs, per token, bf16 copies of
  * its activations and of h (two parts each) plus one keep byte per neuron:
  * about B * (4 H + 5 N) bytes more.  It must be
@@ -142,7 +144,7 @@ SATS_API sats_status sats_sparse_mlp(const sats_layer *layer, const void *x, int
  * every GPU that loads the library holds this array until the process exits.
  * A shape whose workspace (sats_workspace_bytes(H, N, B)) exceeds 256 KiB is
  * rejected with SATS_ENOSPACE; with one 64-bit word per 8 neurons that admits
- * N up to about 259,000 for B <= 2.  The call allocates nothing: before its
+ * N up to about 243,000 for B <= 2.  The call allocates nothing: before its
  * kernel it clears the array's control words with cudaMemsetAsync on `stream`.
  *
  * The first call on each device looks up the array's device address
@@ -197,6 +199,37 @@ SATS_API sats_status sats_sparse_mlp_union(const sats_layer *layer, const void *
 SATS_API sats_status sats_sparse_mlp_union_f32(const sats_layer *layer, const float *x, int B, float t_l,
                                                float *y, int32_t *active_idx, int32_t *active_cnt, void *ws,
                                                size_t ws_bytes, void *stream);
+
+/*
+ * LoRA-aware sparse path (Sec. 4, fine-tuned models: the sparse path of a routed
+ * fine-tuned model runs the thresholded MLP on its adapted weights, with the
+ * low-rank updates folded into the sparse kernel).  An adapter of rank r holds,
+ * for each projection W of the block, factors A, B with W' = W + scale A B:
+ *   A_gate, A_up [H][r], B_gate, B_up [r][N], A_down [N][r], B_down [r][H]
+ * (device bf16, row-major; the adapter keeps its own packed copies, so the
+ * caller may free them after sats_lora_create returns).  r is 8, 16, 24 or 32
+ * (else SATS_ESHAPE); scale finite (else SATS_EINVAL).
+ *
+ * sats_sparse_mlp_lora computes, for each of B tokens,
+ *   g = x W_gate + scale (x A_gate) B_gate,  a = SiLU(g),  keep = |a| >= t_l
+ *   u = x W_up + scale (x A_up) B_up,        h = keep ? a u : 0
+ *   y = h W_down + scale (h A_down) B_down
+ * in the decode kernel: the gate's low-rank term for every neuron, the up and
+ * down terms only for kept neurons; batches run as passes of that kernel.
+ * Arguments, index outputs, workspace and errors are those of sats_sparse_mlp
+ * (x bf16) and sats_sparse_mlp_f32 (x fp32); the adapter must match the
+ * layer's H and N (else SATS_ESHAPE).
+ */
+SATS_API sats_status sats_lora_create(const sats_layer *layer, const void *A_gate, const void *B_gate,
+                                      const void *A_up, const void *B_up, const void *A_down, const void *B_down,
+                                      int r, float scale, void *stream, sats_lora **out);
+SATS_API sats_status sats_lora_destroy(sats_lora *lora);
+SATS_API sats_status sats_sparse_mlp_lora(const sats_layer *layer, const sats_lora *lora, const void *x, int B,
+                                          float t_l, float *y, int32_t *active_idx, int32_t *active_cnt, void *ws,
+                                          size_t ws_bytes, void *stream);
+SATS_API sats_status sats_sparse_mlp_lora_f32(const sats_layer *layer, const sats_lora *lora, const float *x, int B,
+                                              float t_l, float *y, int32_t *active_idx, int32_t *active_cnt,
+                                              void *ws, size_t ws_bytes, void *stream);
 
 /*
  * sats_dense_mlp -- the base gated MLP of Sec. 2, Eq. 1 (every neuron kept):

@@ -22,6 +22,8 @@ WsLayout ws_layout(int H, int N, int B)
     size_t off = 0;
     L.ctl = off;
     off += align256(kCtlInts * sizeof(int));
+    L.lora_z = off;   // cleared with the control words; the fused kernel's last CTA clears it after a LoRA call
+    off += align256((size_t)kLoraZCopies * kMaxTokensPerPass * 2 * kMaxLoraRank * sizeof(float));
     L.flags = off;   // one 64-bit word per chunk of kChunk neurons, then one per CTA of the fused grid
     off += align256(((size_t)nchunks_of(N) + kMaxGrid) * sizeof(uint64_t));
     L.route_perm = off;
@@ -38,7 +40,7 @@ static bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 
 
 cudaError_t clear_fused_state(void *ws, int H, int N, int B, cudaStream_t stream)
 {
-    // the fused kernel clears the chunk flags itself; its counters must start at zero
+    // the fused kernel clears the chunk flags itself; its counters (and the LoRA sums) must start at zero
     return cudaMemsetAsync(ws, 0, ws_layout(H, N, B).flags, stream);
 }
 
@@ -65,12 +67,13 @@ static bool bad_threshold(float t) { return std::isnan(t) || t < 0.0f; }
 // fused_tokens_per_pass(H) tokens.
 sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B, const float *t_per_pass_l,
                       const float *norm_w, float eps, const uint8_t *dense_flags, int out_mode, float *out,
-                      int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws, cudaStream_t stream)
+                      int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws, cudaStream_t stream,
+                      const sats_lora *lora)
 {
     const int H = layer->H, N = layer->N;
     const WsLayout L = ws_layout(H, N, B);
     char *base = static_cast<char *>(ws);
-    if (use_tc_path(H, B)) {
+    if (!lora && use_tc_path(H, B)) {   // the LoRA variant runs in passes of the fused kernel at any batch
         const cudaError_t e = run_tc_layer(layer, x_mode, x, B, *t_per_pass_l, norm_w, eps, dense_flags, out_mode,
                                            out, active_idx, active_cnt, keep_trace, base + L.tc,
                                            reinterpret_cast<int *>(base + L.ctl), stream);
@@ -99,6 +102,15 @@ sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B,
         p.active_idx = active_idx ? active_idx + (size_t)b0 * N : nullptr;
         p.active_cnt = active_cnt ? active_cnt + b0 : nullptr;
         p.keep_trace = keep_trace ? keep_trace + (size_t)b0 * N : nullptr;
+        if (lora) {
+            p.lora = lora;
+            p.lora_blk = lora->blk;
+            p.lora_agu = lora->agu;
+            p.lora_bd = lora->bd;
+            p.lora_r = lora->r;
+            p.lora_scale = lora->scale;
+            p.lora_z = reinterpret_cast<float *>(base + L.lora_z);
+        }
         const cudaError_t e = launch_fused(p, stream);
         if (e != cudaSuccess) return cuda_fail(e, "fused kernel launch");
     }
@@ -218,6 +230,87 @@ sats_status sats_layer_destroy(sats_layer *layer)
     if (e1 != cudaSuccess) return cuda_fail(e1, "cudaFree");
     if (e2 != cudaSuccess) return cuda_fail(e2, "cudaFree");
     return from_cuda(e3, "cudaFree");
+}
+
+sats_status sats_lora_create(const sats_layer *layer, const void *A_gate, const void *B_gate, const void *A_up,
+                             const void *B_up, const void *A_down, const void *B_down, int r, float scale,
+                             void *stream, sats_lora **out)
+{
+    if (!out) return SATS_EINVAL;
+    *out = nullptr;
+    if (!layer || !A_gate || !B_gate || !A_up || !B_up || !A_down || !B_down || !std::isfinite(scale))
+        return SATS_EINVAL;
+    if (r < 8 || r > kMaxLoraRank || (r % 8) != 0) return SATS_ESHAPE;
+    sats_lora *l = new (std::nothrow) sats_lora();
+    if (!l) return cuda_fail(cudaErrorMemoryAllocation, "host allocation");
+    l->H = layer->H;
+    l->N = layer->N;
+    l->r = r;
+    l->scale = scale;
+    cudaGetDevice(&l->device);
+    const size_t nblk = (size_t)nchunks_of(l->N) * kChunk * 3 * r;
+    cudaError_t e = cudaMalloc(&l->blk, nblk * 2);
+    if (e == cudaSuccess) e = cudaMalloc(&l->agu, (size_t)l->H * 2 * r * 2);
+    if (e == cudaSuccess) e = cudaMalloc(&l->bd, (size_t)r * l->H * 2);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (e == cudaSuccess)
+        e = launch_pack_lora(static_cast<const uint16_t *>(A_gate), static_cast<const uint16_t *>(B_gate),
+                             static_cast<const uint16_t *>(A_up), static_cast<const uint16_t *>(B_up),
+                             static_cast<const uint16_t *>(A_down), static_cast<const uint16_t *>(B_down), l->H, l->N,
+                             r, l, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) {
+        cudaFree(l->blk);
+        cudaFree(l->agu);
+        cudaFree(l->bd);
+        delete l;
+        return cuda_fail(e, "adapter allocation or repacking");
+    }
+    *out = l;
+    return SATS_OK;
+}
+
+sats_status sats_lora_destroy(sats_lora *lora)
+{
+    if (!lora) return SATS_EINVAL;
+    cudaDeviceSynchronize();
+    const cudaError_t e1 = cudaFree(lora->blk);
+    const cudaError_t e2 = cudaFree(lora->agu);
+    const cudaError_t e3 = cudaFree(lora->bd);
+    delete lora;
+    if (e1 != cudaSuccess) return cuda_fail(e1, "cudaFree");
+    if (e2 != cudaSuccess) return cuda_fail(e2, "cudaFree");
+    return from_cuda(e3, "cudaFree");
+}
+
+static sats_status lora_common(const sats_layer *layer, const sats_lora *lora, int x_mode, const void *x, int B,
+                               float t_l, float *y, int32_t *active_idx, int32_t *active_cnt, void *ws,
+                               size_t ws_bytes, void *stream)
+{
+    sats_status s = check_layer(layer, ws, ws_bytes, B);
+    if (s != SATS_OK) return s;
+    if (!lora) return SATS_EINVAL;
+    if (lora->H != layer->H || lora->N != layer->N) return SATS_ESHAPE;
+    if (bad_threshold(t_l)) return SATS_EINVAL;
+    if ((active_idx == nullptr) != (active_cnt == nullptr)) return SATS_EINVAL;
+    if (B == 0) return SATS_OK;
+    if (!x || !y || !aligned16(x) || !aligned16(y)) return SATS_EINVAL;
+    return run_layer(layer, x_mode, x, B, &t_l, nullptr, 0.f, nullptr, kOutY, y, active_idx, active_cnt, nullptr, ws,
+                     static_cast<cudaStream_t>(stream), lora);
+}
+
+sats_status sats_sparse_mlp_lora(const sats_layer *layer, const sats_lora *lora, const void *x, int B, float t_l,
+                                 float *y, int32_t *active_idx, int32_t *active_cnt, void *ws, size_t ws_bytes,
+                                 void *stream)
+{
+    return lora_common(layer, lora, kXBf16, x, B, t_l, y, active_idx, active_cnt, ws, ws_bytes, stream);
+}
+
+sats_status sats_sparse_mlp_lora_f32(const sats_layer *layer, const sats_lora *lora, const float *x, int B,
+                                     float t_l, float *y, int32_t *active_idx, int32_t *active_cnt, void *ws,
+                                     size_t ws_bytes, void *stream)
+{
+    return lora_common(layer, lora, kXF32, x, B, t_l, y, active_idx, active_cnt, ws, ws_bytes, stream);
 }
 
 sats_status sats_layer_shape(const sats_layer *layer, int *H, int *N)

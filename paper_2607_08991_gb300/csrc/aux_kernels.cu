@@ -234,6 +234,42 @@ cudaError_t launch_pack(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *
     return cudaGetLastError();
 }
 
+// LoRA adapter layout of the fused kernel (one element per thread, grid-stride):
+//   blk [ceil(N/8)][8][3r]: neuron j = 8c + i holds B_gate[:, j], B_up[:, j], A_down[j, :]
+//   (neurons past N are zero); agu [H][2r]: A_gate[h, :], A_up[h, :]; bd = B_down [r][H].
+__global__ void pack_lora_kernel(const uint16_t *__restrict__ Ag, const uint16_t *__restrict__ Bg,
+                                 const uint16_t *__restrict__ Au, const uint16_t *__restrict__ Bu,
+                                 const uint16_t *__restrict__ Ad, const uint16_t *__restrict__ Bd, int H, int N, int r,
+                                 uint16_t *__restrict__ blk, uint16_t *__restrict__ agu, uint16_t *__restrict__ bd)
+{
+    const size_t nblk = (size_t)((N + 7) / 8) * 8 * 3 * r, nagu = (size_t)H * 2 * r, nbd = (size_t)r * H;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < nblk + nagu + nbd;
+         i += (size_t)gridDim.x * blockDim.x) {
+        if (i < nblk) {
+            const int j = (int)(i / (3 * r)), e = (int)(i % (3 * r));
+            const int part = e / r, q = e % r;
+            uint16_t v = 0;
+            if (j < N) v = part == 0 ? Bg[(size_t)q * N + j] : (part == 1 ? Bu[(size_t)q * N + j] : Ad[(size_t)j * r + q]);
+            blk[i] = v;
+        } else if (i < nblk + nagu) {
+            const size_t k = i - nblk;
+            const int h = (int)(k / (2 * r)), e = (int)(k % (2 * r));
+            agu[k] = e < r ? Ag[(size_t)h * r + e] : Au[(size_t)h * r + (e - r)];
+        } else {
+            const size_t k = i - nblk - nagu;
+            bd[k] = Bd[k];
+        }
+    }
+}
+
+cudaError_t launch_pack_lora(const uint16_t *Ag, const uint16_t *Bg, const uint16_t *Au, const uint16_t *Bu,
+                             const uint16_t *Ad, const uint16_t *Bd, int H, int N, int r, sats_lora *l,
+                             cudaStream_t stream)
+{
+    pack_lora_kernel<<<1024, 256, 0, stream>>>(Ag, Bg, Au, Bu, Ad, Bd, H, N, r, l->blk, l->agu, l->bd);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_route(const int32_t *ids, int B, const uint8_t *lut, int V, int32_t *perm, int32_t *n_dense,
                          uint8_t *flags, int32_t *status, cudaStream_t stream)
 {

@@ -135,10 +135,31 @@ struct Shared {
     int quiet;                  // roles past their last use of the counters (list producer, index warp)
 };
 
+// Extra shared state of the LoRA variant (Sec. 4, fine-tuned sparse path), placed
+// after Shared<BT>, 128-byte aligned.
 template <int BT>
+struct LoraShared {
+    uint16_t blk[kBufs][kChunk * 3 * kMaxLoraRank];        // the chunk's B_gate, B_up columns, A_down rows (pitch 3r)
+    float z[BT][2 * kMaxLoraRank];                         // x A_gate, x A_up summed over every CTA
+    float lu[kUdSlots][kMaxUdRows][BT];                    // scale (x A_up) B_up[:, j] of each W_ud row
+    uint32_t ad[kUdSlots][kMaxUdRows][kMaxLoraRank / 2];   // A_down[j, :] of each W_ud row, bf16 pairs
+    float w[BT][kMaxLoraRank];                             // this CTA's sum of h_j A_down[j, :]
+    float zred[kUdWarps][BT][2 * kMaxLoraRank];            // per-warp partials of this CTA's slice of x A
+    uint64_t zdone;                                        // this CTA's slice of x A has been added
+};
+
+template <int BT, bool LORA>
 constexpr size_t smem_bytes()
 {
-    return (size_t)kGateStages * kGateStageBytes + kUdRingBytes + sizeof(Shared<BT>);
+    return (size_t)kGateStages * kGateStageBytes + kUdRingBytes + sizeof(Shared<BT>) +
+           (LORA ? sizeof(LoraShared<BT>) + 128 : 0);
+}
+
+template <int BT>
+__device__ __forceinline__ LoraShared<BT> &lora_of(Shared<BT> &S)
+{
+    const uintptr_t a = (reinterpret_cast<uintptr_t>(&S) + sizeof(Shared<BT>) + 127) & ~(uintptr_t)127;
+    return *reinterpret_cast<LoraShared<BT> *>(a);
 }
 
 __device__ __forceinline__ void flag_status(int *ctl, int bits) { atomicOr(ctl + kCtlStatus, bits); }
@@ -254,7 +275,7 @@ __device__ bool load_activations(const FusedParams &p, Shared<BT> &S, GroupSync 
 }
 
 // ------------------------------------------------------------------ gate producer
-template <int BT>
+template <int BT, bool LORA>
 __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *gring)
 {
     const uint64_t pol = l2_policy_evict_first();
@@ -327,9 +348,15 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
             d.last = (r0 + nr >= rows) ? 1 : 0;
             d.buf = buf;
             S.gissued[stage] = (int)phase + 1;
-            mbar_arrive_expect_tx(&S.gfull[stage], (uint32_t)nr * row_bytes);
+            uint32_t extra = 0;   // the LoRA variant: the chunk's adapter block rides on its first stage
+            if constexpr (LORA)
+                if (r0 == 0) extra = (uint32_t)rows * 6u * (uint32_t)p.lora_r;
+            mbar_arrive_expect_tx(&S.gfull[stage], (uint32_t)nr * row_bytes + extra);
             bulk_load(gring + (size_t)stage * kGateStageBytes, p.wg_t + (size_t)(n0 + r0) * H, (uint32_t)nr * row_bytes,
                       &S.gfull[stage], pol);
+            if constexpr (LORA)
+                if (extra)
+                    bulk_load(lora_of(S).blk[buf], p.lora_blk + (size_t)n0 * 3 * p.lora_r, extra, &S.gfull[stage], pol);
             if (++stage == kGateStages) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
@@ -432,7 +459,7 @@ __device__ bool wait_prologues(int *ctl)
 // producer's claims precede the list producer's end).  The second call counts
 // the CTA done; the last CTA counted resets the counters for the next call,
 // which uses them only after this grid has ended.
-template <int BT>
+template <int BT, bool LORA>
 __device__ void counters_released(const FusedParams &p, Shared<BT> &S)
 {
     uint32_t prior;
@@ -442,6 +469,14 @@ __device__ void counters_released(const FusedParams &p, Shared<BT> &S)
         atomicExch(p.ctl + kCtlPrologue, 0);
         atomicExch(p.ctl + kCtlChunk, 0);
         atomicExch(p.ctl + kCtlDone, 0);
+        if constexpr (LORA) {   // every CTA has read x A: clear the sums this call used, for the next call
+            const int r2 = 2 * p.lora_r;
+            for (int k = 0; k < kLoraZCopies; ++k)
+                for (int b = 0; b < p.nb; ++b)
+                    for (int c = 0; c < r2; c += 4)
+                        *reinterpret_cast<float4 *>(p.lora_z + (k * kMaxTokensPerPass + b) * 2 * kMaxLoraRank + c) =
+                            make_float4(0.f, 0.f, 0.f, 0.f);
+        }
     }
 }
 
@@ -450,18 +485,39 @@ __device__ void counters_released(const FusedParams &p, Shared<BT> &S)
 // SiLU (Eq. 2), CATS mask (Eqs. 4-5) per token, keep trace.  Returns the
 // union of rows kept by any token, with each lane's a values and the kept rows
 // per token.
-template <int BT>
+template <int BT, bool LORA>
 __device__ uint32_t chunk_keep(const FusedParams &p, Shared<BT> &S, int buf, int n0, int rows, int lane,
-                               float (&a)[BT], uint32_t (&bal)[BT])
+                               float (&a)[BT], uint32_t (&bal)[BT], float (&lu)[BT],
+                               uint32_t (&adr)[kMaxLoraRank / 2])
 {
     const bool in = lane < rows;
     uint32_t uni = 0;
+    const uint16_t *lb = nullptr;   // LoRA: this row's B_gate column, B_up column, A_down row
+    if constexpr (LORA) {
+        lb = lora_of(S).blk[buf] + lane * 3 * p.lora_r;
+#pragma unroll
+        for (int q2 = 0; q2 < kMaxLoraRank / 2; ++q2)
+            adr[q2] = (in && 2 * q2 < p.lora_r) ? reinterpret_cast<const uint32_t *>(lb + 2 * p.lora_r)[q2] : 0u;
+    }
 #pragma unroll
     for (int b = 0; b < BT; ++b) {
         float g = 0.f;
         if (in) {
 #pragma unroll
             for (int w = 0; w < kGateWarps; ++w) g += S.gpart[buf][lane][b][w];
+        }
+        if constexpr (LORA) {
+            // g += scale (x A_gate) B_gate[:, j];  the up term scale (x A_up) B_up[:, j] for the W_ud stage
+            float lg = 0.f, lv = 0.f;
+            if (in) {
+                const float *z = lora_of(S).z[b];
+                for (int q = 0; q < p.lora_r; ++q) {
+                    lg = fmaf(z[q], __uint_as_float((uint32_t)lb[q] << 16), lg);
+                    lv = fmaf(z[p.lora_r + q], __uint_as_float((uint32_t)lb[p.lora_r + q] << 16), lv);
+                }
+            }
+            g = fmaf(p.lora_scale, lg, g);
+            lu[b] = p.lora_scale * lv;
         }
         a[b] = g / (1.0f + expf(-g));                                   // SiLU, Eq. 2
         const bool keep = in && b < p.nb && fabsf(a[b]) >= S.thr[b];    // Eqs. 4-5
@@ -478,7 +534,7 @@ __device__ uint32_t chunk_keep(const FusedParams &p, Shared<BT> &S, int buf, int
     return uni;
 }
 
-template <int BT>
+template <int BT, bool LORA>
 __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *uring, int lane)
 {
     const uint64_t pol = l2_policy_evict_first();
@@ -513,6 +569,7 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
     }
     __threadfence();
     bool ok = mbar_wait(&S.xloaded, 0u, &S.abort);
+    if constexpr (LORA) ok = ok && mbar_wait(&lora_of(S).zdone, 0u, &S.abort);   // this CTA's slice of x A is added
     __syncwarp();
     if (ok && lane == 0) {
         // this CTA has read its activations, zeroed its slice of y and cleared its flags
@@ -549,9 +606,30 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         const int n0 = S.chunkq[buf];
         if (n0 < 0) break;
         const int rows = S.chunkrows[buf];
-        float a[BT];
-        uint32_t bal[BT];
-        const uint32_t uni = chunk_keep<BT>(p, S, buf, n0, rows, lane, a, bal);
+        if constexpr (LORA) {
+            if (seq == 0) {
+                // x A (summed by every CTA before its prologue) is complete once every CTA is past it
+                int open = 1;
+                if (lane == 0 && !flags_open) open = (flags_open = wait_prologues(p.ctl)) ? 1 : 0;
+                if (!__shfl_sync(0xffffffffu, open, 0)) { ok = false; break; }
+                const int r2 = 2 * p.lora_r;
+                for (int i = lane; i < BT * r2; i += 32) {
+                    const int b = i / r2, c = i % r2;
+                    float v[kLoraZCopies];
+#pragma unroll
+                    for (int k = 0; k < kLoraZCopies; ++k)
+                        v[k] = b < p.nb ? __ldcg(p.lora_z + (k * kMaxTokensPerPass + b) * 2 * kMaxLoraRank + c) : 0.f;
+                    float z = 0.f;
+#pragma unroll
+                    for (int k = 0; k < kLoraZCopies; ++k) z += v[k];
+                    lora_of(S).z[b][c] = z;
+                }
+                __syncwarp();
+            }
+        }
+        float a[BT], lu[BT];
+        uint32_t bal[BT], adr[kMaxLoraRank / 2];
+        const uint32_t uni = chunk_keep<BT, LORA>(p, S, buf, n0, rows, lane, a, bal, lu, adr);
         __syncwarp();
         if (lane == 0) mbar_arrive(&S.bfree[buf]);   // partials read: the gate producer may refill the buffer
         if (!p.active_idx) {
@@ -579,6 +657,13 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
             if (in_stage) {
 #pragma unroll
                 for (int b = 0; b < BT; ++b) d.am[pos - k0][b] = ((bal[b] >> lane) & 1u) ? a[b] : 0.f;
+                if constexpr (LORA) {
+                    LoraShared<BT> &L = lora_of(S);
+#pragma unroll
+                    for (int b = 0; b < BT; ++b) L.lu[stage][pos - k0][b] = lu[b];
+#pragma unroll
+                    for (int q2 = 0; q2 < kMaxLoraRank / 2; ++q2) L.ad[stage][pos - k0][q2] = adr[q2];
+                }
             }
             __syncwarp();     // descriptor entries written before lane 0's release below
             if (lane == 0) {
@@ -614,7 +699,7 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         // the CTA adds into y only after every CTA has read its activations
         if (!flags_open && !*(volatile int *)&S.abort) flags_open = wait_prologues(p.ctl);
         S.seen = flags_open ? 1 : 0;
-        counters_released<BT>(p, S);
+        counters_released<BT, LORA>(p, S);
     }
     __syncwarp();
 }
@@ -670,7 +755,7 @@ __device__ __forceinline__ bool wait_words(const uint64_t *w, bool need, Shared<
 //      counts of the slices after the nearest published prefix; it publishes its
 //      own prefix and those of the slices it summed;
 //   3. each chunk's entries, from a warp scan of the chunks' counts.
-template <int BT>
+template <int BT, bool LORA>
 __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
 {
     static_assert(BT <= 2, "slice words carry two tokens' counts");
@@ -684,7 +769,7 @@ __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
     int go = 1;
     if (lane == 0) {
         if (work) go = wait_prologues(p.ctl) ? 1 : 0;   // every word is cleared for this call
-        counters_released<BT>(p, S);                   // the index warp's only counter read is above
+        counters_released<BT, LORA>(p, S);                   // the index warp's only counter read is above
     }
     if (!work) return;
     if (!__shfl_sync(0xffffffffu, go, 0)) {
@@ -809,9 +894,10 @@ __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
 // Down projection of one W_ud stage: y[cols] += h_j * W_down[j, cols], with
 // h_j = am_j * u_j and u_j the cross-warp sum of the stage's up partials; then
 // releases the stage to the list producer.
-template <int BT, int VPT>
+template <int BT, int VPT, bool LORA>
 __device__ __forceinline__ void down_stage(const FusedParams &p, Shared<BT> &S, const uint8_t *sbase, int nr,
-                                           int ub, int st, int t, int lane, f32x2 (&yp)[BT][VPT][4])
+                                           int ub, int st, int t, int lane, f32x2 (&yp)[BT][VPT][4],
+                                           float (&wacc)[BT])
 {
     const int H = p.H, HV = H >> 3;
     const size_t ud_row_bytes = (size_t)H * 4;
@@ -822,8 +908,16 @@ __device__ __forceinline__ void down_stage(const FusedParams &p, Shared<BT> &S, 
             float u = S.upart[ub][k][b][lane & (kUdWarps - 1)];
 #pragma unroll
             for (int o = kUdWarps / 2; o > 0; o >>= 1) u += __shfl_xor_sync(0xffffffffu, u, o);
+            if constexpr (LORA) u += lora_of(S).lu[st][k][b];   // + scale (x A_up) B_up[:, j]
             const float h = S.udesc[st].am[k][b] * u;     // CATS_t(a) * (x W_up), Eqs. 1 and 5
             hh[b] = pack2(h, h);
+            if constexpr (LORA) {
+                // the first up/down warp sums h_j A_down[j, :], lane q holding column q
+                if (t < 32 && lane < p.lora_r) {
+                    const uint32_t wd = lora_of(S).ad[st][k][lane >> 1];
+                    wacc[b] = fmaf(h, __uint_as_float((lane & 1) ? (wd & 0xffff0000u) : (wd << 16)), wacc[b]);
+                }
+            }
         }
         const uint4 *down = reinterpret_cast<const uint4 *>(sbase + (size_t)k * ud_row_bytes + (size_t)H * 2);
 #pragma unroll
@@ -840,9 +934,12 @@ __device__ __forceinline__ void down_stage(const FusedParams &p, Shared<BT> &S, 
     if (lane == 0) mbar_arrive(&S.uempty[st]);
 }
 
-template <int BT, int VPT>
+template <int BT, int VPT, bool LORA>
 __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *uring, f32x2 (&yp)[BT][VPT][4])
 {
+    float wacc[BT];   // LoRA: this lane's column of sum_j h_j A_down[j, :] (first warp only)
+#pragma unroll
+    for (int b = 0; b < BT; ++b) wacc[b] = 0.f;
     const int t = threadIdx.x - kGateThreads;
     const int lane = t & 31, uw = t >> 5;
     const int H = p.H, HV = H >> 3;
@@ -867,6 +964,76 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
         flag_status(p.ctl, kStatusTimeout);
         return;
     }
+    if constexpr (LORA) {
+        // While no W_ud row can arrive yet (the first one follows the first chunk's mask, which
+        // needs x A_gate from every CTA): this CTA's share of x A_gate, x A_up over hidden rows
+        // [h0, h1).  Thread t takes row h0 + 32 pass + t / 8 and columns (t % 8) cw .. + cw - 1;
+        // the partials are summed over the rows in the warp (shuffles), then over the warps
+        // (shared memory), and added into one of kLoraZCopies copies of the sums.
+        LoraShared<BT> &L = lora_of(S);
+        const int r2 = 2 * p.lora_r, cw = r2 / 8;   // 2, 4, 6 or 8 columns per thread
+        const int h0 = (int)(((long long)H * blockIdx.x) / gridDim.x);
+        const int h1 = (int)(((long long)H * (blockIdx.x + 1)) / gridDim.x);
+        const int cg = t & 7;
+        float zp[BT][8];
+#pragma unroll
+        for (int b = 0; b < BT; ++b)
+#pragma unroll
+            for (int c = 0; c < 8; ++c) zp[b][c] = 0.f;
+        for (int h = h0 + (t >> 3); h < h1; h += kUdThreads / 8) {
+            float xv[BT];
+#pragma unroll
+            for (int b = 0; b < BT; ++b)
+                xv[b] = b >= p.nb ? 0.f
+                        : p.x_mode == kXBf16
+                            ? __uint_as_float((uint32_t)static_cast<const uint16_t *>(p.x)[(size_t)b * H + h] << 16)
+                            : static_cast<const float *>(p.x)[(size_t)b * H + h];
+            const uint16_t *arow = p.lora_agu + (size_t)h * r2 + cg * cw;
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                if (c < cw) {
+                    const float av = __uint_as_float((uint32_t)arow[c] << 16);
+#pragma unroll
+                    for (int b = 0; b < BT; ++b) zp[b][c] = fmaf(xv[b], av, zp[b][c]);
+                }
+            }
+        }
+        // lanes l, l ^ 8, l ^ 16, l ^ 24 hold the same columns for four rows
+#pragma unroll
+        for (int b = 0; b < BT; ++b)
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                zp[b][c] += __shfl_xor_sync(0xffffffffu, zp[b][c], 8);
+                zp[b][c] += __shfl_xor_sync(0xffffffffu, zp[b][c], 16);
+            }
+        if (lane < 8) {
+#pragma unroll
+            for (int b = 0; b < BT; ++b)
+#pragma unroll
+                for (int c = 0; c < 8; ++c)
+                    if (c < cw) L.zred[uw][b][cg * cw + c] = zp[b][c];
+        }
+        if (!us(lane, &S.abort)) {
+            S.abort = 1;
+            flag_status(p.ctl, kStatusTimeout);
+            return;
+        }
+        if (t < BT * r2) {
+            const int b = t / r2, c = t % r2;
+            float z = 0.f;
+#pragma unroll
+            for (int w = 0; w < kUdWarps; ++w) z += L.zred[w][b][c];
+            if (b < p.nb && h1 > h0)   // one of kLoraZCopies copies: few additions per address
+                atomicAdd(p.lora_z + ((blockIdx.x % kLoraZCopies) * kMaxTokensPerPass + b) * 2 * kMaxLoraRank + c, z);
+        }
+        __threadfence();
+        if (!us(lane, &S.abort)) {
+            S.abort = 1;
+            flag_status(p.ctl, kStatusTimeout);
+            return;
+        }
+        if (t == 0) mbar_arrive(&L.zdone);
+    }
     uint32_t stage = 0, phase = 0;
     int ud_seq = 0;
     // a W_ud stage whose up sums are complete but whose down projection is
@@ -881,8 +1048,8 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
         const UdDesc<BT> &d = S.udesc[stage];
         if (d.kind == kEnd) {
             if (pend_stage >= 0)
-                down_stage<BT, VPT>(p, S, uring + (size_t)pend_stage * geo.stage_bytes, pend_nr, pend_ub, pend_stage,
-                                    t, lane, yp);
+                down_stage<BT, VPT, LORA>(p, S, uring + (size_t)pend_stage * geo.stage_bytes, pend_nr, pend_ub,
+                                          pend_stage, t, lane, yp, wacc);
             break;
         }
         const int nr = d.nrows;
@@ -919,8 +1086,8 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
         }
         us.arrive(lane);
         if (pend_stage >= 0)
-            down_stage<BT, VPT>(p, S, uring + (size_t)pend_stage * geo.stage_bytes, pend_nr, pend_ub, pend_stage, t,
-                                lane, yp);
+            down_stage<BT, VPT, LORA>(p, S, uring + (size_t)pend_stage * geo.stage_bytes, pend_nr, pend_ub, pend_stage,
+                                      t, lane, yp, wacc);
         if (!us.wait(&S.abort)) {
             S.abort = 1;
             flag_status(p.ctl, kStatusTimeout);
@@ -931,6 +1098,44 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
         pend_ub = ub;
         ++ud_seq;
         if (++stage == (uint32_t)geo.stages) { stage = 0; phase ^= 1u; }
+    }
+    if constexpr (LORA) {
+        // y += scale (sum_j h_j A_down[j, :]) B_down over this CTA's rows, before the L2 reduction
+        LoraShared<BT> &L = lora_of(S);
+        if (t < 32 && lane < p.lora_r) {
+#pragma unroll
+            for (int b = 0; b < BT; ++b) L.w[b][lane] = wacc[b];
+        }
+        if (!us(lane, &S.abort)) {
+            S.abort = 1;
+            flag_status(p.ctl, kStatusTimeout);
+            return;
+        }
+        // four rank columns at a time, their B_down loads issued together (the rank is a multiple of 8)
+        for (int q0 = 0; q0 < p.lora_r; q0 += 4) {
+            uint4 wv[4][VPT];
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+#pragma unroll
+                for (int i = 0; i < VPT; ++i) {
+                    const int v = t + i * kUdThreads;
+                    wv[j][i] = v < HV ? __ldg(reinterpret_cast<const uint4 *>(p.lora_bd + (size_t)(q0 + j) * H) + v)
+                                      : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                f32x2 wq[BT];
+#pragma unroll
+                for (int b = 0; b < BT; ++b) {
+                    const float v = p.lora_scale * L.w[b][q0 + j];
+                    wq[b] = pack2(v, v);
+                }
+#pragma unroll
+                for (int i = 0; i < VPT; ++i)
+#pragma unroll
+                    for (int b = 0; b < BT; ++b) axpy8(wv[j][i], wq[b], yp[b][i]);
+            }
+        }
     }
 }
 
@@ -946,7 +1151,7 @@ __device__ void drain_copies(Shared<BT> &S)
 }
 
 
-template <int BT, int VPT>
+template <int BT, int VPT, bool LORA>
 __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParams p)
 {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -972,6 +1177,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
             mbar_init(&S.bfree[b], 1);
         }
         mbar_init(&S.xloaded, kGateWarps + kUdWarps);
+        if constexpr (LORA) mbar_init(&lora_of(S).zdone, 1);
         mbar_init(&S.gbar, kGateWarps);
         mbar_init(&S.ubar, kUdWarps);
         S.abort = 0;
@@ -988,14 +1194,14 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
     if (warp < kGateWarps) {
         gate_warps<BT, VPT>(p, S, gring);
     } else if (warp < kGateProducerWarp) {
-        updown_warps<BT, VPT>(p, S, uring, yp);
+        updown_warps<BT, VPT, LORA>(p, S, uring, yp);
     } else if (warp == kGateProducerWarp) {
-        if (lane == 0) gate_producer<BT>(p, S, gring);
+        if (lane == 0) gate_producer<BT, LORA>(p, S, gring);
         __syncwarp();
     } else if (warp == kListWarp) {
-        list_producer<BT>(p, S, uring, lane);
+        list_producer<BT, LORA>(p, S, uring, lane);
     } else {
-        index_warp<BT>(p, S, lane);
+        index_warp<BT, LORA>(p, S, lane);
     }
     __syncthreads();
     if (tid == 0 && S.abort) drain_copies<BT>(S);
@@ -1023,16 +1229,16 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
     }
 }
 
-template <int BT, int VPT>
+template <int BT, int VPT, bool LORA>
 cudaError_t launch_t(const FusedParams &p, int grid, cudaStream_t stream)
 {
     static unsigned long long configured = 0;   // one bit per device ordinal
-    const size_t smem = smem_bytes<BT>();
+    const size_t smem = smem_bytes<BT, LORA>();
     int dev = 0;
     cudaGetDevice(&dev);
     const unsigned long long bit = 1ull << (dev & 63);
     if (!(configured & bit)) {
-        cudaError_t e = cudaFuncSetAttribute(fused_mlp_kernel<BT, VPT>,
+        cudaError_t e = cudaFuncSetAttribute(fused_mlp_kernel<BT, VPT, LORA>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         configured |= bit;
@@ -1047,7 +1253,7 @@ cudaError_t launch_t(const FusedParams &p, int grid, cudaStream_t stream)
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, fused_mlp_kernel<BT, VPT>, p);
+    return cudaLaunchKernelEx(&cfg, fused_mlp_kernel<BT, VPT, LORA>, p);
 }
 
 }  // namespace
@@ -1074,15 +1280,22 @@ cudaError_t launch_fused(const FusedParams &p, cudaStream_t stream)
     const int grid = fused_grid(p.nchunks);
     const int vpt = fused_vectors_per_thread(p.H);
     if (p.nb < 1 || p.nb > fused_tokens_per_pass(p.H)) return cudaErrorInvalidValue;
+    if (p.lora_blk) {   // the LoRA variant
+        if (p.lora_r < 8 || p.lora_r > kMaxLoraRank || (p.lora_r % 8) || p.x_mode == kXResidNorm)
+            return cudaErrorInvalidValue;
+        if (vpt == 1) return p.nb <= 1 ? launch_t<1, 1, true>(p, grid, stream) : launch_t<2, 1, true>(p, grid, stream);
+        if (vpt == 2) return p.nb <= 1 ? launch_t<1, 2, true>(p, grid, stream) : launch_t<2, 2, true>(p, grid, stream);
+        return launch_t<1, 4, true>(p, grid, stream);
+    }
     if (vpt == 1) {
-        if (p.nb <= 1) return launch_t<1, 1>(p, grid, stream);
-        return launch_t<2, 1>(p, grid, stream);
+        if (p.nb <= 1) return launch_t<1, 1, false>(p, grid, stream);
+        return launch_t<2, 1, false>(p, grid, stream);
     }
     if (vpt == 2) {
-        if (p.nb <= 1) return launch_t<1, 2>(p, grid, stream);
-        return launch_t<2, 2>(p, grid, stream);
+        if (p.nb <= 1) return launch_t<1, 2, false>(p, grid, stream);
+        return launch_t<2, 2, false>(p, grid, stream);
     }
-    return launch_t<1, 4>(p, grid, stream);
+    return launch_t<1, 4, false>(p, grid, stream);
 }
 
 }  // namespace sats

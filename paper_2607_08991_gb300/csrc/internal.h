@@ -26,6 +26,16 @@ struct sats_layer {
     int ldn = 0;                  // row stride of h (N rounded up to a multiple of 8)
 };
 
+// A LoRA adapter of one MLP block for the sparse path of a fine-tuned model
+// (Sec. 4): W + scale A B for gate, up and down, packed for the fused kernel.
+struct sats_lora {
+    int H = 0, N = 0, r = 0, device = 0;
+    float scale = 0.f;
+    uint16_t *blk = nullptr;      // [ceil(N / 8)][8][3 r]: neuron j's B_gate[:, j], B_up[:, j], A_down[j, :]
+    uint16_t *agu = nullptr;      // [H][2 r]: A_gate[h, :], A_up[h, :]
+    uint16_t *bd = nullptr;       // [r][H]: B_down
+};
+
 namespace sats {
 
 constexpr int kChunk = 8;               // neurons per scheduling unit of the fused kernel
@@ -33,6 +43,8 @@ constexpr int kMaxTokensPerPass = 4;    // tokens one fused launch carries
 constexpr int kMaxGrid = 256;           // upper bound of the fused grid
 constexpr int kMaxH = 8192;
 constexpr int kMaxN = 1 << 20;
+constexpr int kMaxLoraRank = 32;        // LoRA rank of the fused kernel, a multiple of 8
+constexpr int kLoraZCopies = 16;        // copies of the x A sums, CTA c adding into copy c mod 16
 
 // Control block at the start of the workspace (ints).
 enum {
@@ -51,7 +63,7 @@ enum {
 // word per chunk of kChunk neurons (its kept rows) and one per CTA (its slice's
 // kept counts and prefix), cleared by the kernel itself at the start of each call.
 struct WsLayout {
-    size_t ctl, flags, route_perm, route_flags, tc, total;
+    size_t ctl, lora_z, flags, route_perm, route_flags, tc, total;
 };
 
 // Zeroes the control words of a workspace (the fused kernel's counters and status).
@@ -79,6 +91,11 @@ struct FusedParams {
     int32_t *active_idx;          // [nb][N] or nullptr
     int32_t *active_cnt;          // [nb] or nullptr
     uint8_t *keep_trace;          // [nb][N] or nullptr
+    const sats_lora *lora;        // host view of the adapter, or nullptr (the kernel reads the fields below)
+    const uint16_t *lora_blk, *lora_agu, *lora_bd;
+    int lora_r;
+    float lora_scale;
+    float *lora_z;                // [kLoraZCopies][kMaxTokensPerPass][2 kMaxLoraRank]: partial sums of x A_gate, x A_up
 };
 
 // Records the CUDA error behind a SATS_ECUDA result (per host thread), with a
@@ -92,6 +109,9 @@ cudaError_t launch_fused(const FusedParams &p, cudaStream_t stream);
 
 cudaError_t launch_pack(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd, int H, int N,
                         uint16_t *wg_t, uint16_t *w_ud, cudaStream_t stream);
+cudaError_t launch_pack_lora(const uint16_t *Ag, const uint16_t *Bg, const uint16_t *Au, const uint16_t *Bu,
+                             const uint16_t *Ad, const uint16_t *Bd, int H, int N, int r, sats_lora *l,
+                             cudaStream_t stream);
 
 // Tensor-core path (gemm_tc.cu) for batches larger than one fused pass.
 // tc_pack_layer allocates and fills gu_blk / wd_blk from wg_t and w_ud;
@@ -120,7 +140,8 @@ cudaError_t launch_gate_act_f32(const sats_layer *layer, const float *x, int B, 
 // (api.cu).  ws: a workspace of ws_layout(H, N, B).total bytes with zeroed control words.
 sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B, const float *t_l,
                       const float *norm_w, float eps, const uint8_t *dense_flags, int out_mode, float *out,
-                      int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws, cudaStream_t stream);
+                      int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws, cudaStream_t stream,
+                      const sats_lora *lora = nullptr);
 size_t select_ws_bytes();
 cudaError_t launch_select(const float *a, int64_t n, int64_t m, void *ws, float *t_dev,
                           cudaStream_t stream);

@@ -54,6 +54,10 @@ def lib() -> ctypes.CDLL:
             "sats_sparse_mlp_fixed_scratch": (I, [P, P, I, F, P, P, P, P]),
             "sats_sparse_mlp_union": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_sparse_mlp_union_f32": (I, [P, P, I, F, P, P, P, P, Z, P]),
+            "sats_lora_create": (I, [P, P, P, P, P, P, P, I, F, P, ctypes.POINTER(P)]),
+            "sats_lora_destroy": (I, [P]),
+            "sats_sparse_mlp_lora": (I, [P, P, P, I, F, P, P, P, P, Z, P]),
+            "sats_sparse_mlp_lora_f32": (I, [P, P, P, I, F, P, P, P, P, Z, P]),
             "sats_uses_tensor_cores": (I, [I, I]),
             "sats_last_cuda_error": (ctypes.c_char_p, []),
             "sats_dense_mlp": (I, [P, P, I, P, P, Z, P]),
@@ -88,6 +92,7 @@ def exported_symbols() -> Sequence[str]:
     return ("sats_version", "sats_status_string", "sats_layer_create", "sats_layer_destroy", "sats_layer_shape",
             "sats_workspace_bytes", "sats_workspace_init", "sats_sparse_mlp", "sats_sparse_mlp_f32",
             "sats_sparse_mlp_fixed_scratch", "sats_sparse_mlp_union", "sats_sparse_mlp_union_f32",
+            "sats_lora_create", "sats_lora_destroy", "sats_sparse_mlp_lora", "sats_sparse_mlp_lora_f32",
             "sats_uses_tensor_cores", "sats_last_cuda_error", "sats_dense_mlp", "sats_route", "sats_mlp_stack",
             "sats_gate_act",
             "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_rmsnorm", "sats_gate_act_f32",
@@ -184,6 +189,50 @@ def sparse_mlp_f32(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor, w
     _check(lib().sats_sparse_mlp_f32(layer.handle, _ptr(x, "x", 4), B, float(t_l), _ptr(y, "y", 4),
                                      _ptr(active_idx, "active_idx", 4), _ptr(active_cnt, "active_cnt", 4),
                                      ws.ptr, ws.nbytes, _stream(stream)), "sats_sparse_mlp_f32")
+
+
+class Lora:
+    """A LoRA adapter of one block (sats_lora_create): A_gate, A_up [H][r], B_gate, B_up [r][N],
+    A_down [N][r], B_down [r][H] as int16 device tensors of bf16 bit patterns."""
+
+    def __init__(self, layer: Layer, A_gate, B_gate, A_up, B_up, A_down, B_down, scale: float = 1.0,
+                 stream: Optional[torch.cuda.Stream] = None):
+        r = A_gate.shape[1]
+        self.r = r
+        out = ctypes.c_void_p()
+        _check(lib().sats_lora_create(layer.handle, _ptr(A_gate, "A_gate", 2), _ptr(B_gate, "B_gate", 2),
+                                      _ptr(A_up, "A_up", 2), _ptr(B_up, "B_up", 2), _ptr(A_down, "A_down", 2),
+                                      _ptr(B_down, "B_down", 2), int(r), float(scale), _stream(stream),
+                                      ctypes.byref(out)), "sats_lora_create")
+        self.handle = out.value
+
+    def close(self):
+        if self.handle:
+            _check(lib().sats_lora_destroy(self.handle), "sats_lora_destroy")
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def sparse_mlp_lora(layer: Layer, lora: Lora, x: torch.Tensor, t_l: float, y: torch.Tensor, ws: Workspace,
+                    active_idx: Optional[torch.Tensor] = None, active_cnt: Optional[torch.Tensor] = None,
+                    stream: Optional[torch.cuda.Stream] = None):
+    """sats_sparse_mlp on the adapted weights W + scale A B (x bf16 or fp32)."""
+    B = x.shape[0]
+    if x.dtype == torch.float32:
+        _check(lib().sats_sparse_mlp_lora_f32(layer.handle, lora.handle, _ptr(x, "x", 4), B, float(t_l),
+                                              _ptr(y, "y", 4), _ptr(active_idx, "active_idx", 4),
+                                              _ptr(active_cnt, "active_cnt", 4), ws.ptr, ws.nbytes,
+                                              _stream(stream)), "sats_sparse_mlp_lora_f32")
+    else:
+        _check(lib().sats_sparse_mlp_lora(layer.handle, lora.handle, _ptr(x, "x", 2), B, float(t_l),
+                                          _ptr(y, "y", 4), _ptr(active_idx, "active_idx", 4),
+                                          _ptr(active_cnt, "active_cnt", 4), ws.ptr, ws.nbytes, _stream(stream)),
+               "sats_sparse_mlp_lora")
 
 
 def sparse_mlp_union(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor, ws: Workspace,
