@@ -429,7 +429,7 @@ def run_gpu(args):
                          "frac": achieved / hbm_peak, "peak_kind": peak_kind,
                          "traffic": None if traffic is None else
                          sum(traffic[s] for s in SPARSITY) / len(SPARSITY),
-                         "kernel": "fused_mlp_kernel<1,2>"},
+                         "kernel": "fused_mlp_kernel<1,2,0>"},
             "e2e": {"value": e2e_us, "unit": "us/token", "h2d_bytes_per_step": len(calls) * 2 * H,
                     "d2h_bytes_per_step": len(calls) * (4 * H + 4)},
             "gpu_launches": K * len(calls),
@@ -672,6 +672,52 @@ def run_workload(args):
                         "value": min(v["us_union"] for v in res.values()), "per_case": res,
                         "input": "x ~ N(0,1) per token (rho 0) or rho z_0 + sqrt(1-rho^2) z_m (rho 0.9), bf16",
                         "clocks": clk})
+        elif wl == "lora_llama_layer_4096x14336_b1":
+            # sats_sparse_mlp_lora against sats_sparse_mlp on the same layer copies and thresholds
+            H, N = spec["H"], spec["N"]
+            layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l)) for l in range(LAYER_COPIES)]
+            xc = torch.from_numpy(inputs.activations_bf16(spec["calib"], H, seed=inputs.SEED_CALIB).view(np.int16)).to(dev)
+            a = torch.empty(spec["calib"], N, dtype=torch.float32, device=dev)
+            sats.gate_act(layers[0], xc, a, stream=stream)
+            sel = torch.empty(sats.select_workspace_bytes(), dtype=torch.uint8, device=dev)
+            ts = {k: sats.percentile_threshold(a, k, sel, stream=stream) for k in spec["sparsity"]}
+            del a
+            ws = sats.Workspace(H, N, 1, device=dev)
+            x = torch.from_numpy(inputs.activations_bf16(1, H).view(np.int16)).to(dev)
+            y = torch.empty(1, H, dtype=torch.float32, device=dev)
+            idx = torch.empty(1, N, dtype=torch.int32, device=dev)
+            cnt = torch.empty(1, dtype=torch.int32, device=dev)
+            reps = max(args.steps, 50)
+            res = {}
+            clocks.start()
+            for k, t in ts.items():
+                base = lambda i, t=t: sats.sparse_mlp(layers[i % LAYER_COPIES], x, t, y, ws, idx, cnt, stream=stream)
+                for i in range(args.warmup + 3):
+                    base(i)
+                res["base_s%.1f" % k] = {"us": _timed(stream, base, reps)}
+            for r in spec["ranks"]:
+                los = [sats.Lora(layers[l], *(torch.from_numpy(m.view(np.int16)).to(dev)
+                                              for m in inputs.lora_adapter(H, N, r, seed=7000 + l)),
+                                 scale=spec["scale"], stream=stream) for l in range(LAYER_COPIES)]
+                for k, t in ts.items():
+                    call = lambda i, t=t: sats.sparse_mlp_lora(layers[i % LAYER_COPIES], los[i % LAYER_COPIES], x, t, y,
+                                                               ws, idx, cnt, stream=stream)
+                    for i in range(args.warmup + 3):
+                        call(i)
+                    stream.synchronize()
+                    kept = int(cnt.item())
+                    us = _timed(stream, call, reps)
+                    base_bytes = 2.0 * H * N + 4.0 * H * kept + 2.0 * H + 4.0 * H + 4.0 * kept + 4.0
+                    lora_bytes = N * 6.0 * r + H * 4.0 * r + r * 2.0 * H   # adapter blocks, A_gate | A_up, B_down
+                    res["r%d_s%.1f" % (r, k)] = {
+                        "us": us, "overhead_us": us - res["base_s%.1f" % k]["us"], "realised_sparsity": 1.0 - kept / N,
+                        "algo_bytes": base_bytes + lora_bytes, "achieved_gbs": (base_bytes + lora_bytes) / us / 1e3}
+                for l in los:
+                    l.close()
+            clk = clocks.stop()
+            out.update({"metric": "us/token, LoRA-aware sparse MLP (one layer)", "unit": "us/token",
+                        "value": res["r16_s0.5"]["us"], "per_case": res, "clocks": clk,
+                        "adapter": "synthetic rank-r factors N(0, 0.02) in bf16 on gate, up and down, scale 1"})
         elif wl == "sats_calibration_llama_32x4096x14336":
             H, N, L, C = spec["H"], spec["N"], spec["L"], spec["calib"]
             layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l)) for l in range(L)]

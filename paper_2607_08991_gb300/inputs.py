@@ -202,6 +202,9 @@ WORKLOADS: Dict[str, dict] = {
     # batched decode on the union of the kept neurons, independent and correlated tokens
     "union_batch_llama_4096x14336": dict(H=LLAMA_H, N=LLAMA_N, batches=[3, 4, 8], sparsity=[0.7, 0.9],
                                          rho=[0.0, 0.9], calib=256),
+    # the LoRA-aware sparse path (Sec. 4, fine-tuned routing) on the Llama layer, one decode token
+    "lora_llama_layer_4096x14336_b1": dict(H=LLAMA_H, N=LLAMA_N, ranks=[16, 32], sparsity=[0.5, 0.7, 0.9],
+                                           calib=256, scale=1.0),
     # SATS calibration (Sec. 3.1) of the 32-block Llama-shaped stack
     "sats_calibration_llama_32x4096x14336": dict(H=LLAMA_H, N=LLAMA_N, L=LLAMA_L, calib=64, K0=20, K1=8,
                                                   target=0.5, eps=1e-5),
