@@ -725,26 +725,6 @@ __device__ __forceinline__ bool wait_word(const uint64_t *w, Shared<BT> &S, unsi
     return __shfl_sync(0xffffffffu, good, 0) != 0;
 }
 
-// Each lane whose `need` is set waits (bounded, with backoff) until its word is
-// published; warp-uniform result.
-template <int BT>
-__device__ __forceinline__ bool wait_words(const uint64_t *w, bool need, Shared<BT> &S, unsigned long long t0)
-{
-    int good = 1;
-    if (need) {
-        uint32_t ns = 64;
-        while (flag_state(ld_relaxed_gpu_u64(w)) == 0u) {
-            if (global_ns() - t0 > kWaitLimitNs || *(volatile int *)&S.abort) {
-                good = 0;
-                break;
-            }
-            __nanosleep(ns);
-            ns = min(ns * 2u, 512u);
-        }
-    }
-    return __all_sync(0xffffffffu, good) != 0;
-}
-
 // The ascending per-token index lists, one slice of chunks per CTA.  The
 // entries of a chunk start at the number of neurons kept in all earlier chunks:
 //   1. the slice's kept counts, summed once each of its chunk words is published
@@ -799,14 +779,14 @@ __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
     uint64_t excl = 0;
     if (ok && lane == 0) st_relaxed_gpu_u64(sw + c, (c == 0 ? kFlagInc : kFlagAgg) | own);
     if (ok && c > 0) {
-        for (;;) {
-            // slice c-1-d for d = 32 i + lane
-            uint64_t f[kLookWords];
+        // slice c-1-d for d = 32 i + lane
+        uint64_t f[kLookWords];
 #pragma unroll
-            for (int i = 0; i < kLookWords; ++i) {
-                const int j = c - 1 - (32 * i + lane);
-                f[i] = j >= 0 ? ld_relaxed_gpu_u64(sw + j) : kFlagInc;   // before slice 0: 0
-            }
+        for (int i = 0; i < kLookWords; ++i) {
+            const int j = c - 1 - (32 * i + lane);
+            f[i] = j >= 0 ? ld_relaxed_gpu_u64(sw + j) : kFlagInc;   // before slice 0: 0
+        }
+        for (;;) {
             int first = 32 * kLookWords, missing = 32 * kLookWords;
 #pragma unroll
             for (int i = kLookWords - 1; i >= 0; --i) {
@@ -816,13 +796,23 @@ __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
                 if (unready) missing = 32 * i + __ffs(unready) - 1;
             }
             // first <= c always (the words before slice 0 read as prefix 0); wait for
-            // every unpublished word before the nearest prefix at once, then read again
+            // every unpublished word before the nearest prefix at once (each lane polls
+            // its own, bounded, with backoff) and keep the values the polls read
             if (missing < first) {
                 bool wait_ok = true;
 #pragma unroll
                 for (int i = 0; i < kLookWords; ++i) {
                     const int d = 32 * i + lane;
-                    wait_ok = wait_words<BT>(sw + (c - 1 - d), d < first && flag_state(f[i]) == 0u, S, t0) && wait_ok;
+                    int good = 1;
+                    if (d < first && flag_state(f[i]) == 0u) {
+                        uint32_t ns = 32;
+                        while (flag_state(f[i] = ld_relaxed_gpu_u64(sw + (c - 1 - d))) == 0u) {
+                            if (global_ns() - t0 > kWaitLimitNs || *(volatile int *)&S.abort) { good = 0; break; }
+                            __nanosleep(ns);
+                            ns = min(ns * 2u, 256u);
+                        }
+                    }
+                    wait_ok = __all_sync(0xffffffffu, good) && wait_ok;
                 }
                 if (!wait_ok) { ok = false; break; }
                 continue;
