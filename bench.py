@@ -152,6 +152,24 @@ def _dist_env():
     return ws, rank, local
 
 
+def _max_over_ranks(values, world: int, device=None):
+    """Each value's maximum over the ranks of the default process group: the replicas run
+    independently, and the job takes as long as the slowest."""
+    if world <= 1:
+        return [float(v) for v in values]
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t]
+
+
+def _us_per_token(total_ms: float, steps: int, calls: int, world: int) -> float:
+    """Whole-job time per token: each of `world` replicas runs steps x calls one-token calls
+    in total_ms (the slowest replica's time)."""
+    return total_ms * 1e3 / (steps * calls * world)
+
+
 # ---------------------------------------------------------------------------- CPU oracle arm
 def _oracle_sample(budget_s: float, max_calls: int = 64):
     """Times the oracle on the workload: one token through the layer per call, cycling sparsity levels."""
@@ -393,10 +411,7 @@ def run_gpu(args):
     e2e_us = 1e3 * e2e_s.elapsed_time(e2e_e) / (Ke * len(calls))
 
     # aggregate over ranks (replicas): max time
-    if world > 1:
-        tt = torch.tensor([total_ms, e2e_us], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms, e2e_us = float(tt[0]), float(tt[1])
+    total_ms, e2e_us = _max_over_ranks([total_ms, e2e_us], world, device=dev)
     if rank == 0:
         hbm_peak, peak_kind = _peaks()
         per = {}
@@ -412,7 +427,7 @@ def run_gpu(args):
             us_all += mean_us[i]
         achieved = bytes_all / (us_all * 1e-6) / 1e9
         traffic = _ncu_traffic()
-        value = total_ms * 1e3 / (K * len(calls) * world)
+        value = _us_per_token(total_ms, K, len(calls), world)
         line = {
             "metric": METRIC, "value": value, "unit": "us/token", "n_gpus": world, "steps": K,
             "warmup": max(args.warmup, 3), "ms_per_step": total_ms / K, "higher_is_better": False,
