@@ -69,6 +69,8 @@ constexpr int kUdSlots = 4;
 constexpr int kUdSlotBytes = kUdRingBytes / kUdSlots;      // 32 KB
 constexpr int kBufs = 4;                                   // list buffers (gate lookahead, chunks)
 constexpr int kStaticChunks = 3;                           // fixed chunks per CTA before the claimed ones
+constexpr int kTailChunks = 4;                             // the last kTailChunks * G chunks are claimed ...
+constexpr int kTailLag = 2;                                // ... only kTailLag chunks ahead of the W_ud rows
 constexpr int kPendingChunks = 16;                        // chunk words held back until every CTA has cleared its flags
 constexpr int kMaxUdRows = 8;                              // W_ud rows per stage (small H)
 constexpr uint32_t kL2PrefetchBytes = 128 * 1024;          // gate rows brought into L2 before the previous call ends
@@ -133,6 +135,7 @@ struct Shared {
     int abort;
     int seen;                   // the list producer has seen every CTA past its prologue
     int quiet;                  // roles past their last use of the counters (list producer, index warp)
+    int ldone;                  // chunks whose W_ud rows the list producer has issued (read by the gate producer)
 };
 
 // Extra shared state of the LoRA variant (Sec. 4, fine-tuned sparse path), placed
@@ -360,9 +363,22 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
             if (++stage == kGateStages) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
-        // the next chunk is a claimed one: claim it while this chunk's rows stream
+        // the next chunk is a claimed one: claim it while this chunk's rows stream.  Near the
+        // end of the chunks, first let the list producer catch up (its W_ud rows issued up to
+        // kTailLag chunks behind this one): a CTA whose kept rows pile up takes no more chunks,
+        // so that the CTAs run out of W_ud rows at about the same time
         const bool next_fixed = seq + 1 < kStaticChunks && static_chunk(seq + 1) < nch;
-        if (!next_fixed) next_k = claim();
+        if (!next_fixed) {
+            if (k >= nch - kTailChunks * G) {
+                const unsigned long long t0 = global_ns();
+                while (*(volatile int *)&S.ldone < seq + 1 - kTailLag) {
+                    if (global_ns() - t0 > kWaitLimitNs || *(volatile int *)&S.abort) { ok = false; break; }
+                    __nanosleep(32);
+                }
+                if (!ok) break;
+            }
+            next_k = claim();
+        }
     }
     if (ok && mbar_wait(&S.gempty[stage], phase ^ 1u, &S.abort)) {
         S.gdesc[stage].kind = kEnd;
@@ -680,6 +696,7 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
             if (++stage == (uint32_t)geo.stages) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
+        if (lane == 0) *(volatile int *)&S.ldone = seq + 1;   // the gate producer may claim further
     }
     if (ok && p.active_idx) {
         int good = 1;
@@ -1173,6 +1190,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
         S.abort = 0;
         S.seen = 0;
         S.quiet = 0;
+        S.ldone = 0;
         mbar_init_fence();
     }
     __syncthreads();
