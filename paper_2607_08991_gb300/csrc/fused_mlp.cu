@@ -415,44 +415,103 @@ __device__ void gate_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *g
             flag_status(p.ctl, kStatusTimeout);
             return;
         }
-        const GateDesc &d = S.gdesc[stage];
-        if (d.kind == kEnd) break;
-        const int nr = d.nrows, r0 = d.chunk_pos, buf = d.buf, last = d.last;
-        const uint8_t *sbase = gring + (size_t)stage * kGateStageBytes;
-        for (int q = 0; q < nr; q += 2) {
-            // two rows at once: independent FMA chains, one transposed reduction
-            f32x2 acc[2][BT];
+        const GateDesc &d0 = S.gdesc[stage];
+        if (d0.kind == kEnd) break;
+        const int nr0 = d0.nrows, r0 = d0.chunk_pos, buf = d0.buf;
+        int last = d0.last;
+        const uint8_t *sb0 = gring + (size_t)stage * kGateStageBytes;
+        // Four rows share one transposed warp reduction (its shuffle chain bounds these
+        // warps).  Stages of four rows or more are taken alone; stages of one or two rows
+        // (H >= 4096) in pairs of one chunk, each stage released once its rows are in registers.
+        int adv = 1;
+        if (nr0 > 2) {
+            for (int q = 0; q < nr0; q += 4) {
+                f32x2 acc[4][BT];
 #pragma unroll
-            for (int r = 0; r < 2; ++r)
+                for (int r = 0; r < 4; ++r)
 #pragma unroll
-                for (int b = 0; b < BT; ++b) acc[r][b] = 0ull;
-            const bool pair = q + 2 <= nr;
+                    for (int b = 0; b < BT; ++b) acc[r][b] = 0ull;
 #pragma unroll
-            for (int i = 0; i < VPT; ++i) {
-                const int v = t + i * kGateThreads;
-                if (v < HV) {
-                    const uint4 w0 = reinterpret_cast<const uint4 *>(sbase + (size_t)q * row_bytes)[v];
-                    const uint4 w1 = pair ? reinterpret_cast<const uint4 *>(sbase + (size_t)(q + 1) * row_bytes)[v] : zero4;
+                for (int i = 0; i < VPT; ++i) {
+                    const int v = t + i * kGateThreads;
+                    if (v < HV) {
+                        uint4 w[4];
 #pragma unroll
-                    for (int b = 0; b < BT; ++b) {
-                        acc[0][b] = dot8_acc(w0, xp[b][i], acc[0][b]);
-                        acc[1][b] = dot8_acc(w1, xp[b][i], acc[1][b]);
+                        for (int r = 0; r < 4; ++r)
+                            w[r] = q + r < nr0 ? reinterpret_cast<const uint4 *>(sb0 + (size_t)(q + r) * row_bytes)[v] : zero4;
+#pragma unroll
+                        for (int r = 0; r < 4; ++r)
+#pragma unroll
+                            for (int b = 0; b < BT; ++b) acc[r][b] = dot8_acc(w[r], xp[b][i], acc[r][b]);
                     }
                 }
+                if (q + 4 >= nr0) {   // every row of the stage is in registers: the producer may refill it
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&S.gempty[stage]);
+                }
+#pragma unroll
+                for (int b = 0; b < BT; ++b) {
+                    const float tot = warp_sum4_transposed(hsum2(acc[0][b]), hsum2(acc[1][b]), hsum2(acc[2][b]),
+                                                           hsum2(acc[3][b]), lane);
+                    const int r = (lane >> 3) & 3;
+                    if ((lane & 7) == 0 && q + r < nr0) S.gpart[buf][r0 + q + r][b][warp] = tot;
+                }
+            }
+        } else {
+            // acc[0..1]: this stage's rows; acc[2..3]: the next stage's, when the chunk goes on
+            f32x2 acc[4][BT];
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+#pragma unroll
+                for (int b = 0; b < BT; ++b) acc[r][b] = 0ull;
+            auto rows2 = [&](const uint8_t *sb, int n, int o) {
+#pragma unroll
+                for (int i = 0; i < VPT; ++i) {
+                    const int v = t + i * kGateThreads;
+                    if (v < HV) {
+                        const uint4 w0 = reinterpret_cast<const uint4 *>(sb)[v];
+                        const uint4 w1 = n > 1 ? reinterpret_cast<const uint4 *>(sb + row_bytes)[v] : zero4;
+#pragma unroll
+                        for (int b = 0; b < BT; ++b) {
+                            acc[o][b] = dot8_acc(w0, xp[b][i], acc[o][b]);
+                            acc[o + 1][b] = dot8_acc(w1, xp[b][i], acc[o + 1][b]);
+                        }
+                    }
+                }
+            };
+            rows2(sb0, nr0, 0);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&S.gempty[stage]);
+            int nr1 = 0;
+            if (!last) {
+                const uint32_t stage1 = stage + 1 == kGateStages ? 0u : stage + 1;
+                const uint32_t phase1 = stage + 1 == kGateStages ? phase ^ 1u : phase;
+                if (!mbar_wait(&S.gfull[stage1], phase1, &S.abort)) {
+                    S.abort = 1;
+                    flag_status(p.ctl, kStatusTimeout);
+                    return;
+                }
+                const GateDesc &d1 = S.gdesc[stage1];
+                nr1 = d1.nrows;
+                last = d1.last;
+                rows2(gring + (size_t)stage1 * kGateStageBytes, nr1, 2);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&S.gempty[stage1]);
+                adv = 2;
             }
 #pragma unroll
             for (int b = 0; b < BT; ++b) {
-                const float tot = warp_sum2_transposed(hsum2(acc[0][b]), hsum2(acc[1][b]), lane);
-                const int r = lane >> 4;
-                if ((lane & 15) == 0 && q + r < nr) S.gpart[buf][r0 + q + r][b][warp] = tot;
+                const float tot = warp_sum4_transposed(hsum2(acc[0][b]), hsum2(acc[1][b]), hsum2(acc[2][b]),
+                                                       hsum2(acc[3][b]), lane);
+                const int j = (lane >> 3) & 3;   // rows j < 2 of this stage, j - 2 of the next
+                const bool valid = j < 2 ? j < nr0 : j - 2 < nr1;
+                if ((lane & 7) == 0 && valid) S.gpart[buf][r0 + (j < 2 ? j : nr0 + j - 2)][b][warp] = tot;
             }
         }
         __syncwarp();
-        if (lane == 0) {
-            mbar_arrive(&S.gempty[stage]);
-            if (last) mbar_arrive(&S.gsync[buf]);   // this warp's partials of the chunk are written
-        }
-        if (++stage == kGateStages) { stage = 0; phase ^= 1u; }
+        if (lane == 0 && last) mbar_arrive(&S.gsync[buf]);   // this warp's partials of the chunk are written
+        for (int k = 0; k < adv; ++k)
+            if (++stage == kGateStages) { stage = 0; phase ^= 1u; }
     }
 }
 
