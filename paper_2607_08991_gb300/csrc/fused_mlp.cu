@@ -68,12 +68,15 @@ constexpr int kUdRingBytes = 131072;
 constexpr int kUdSlots = 4;
 constexpr int kUdSlotBytes = kUdRingBytes / kUdSlots;      // 32 KB
 constexpr int kBufs = 4;                                   // list buffers (gate lookahead, chunks)
-constexpr int kStaticChunks = 3;                           // fixed chunks per CTA before the claimed ones
+// Fixed chunks per CTA before the claimed ones, and the gate bytes of the fixed chunks past
+// the first brought into L2 before the previous call ends.  With a LoRA adapter the first
+// mask waits for every CTA's share of x A, and the deeper prefetch measured slower there.
+template <bool LORA> constexpr int kStaticChunks = LORA ? 3 : 4;
+template <bool LORA> constexpr uint32_t kL2PrefetchBytes = (LORA ? 128u : 192u) * 1024u;
 constexpr int kTailChunks = 4;                             // the last kTailChunks * G chunks are claimed ...
 constexpr int kTailLag = 2;                                // ... only kTailLag chunks ahead of the W_ud rows
 constexpr int kPendingChunks = 16;                        // chunk words held back until every CTA has cleared its flags
 constexpr int kMaxUdRows = 8;                              // W_ud rows per stage (small H)
-constexpr uint32_t kL2PrefetchBytes = 128 * 1024;          // gate rows brought into L2 before the previous call ends
 
 // Index-list words (the flags region: nchunks chunk words, then one slice word
 // per CTA; CTA c's slice is chunks [c per, (c + 1) per), per = ceil(nchunks / G)).
@@ -287,14 +290,15 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
     const int rows_per_stage = min(kChunk, kGateStageBytes / (int)row_bytes);
     // chunk k holds neurons [8k, 8k + 8); chunks c + s G (s < kStaticChunks) are this
     // CTA's; the others, from kStaticChunks * G on, are claimed in increasing order
-    const int nstatic = kStaticChunks * G;
+    constexpr int kStatic = kStaticChunks<LORA>;
+    const int nstatic = kStatic * G;
     auto static_chunk = [&](int s) { return (int)blockIdx.x + s * G; };
     {
         // The weights do not depend on the previous call: while it finishes (its tail
         // leaves HBM mostly idle), start moving this CTA's fixed chunks past the first
         // (which the gate ring takes) into L2.
-        size_t left = kL2PrefetchBytes;
-        for (int s = 1; s < kStaticChunks && left > 0; ++s) {
+        size_t left = kL2PrefetchBytes<LORA>;
+        for (int s = 1; s < kStatic && left > 0; ++s) {
             const int k = static_chunk(s);
             if (k >= nch) break;
             const int n0 = k * kChunk;
@@ -324,7 +328,7 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
         const int buf = seq % kBufs;
         // the buffer's previous list has been formed (first kBufs uses pass)
         if (!mbar_wait(&S.bfree[buf], ((uint32_t)(seq / kBufs) & 1u) ^ 1u, &S.abort)) { ok = false; break; }
-        const bool fixed = seq < kStaticChunks && static_chunk(seq) < nch;
+        const bool fixed = seq < kStatic && static_chunk(seq) < nch;
         int k;
         if (fixed) {
             k = static_chunk(seq);
@@ -367,7 +371,7 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
         // end of the chunks, first let the list producer catch up (its W_ud rows issued up to
         // kTailLag chunks behind this one): a CTA whose kept rows pile up takes no more chunks,
         // so that the CTAs run out of W_ud rows at about the same time
-        const bool next_fixed = seq + 1 < kStaticChunks && static_chunk(seq + 1) < nch;
+        const bool next_fixed = seq + 1 < kStatic && static_chunk(seq + 1) < nch;
         if (!next_fixed) {
             if (k >= nch - kTailChunks * G) {
                 const unsigned long long t0 = global_ns();
@@ -795,7 +799,7 @@ __device__ __forceinline__ bool wait_word(const uint64_t *w, Shared<BT> &S, unsi
                 break;
             }
             __nanosleep(ns);
-            ns = min(ns * 2u, 512u);
+            ns = min(ns * 2u, 1024u);
         }
     }
     return __shfl_sync(0xffffffffu, good, 0) != 0;
