@@ -71,6 +71,7 @@ def _run(sats, oracle, H, N, B, k, seed=0, f32=False, want_lists=True):
     (512, 1408, 5, 0.5),        # five tokens: two passes
     (520, 200, 9, 0.6),         # H not a multiple of the thread count; three passes
     (2048, 700, 1, 0.9),
+    (2560, 1003, 2, 0.6),       # three gate rows per 16 KB stage (chunks of 3 + 3 + 2 rows; a 3-row tail)
     (4096, 640, 4, 0.5),        # two vectors per consumer thread
     (6144, 300, 3, 0.5),        # four vectors per consumer thread, passes of two
     (8192, 130, 2, 0.5),        # the largest hidden size
