@@ -13,26 +13,29 @@
 // One CTA per SM, 608 threads in five roles, two shared-memory rings fed by
 // cp.async.bulk copies that complete on per-stage mbarriers:
 //   * gate producer (one thread): works through chunks of 8 neurons: first the
-//     CTA's three fixed chunks (c, c + G, c + 2G, which it may stream before the
-//     previous call has finished), then chunks claimed in increasing order from
-//     one counter, so that faster SMs take more of them; a chunk is started only
-//     when one of four list buffers is free.  Streams gate rows into the gate
-//     ring (5 x 16 KB).
+//     CTA's fixed chunks c, c + G, ... (four, three with a LoRA adapter; it
+//     streams the first and brings the others into L2 before the previous call
+//     has finished), then chunks claimed in increasing order from one counter,
+//     so that faster SMs take more of them (over the last chunks, only while its
+//     W_ud rows keep up); a chunk is started only when one of four list buffers
+//     is free.  Streams gate rows into the gate ring (5 x 16 KB).
 //   * 8 gate warps: thread t owns the 16-byte vectors t, t + 256, ... of every
 //     gate row and keeps the matching activations in registers as float pairs;
-//     dot products use paired FP32 FMAs (fma.rn.f32x2), two rows at a time
-//     with a transposed warp reduction; per-warp partials go to the chunk's
-//     list buffer, then each warp arrives on the buffer's barrier.
+//     dot products use paired FP32 FMAs (fma.rn.f32x2), four rows per
+//     transposed warp reduction (stages of one or two rows taken in pairs);
+//     per-warp partials go to the chunk's list buffer, then each warp arrives on
+//     the buffer's barrier.
 //   * list producer (one warp, lane = row): sums the partials of a chunk,
 //     applies SiLU (Eq. 2) and the mask (Eqs. 4-5) per token, publishes the
 //     chunk's kept counts, frees the buffer, and streams the W_ud rows of the
 //     kept neurons into the W_ud ring (4 slots of 32 KB).
-//   * index warp: turns each chunk's kept rows into its entries of the
-//     ascending index lists.  A chunk's place in the list is the number of
-//     neurons kept in all earlier chunks, found by a decoupled look-back over
-//     the chunks' flag words (each holds the chunk's own counts, then the
-//     inclusive prefix once known), so the lists are complete as soon as every
-//     chunk's gate work is done.
+//   * index warp: turns the kept rows of its CTA's slice of consecutive chunks
+//     into their entries of the ascending index lists.  A chunk's place in the
+//     list is the number of neurons kept in all earlier chunks: the slice's
+//     counts are summed from its chunks' published words, and the counts of the
+//     slices before it found by a decoupled look-back over the slice words (each
+//     holds a slice's own counts, then its inclusive prefix once known), so the
+//     lists are complete soon after every chunk's gate work is done.
 //   * 8 up/down warps: thread t owns vectors t, t + 256, ... of the up and
 //     down halves of each W_ud row and keeps its y columns in registers.  The
 //     up dot products of a stage are reduced across these warps through a
@@ -1125,7 +1128,7 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
         const int nr = d.nrows;
         const int ub = ud_seq % 3;
         const uint8_t *sbase = uring + (size_t)stage * geo.stage_bytes;
-        // up dot products, two rows at a time
+        // up dot products, two rows per transposed reduction
         for (int q = 0; q < nr; q += 2) {
             f32x2 acc[2][BT];
 #pragma unroll
