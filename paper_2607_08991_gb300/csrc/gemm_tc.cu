@@ -125,6 +125,7 @@ struct SkinnyGuParams {
     const uint16_t *w;            // gu_blk
     int M, N, R, KBh, NT;
     int split;                    // 1: two B operands (bf16 hi and lo parts of fp32 x)
+    int merge;                    // split and NT <= 128: one MMA of N = 2 NT over both parts
     float t_l;                    // threshold of sparse-path tokens
     const uint8_t *dense_flags;   // [M] (1 = base path, threshold 0) or nullptr
     uint16_t *hact;               // [M][ldh] bf16: h rounded to bf16
@@ -161,6 +162,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ int abort_flag, issued_s, consumed_s;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int t = blockIdx.x, R = p.R, NT = p.NT, S = p.stages;
+    const int NX = p.merge ? 2 * NT : NT;   // accumulator columns per matrix: tokens, or their high then low parts
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -206,7 +208,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         issued_s = kb;   // a break happens only before stage kb's loads are issued (kb >= npre)
     } else if (warp == 1 && lane == 0) {
-        const uint32_t idesc = instr_desc(BM, NT);
+        // x's high and low parts sit back to back in the stage (one 2 NT-row tile): merged,
+        // one MMA of N = 2 NT covers both, its two column halves summed in the epilogue;
+        // otherwise (N would pass 256) a second MMA adds the low part into the same columns
+        const uint32_t idesc = instr_desc(BM, NX);
         int kb = 0;
         for (int s = 0, ph = 0; kb < p.KBh; ++kb) {
             if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
@@ -220,11 +225,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint64_t au = smem_desc(st + R * kTileBytes + kk * 32);
                 const uint64_t b = smem_desc(xa + kk * 32);
                 mma_bf16(tmem, ag, b, idesc, acc);
-                if (!p.gate_only) mma_bf16(tmem + NT, au, b, idesc, acc);
-                if (p.split) {
+                if (!p.gate_only) mma_bf16(tmem + NX, au, b, idesc, acc);
+                if (p.split && !p.merge) {
                     const uint64_t b2 = smem_desc(xa + p.x_bytes + kk * 32);
                     mma_bf16(tmem, ag, b2, idesc, 1u);
-                    if (!p.gate_only) mma_bf16(tmem + NT, au, b2, idesc, 1u);
+                    if (!p.gate_only) mma_bf16(tmem + NX, au, b2, idesc, 1u);
                 }
             }
             mma_commit(&empty[s]);
@@ -249,8 +254,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool row_ok = ok && r < R && n < p.N;
         bool any = false;   // gate-only mode: some token keeps neuron n
         for (int c0 = 0; c0 < NT; c0 += 16) {
-            float g[16], u[16];
+            float g[16], u[16], lo[16];
             tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)c0, g);
+            if (p.merge) {
+                tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(NT + c0), lo);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 16; ++e) g[e] += lo[e];
+            }
             if (p.gate_only) {
                 tmem_ld_wait();
                 if (!row_ok) continue;
@@ -268,7 +279,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 continue;
             }
-            tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(NT + c0), u);
+            tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(NX + c0), u);
+            if (p.merge) {
+                tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(NX + NT + c0), lo);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 16; ++e) u[e] += lo[e];
+            }
             tmem_ld_wait();
             if (!row_ok) continue;
 #pragma unroll
@@ -306,14 +323,16 @@ struct SkinnyDownParams {
     float *out;                   // [M][H] fp32, added to with L2 reductions
     int *ctl;
     int stages, stage_bytes, a_bytes;
-    uint32_t tmem_cols;           // two accumulators of NT columns
+    int merge;                    // NT <= 128: one MMA of N = 2 NT over h's high and low parts
+    uint32_t tmem_cols;           // two accumulators of NX columns (NX = 2 NT merged, else NT)
 };
 
 // CTA c handles units [c U / G, (c+1) U / G) in order; consecutive units of one
 // hidden tile form a segment accumulated in TMEM (two buffers, so that the
 // epilogue of one segment overlaps the MMAs of the next) and added into y.
 // Unit u's weight tile is tile u of wd_blk; h arrives as its high and low bf16
-// parts, two MMAs into the same accumulator.
+// parts, one tile of 2 NT rows: merged, one MMA per step whose column halves the
+// epilogue sums; otherwise two MMAs into the same accumulator.
 __global__ void __launch_bounds__(kThreads, 1)
     down_skinny_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmH2,
                        const SkinnyDownParams p)
@@ -329,6 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ int abort_flag, issued_s, consumed_s;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int S = p.stages, NT = p.NT, KBn = p.KBn;
+    const int NX = p.merge ? 2 * NT : NT;
     const int u0 = (int)((long long)blockIdx.x * p.units / gridDim.x);
     const int u1 = (int)((long long)(blockIdx.x + 1) * p.units / gridDim.x);
     const int nu = u1 - u0;
@@ -381,7 +401,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         issued_s = i;   // a break happens only before stage i's loads are issued (i >= npre)
     } else if (warp == 1 && lane == 0) {
-        const uint32_t idesc = instr_desc(BM, NT);
+        const uint32_t idesc = instr_desc(BM, NX);
         int i = 0, q = 0;
         int s = 0, ph = 0;
         for (int u = u0; u < u1 && !abort_flag;) {
@@ -400,10 +420,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int kk = 0; kk < BK / 16; ++kk) {
                     const uint64_t w = smem_desc(st + kk * 32);
-                    mma_bf16(tmem + (uint32_t)(buf * NT), w, smem_desc(st + p.a_bytes + kk * 32), idesc,
+                    mma_bf16(tmem + (uint32_t)(buf * NX), w, smem_desc(st + p.a_bytes + kk * 32), idesc,
                              (first && kk == 0) ? 0u : 1u);
-                    mma_bf16(tmem + (uint32_t)(buf * NT), w, smem_desc(st + p.a_bytes + NT * kTileBytes + kk * 32),
-                             idesc, 1u);
+                    if (!p.merge)
+                        mma_bf16(tmem + (uint32_t)(buf * NX), w, smem_desc(st + p.a_bytes + NT * kTileBytes + kk * 32),
+                                 idesc, 1u);
                 }
                 first = false;
                 mma_commit(&empty[s]);
@@ -425,8 +446,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const int h = d * BM + lb + lane;
             for (int c0 = 0; c0 < NT; c0 += 16) {
-                float v[16];
-                tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * NT + c0), v);
+                float v[16], lo[16];
+                tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * NX + c0), v);
+                if (p.merge) {
+                    tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * NX + NT + c0), lo);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) v[e] += lo[e];
+                }
                 tmem_ld_wait();
                 if (!ok || h >= p.H) continue;
 #pragma unroll
@@ -980,7 +1007,8 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         const int slack = over > 0 ? ((over + 1023) & ~1023) : 0;
         gp.stages = stages_for(gp.stage_bytes, kSmemBudget - slack);
         gp.ring_bytes = gp.stages * gp.stage_bytes + slack;
-        gp.tmem_cols = tmem_cols_for(NT);
+        gp.merge = split && NT <= 128 ? 1 : 0;
+        gp.tmem_cols = tmem_cols_for(gp.merge ? 2 * NT : NT);
         if ((e = set_smem(gu_skinny_kernel, smem_for(1, gp.ring_bytes), cfg_gu_skinny)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
         e = launch_pdl(gu_skinny_kernel, dim3(layer->tc_T), smem_for(1, gp.ring_bytes), stream, mX, mX2, gp);
@@ -1023,7 +1051,8 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         const int slack = over > 0 ? ((over + 1023) & ~1023) : 0;
         gp.stages = stages_for(gp.stage_bytes, kSmemBudget - slack);
         gp.ring_bytes = gp.stages * gp.stage_bytes + slack;
-        gp.tmem_cols = tmem_cols_for(2 * NT);
+        gp.merge = split && NT <= 128 ? 1 : 0;
+        gp.tmem_cols = tmem_cols_for((gp.merge ? 4 : 2) * NT);
         if ((e = set_smem(gu_skinny_kernel, smem_for(1, gp.ring_bytes), cfg_gu_skinny)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
         e = launch_pdl(gu_skinny_kernel, dim3(layer->tc_T), smem_for(1, gp.ring_bytes), stream, mX, mX2, gp);
@@ -1041,7 +1070,8 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         dp.a_bytes = BM * kTileBytes;
         dp.stage_bytes = dp.a_bytes + 2 * NT * kTileBytes;
         dp.stages = stages_for(dp.stage_bytes);
-        dp.tmem_cols = tmem_cols_for(2 * NT);
+        dp.merge = NT <= 128 ? 1 : 0;
+        dp.tmem_cols = tmem_cols_for((dp.merge ? 4 : 2) * NT);
         static std::atomic<int> cfg_dn[64];
         if ((e = set_smem(down_skinny_kernel, smem_for(dp.stages, dp.stage_bytes), cfg_dn)) != cudaSuccess)
             return fail(e, "shared-memory attribute");

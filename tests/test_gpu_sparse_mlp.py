@@ -105,10 +105,16 @@ def test_tensor_core_batches_match_oracle(sats, oracle, H, N, B, k):
     assert abs(frac - k) < 0.1
 
 
-def test_tensor_core_fp32_activations(sats, oracle):
+@pytest.mark.parametrize("H,N,B", [
+    (4096, 640, 3),     # 16 token columns: hi and lo parts in one MMA of N = 32
+    (1024, 777, 40),
+    (512, 1408, 128),   # 128 columns: the largest merged MMA (N = 256; 512 TMEM columns)
+    (512, 1408, 200),   # 208 columns: two MMAs per step, hi and lo into the same accumulator
+])
+def test_tensor_core_fp32_activations(sats, oracle, H, N, B):
     """fp32 x split into bf16 hi + lo parts: the gate keeps ~fp32 accuracy."""
-    assert sats.uses_tensor_cores(1024, 40)
-    _run(sats, oracle, 1024, 777, 40, 0.5, f32=True)
+    assert sats.uses_tensor_cores(H, B)
+    _run(sats, oracle, H, N, B, 0.5, f32=True)
 
 
 @pytest.mark.parametrize("B,k", [(8, 0.5), (64, 0.7), (256, 0.9), (2048, 0.5)])
