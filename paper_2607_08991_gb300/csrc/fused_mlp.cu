@@ -140,6 +140,7 @@ struct Shared {
     int pend_chunk[kPendingChunks];
     int abort;
     int seen;                   // the list producer has seen every CTA past its prologue
+    int lend;                   // the list producer has published its last chunk word
     int quiet;                  // roles past their last use of the counters (list producer, index warp)
     int ldone;                  // chunks whose W_ud rows the list producer has issued (read by the gate producer)
 };
@@ -769,6 +770,7 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         if (lane == 0 && npend > 0) good = publish(-1, 0ull, true) ? 1 : 0;
         ok = __shfl_sync(0xffffffffu, good, 0) != 0;
     }
+    if (lane == 0) *(volatile int *)&S.lend = 1;   // the index warp may poll harder: the stream is ending
     if (ok && mbar_wait(&S.uempty[stage], phase ^ 1u, &S.abort)) {
         if (lane == 0) {
             S.udesc[stage].kind = kEnd;
@@ -844,11 +846,23 @@ __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
     bool ok = true;
     // 1.
     uint64_t own = 0, f_first = 0;   // f_first: the words of the slice's first 32 chunks, kept for step 3
+    uint64_t lw[kLookWords];         // step 2's words, read early once this CTA's list producer is done
+    bool have_lw = false;
     for (int base = k0; base < k1 && ok; base += 32) {
         const int k = base + lane;
         uint64_t f;
         for (;;) {
+            // once this CTA's stream has ended few CTAs still poll: the last reload of the
+            // slice's words also reads the look-back words (one round trip fewer at the end)
+            have_lw = c > 0 && base + 32 >= k1 && *(volatile int *)&S.lend != 0;
             f = k < k1 ? ld_relaxed_gpu_u64(p.flags + k) : kChunkKept;
+            if (have_lw) {
+#pragma unroll
+                for (int i = 0; i < kLookWords; ++i) {
+                    const int j = c - 1 - (32 * i + lane);
+                    lw[i] = j >= 0 ? ld_relaxed_gpu_u64(p.flags + nch + j) : kFlagInc;
+                }
+            }
             const uint32_t missing = __ballot_sync(0xffffffffu, flag_state(f) == 0u);
             if (!missing) break;
             if (!wait_word<BT>(p.flags + base + __ffs(missing) - 1, S, t0, lane)) { ok = false; break; }
@@ -867,7 +881,7 @@ __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
 #pragma unroll
         for (int i = 0; i < kLookWords; ++i) {
             const int j = c - 1 - (32 * i + lane);
-            f[i] = j >= 0 ? ld_relaxed_gpu_u64(sw + j) : kFlagInc;   // before slice 0: 0
+            f[i] = have_lw ? lw[i] : j >= 0 ? ld_relaxed_gpu_u64(sw + j) : kFlagInc;   // before slice 0: 0
         }
         for (;;) {
             int first = 32 * kLookWords, missing = 32 * kLookWords;
@@ -1255,6 +1269,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
         mbar_init(&S.ubar, kUdWarps);
         S.abort = 0;
         S.seen = 0;
+        S.lend = 0;
         S.quiet = 0;
         S.ldone = 0;
         mbar_init_fence();
