@@ -388,6 +388,18 @@ SATS_API sats_status sats_route_calibrate(const float *score, int V, const int32
                                           size_t ws_bytes, void *stream);
 
 /*
+ * sats_selftest_wait_timeout -- exercises the failure path of the device-side
+ * waits without a fault: one small kernel runs the library's bounded waits on
+ * conditions nothing satisfies (an mbarrier phase no thread completes, a
+ * workspace counter no CTA raises).  Each gives up after its time limit (2 s)
+ * and records a timeout in the workspace status word, so a following
+ * sats_get_error returns SATS_ETIMEOUT (and clears it).  Takes about 4 s;
+ * the workspace and the device stay usable.  ws: a workspace of any layer
+ * shape (at least 256 bytes), not in use by another call.
+ */
+SATS_API sats_status sats_selftest_wait_timeout(void *ws, size_t ws_bytes, void *stream);
+
+/*
  * sats_get_error -- synchronises `stream`, reads the status word in the
  * workspace, clears it, and returns SATS_OK, SATS_EDEVICE (bad token id) or
  * SATS_ETIMEOUT (a device wait gave up).

@@ -498,6 +498,12 @@ static sats_status read_status(int32_t *word, cudaStream_t st)
     return SATS_OK;
 }
 
+sats_status sats_selftest_wait_timeout(void *ws, size_t ws_bytes, void *stream)
+{
+    if (!ws || ws_bytes < (size_t)kCtlInts * sizeof(int)) return SATS_EINVAL;
+    return from_cuda(launch_wait_timeout(static_cast<int *>(ws), static_cast<cudaStream_t>(stream)));
+}
+
 sats_status sats_get_error(void *ws, size_t ws_bytes, void *stream)
 {
     if (!ws || ws_bytes < (size_t)kCtlInts * sizeof(int)) return SATS_EINVAL;

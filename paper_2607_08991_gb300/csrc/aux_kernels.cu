@@ -277,6 +277,38 @@ cudaError_t launch_route(const int32_t *ids, int B, const uint8_t *lut, int V, i
     return cudaGetLastError();
 }
 
+// The library's bounded waits, made to run out: an mbarrier phase that no thread
+// completes (the wait every ring of the MLP kernels uses) and a counter in the
+// workspace that no CTA raises (the form of the fused kernel's prologue wait).
+// Each gives up after kWaitLimitNs and records a timeout in the status word.
+__global__ void wait_timeout_kernel(int *ctl)
+{
+    __shared__ uint64_t bar;
+    __shared__ int never;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        never = 0;
+        mbar_init_fence();
+    }
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+    if (!mbar_wait(&bar, 0u, &never)) atomicOr(ctl + kCtlStatus, kStatusTimeout);
+    const unsigned long long t0 = global_ns();
+    while (ld_acquire_gpu(ctl + kCtlSelftest) == 0) {
+        if (global_ns() - t0 > kWaitLimitNs) {
+            atomicOr(ctl + kCtlStatus, kStatusTimeout);
+            break;
+        }
+        __nanosleep(256);
+    }
+}
+
+cudaError_t launch_wait_timeout(int *ctl, cudaStream_t stream)
+{
+    wait_timeout_kernel<<<1, 32, 0, stream>>>(ctl);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_gate_act(const sats_layer *layer, const uint16_t *x, int B, float *a, cudaStream_t stream)
 {
     const int threads = 256;

@@ -55,7 +55,7 @@ enum {
     kCtlNDense = 4,     // route output of the stack driver
     kCtlPrologue = 5,   // CTAs that have read their activations (reset by the last CTA)
     kCtlDone = 6,       // CTAs past their last use of the counters (reset by the last CTA)
-    kCtlReserved7 = 7,  // reserved
+    kCtlSelftest = 7,   // stays 0: the wait self-test polls it until its time limit
     kCtlInts = 64
 };
 
@@ -130,6 +130,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
                          float eps, const uint8_t *dense_flags, int out_mode, float *out, int32_t *active_idx,
                          int32_t *active_cnt, uint8_t *keep_trace, void *tc_ws, int *ctl, cudaStream_t stream,
                          bool union_path = false);
+cudaError_t launch_wait_timeout(int *ctl, cudaStream_t stream);
 cudaError_t launch_route(const int32_t *ids, int B, const uint8_t *lut, int V, int32_t *perm,
                          int32_t *n_dense, uint8_t *flags, int32_t *status, cudaStream_t stream);
 cudaError_t launch_gate_act(const sats_layer *layer, const uint16_t *x, int B, float *a,

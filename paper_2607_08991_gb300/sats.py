@@ -78,6 +78,7 @@ def lib() -> ctypes.CDLL:
             "sats_route_calibrate": (I, [P, I, P, I64, D, ctypes.POINTER(F), ctypes.POINTER(D), P, P, Z, P]),
             "sats_get_error": (I, [P, Z, P]),
             "sats_get_status_word": (I, [P, P]),
+            "sats_selftest_wait_timeout": (I, [P, Z, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -98,7 +99,7 @@ def exported_symbols() -> Sequence[str]:
             "sats_select_workspace_bytes", "sats_percentile_threshold", "sats_rmsnorm", "sats_gate_act_f32",
             "sats_layer_err_workspace_bytes", "sats_layer_err", "sats_sats_select", "sats_sats_workspace_bytes",
             "sats_sats_calibrate", "sats_route_calib_workspace_bytes", "sats_token_scores", "sats_route_calibrate",
-            "sats_get_error", "sats_get_status_word")
+            "sats_get_error", "sats_get_status_word", "sats_selftest_wait_timeout")
 
 
 def status_string(s: int) -> str:
@@ -413,6 +414,12 @@ def route_calibrate(score: torch.Tensor, heldout_ids: torch.Tensor, r_tar: float
                                       heldout_ids.numel(), float(r_tar), ctypes.byref(tau), ctypes.byref(R),
                                       _ptr(lut, "lut", 1), ws, n, _stream(stream)), "sats_route_calibrate")
     return tau.value, R.value, lut
+
+
+def selftest_wait_timeout(ws: Workspace, stream: Optional[torch.cuda.Stream] = None):
+    """Runs the library's bounded device waits against conditions nothing satisfies; the
+    next get_error(ws) reads ETIMEOUT (takes about 4 s)."""
+    _check(lib().sats_selftest_wait_timeout(ws.ptr, ws.nbytes, _stream(stream)), "sats_selftest_wait_timeout")
 
 
 def get_error(ws: Workspace, stream: Optional[torch.cuda.Stream] = None) -> int:
