@@ -66,3 +66,36 @@ def test_host_side_checks(libsats):
     assert L.sats_percentile_threshold(None, 10, 0.0, ctypes.byref(t), None, 0, None) == sats.OK and t.value == 0.0
     assert L.sats_percentile_threshold(None, 10, 1.5, ctypes.byref(t), None, 0, None) == sats.OK
     assert t.value == float("inf")
+
+
+def test_every_entry_rejects_missing_arguments_before_any_cuda_call(libsats):
+    """Null pointers and impossible sizes come back as SATS_EINVAL from the host
+    checks, with no CUDA call made (this host has no GPU)."""
+    from paper_2607_08991_gb300 import sats
+    L = sats.lib()
+    E = sats.EINVAL
+    out = ctypes.c_void_p()
+    f, d = ctypes.c_float(), ctypes.c_double()
+    assert L.sats_sparse_mlp_f32(None, None, 1, 0.5, None, None, None, None, 0, None) == E
+    assert L.sats_sparse_mlp_fixed_scratch(None, None, 1, 0.5, None, None, None, None) == E
+    assert L.sats_sparse_mlp_union(None, None, 4, 0.5, None, None, None, None, 0, None) == E
+    assert L.sats_sparse_mlp_union_f32(None, None, 4, 0.5, None, None, None, None, 0, None) == E
+    assert L.sats_lora_create(None, None, None, None, None, None, None, 16, 1.0, None, ctypes.byref(out)) == E
+    assert L.sats_sparse_mlp_lora(None, None, None, 1, 0.5, None, None, None, None, 0, None) == E
+    assert L.sats_dense_mlp(None, None, 1, None, None, 0, None) == E
+    assert L.sats_gate_act(None, None, 1, None, None, 0, None) == E
+    assert L.sats_rmsnorm(None, 1, 64, None, 1e-5, None, None) == E
+    assert L.sats_layer_err(None, None, 1, None, 1, 1e-6, None, None, None, 0, None) == E
+    assert L.sats_token_scores(None, None, None, 10, 100, None, None, 0, None) == E
+    assert L.sats_route_calibrate(None, 100, None, 10, 0.5, ctypes.byref(f), ctypes.byref(d), None, None, 0,
+                                  None) == E
+    assert L.sats_selftest_wait_timeout(None, 0, None) == E
+    assert L.sats_selftest_wait_timeout(1, 16, None) == E        # smaller than the control block
+    assert L.sats_get_error(None, 0, None) == E
+    assert L.sats_get_status_word(None, None) == E
+    # the calibration workspaces are host-computed sizes
+    assert L.sats_select_workspace_bytes() > 0
+    assert L.sats_layer_err_workspace_bytes(4096, 14336, 64, 20) > 0
+    assert L.sats_route_calib_workspace_bytes(151936) >= 151936
+    assert L.sats_sats_workspace_bytes(4096, 14336, 32, 64, 20, 8) >= L.sats_layer_err_workspace_bytes(4096, 14336,
+                                                                                                         64, 20)
