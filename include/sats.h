@@ -142,21 +142,35 @@ SATS_API sats_status sats_sparse_mlp(const sats_layer *layer, const void *x, int
  * Arguments, results and errors are those of sats_sparse_mlp.  Instead of a
  * workspace the call uses one 256 KiB array in the library's device memory;
  * every GPU that loads the library holds this array until the process exits.
- * A shape whose workspace (sats_workspace_bytes(H, N, B)) exceeds 256 KiB is
- * rejected with SATS_ENOSPACE; with one 64-bit word per 8 neurons that admits
- * N up to about 243,000 for B <= 2.  The call allocates nothing: before its
- * kernel it clears the array's control words with cudaMemsetAsync on `stream`.
+ * A call whose workspace would exceed the array, i.e. with
+ * sats_workspace_bytes(H, N, B) > 256 KiB, is rejected with SATS_ENOSPACE
+ * before anything is enqueued.  On the fused small-batch kernel (B <= 2 for
+ * H <= 4096, B = 1 above) the workspace is one 64-bit word per 8 neurons plus
+ * about 17 KB, which admits N up to about 243,000; a batch on the tensor-core
+ * path (sats_uses_tensor_cores) also needs its staging (activations, h and
+ * keep bytes per token, and padding to whole tiles), so only small layers fit
+ * there: for example N <= 5504 at H = 8192, B = 2, and N <= 1008 at H = 4096,
+ * B = 8.  The call allocates nothing: before its kernels it clears the
+ * array's control words with cudaMemsetAsync on `stream`.
  *
- * The first call on each device looks up the array's device address
- * (cudaGetSymbolAddress); make that first call before any stream capture.
- * All calls share the one array, so calls that can overlap on the GPU (on
- * different streams, or from several host threads without ordering) race and
- * must be serialised by the caller.  Device-side errors of this call (a
- * bounded wait that gave up) are not reported.
+ *   dev_status : device int32 [1] or NULL.  If given, it receives this call's
+ *                device status word after the kernels, in stream order (0 when
+ *                every bounded device wait completed); sats_get_status_word
+ *                reads it back and returns SATS_OK, SATS_ETIMEOUT or
+ *                SATS_EDEVICE.  Without it, device-side errors of this call (a
+ *                bounded wait that gave up, leaving y and the index lists
+ *                incomplete) are not reported.
+ *
+ * Each call looks up the array's device address on the current device
+ * (cudaGetSymbolAddress, which neither allocates nor synchronises), so the
+ * address is always that of the current device and context.  All calls share
+ * the one array, so calls that can overlap on the GPU (on different streams,
+ * or from several host threads without ordering) race and must be serialised
+ * by the caller.
  */
 SATS_API sats_status sats_sparse_mlp_fixed_scratch(const sats_layer *layer, const void *x, int B, float t_l,
                                                    float *y, int32_t *active_idx, int32_t *active_cnt,
-                                                   void *stream);
+                                                   int32_t *dev_status, void *stream);
 
 /*
  * sats_uses_tensor_cores -- 1 if a call with batch B on a layer of hidden size

@@ -4,7 +4,6 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
-#include <mutex>
 #include <new>
 
 #include "common.cuh"
@@ -143,26 +142,20 @@ static sats_status sparse_common(const sats_layer *layer, int x_mode, const void
 // Fixed scratch for sats_sparse_mlp_fixed_scratch: one array in this file's
 // device memory, present on every GPU that loads the library until the
 // process exits.  Host code cannot use the symbol itself as a device address;
-// the address is looked up per device with cudaGetSymbolAddress.
+// the address is looked up with cudaGetSymbolAddress on every call (it
+// allocates nothing and does not synchronise), so it always belongs to the
+// current device and context, also after a cudaDeviceReset reloaded the module.
 constexpr size_t kFixedScratchBytes = (size_t)1 << 18;   // 256 KiB
 static __device__ __align__(256) unsigned char g_fixed_scratch[kFixedScratchBytes];
 
-static std::mutex g_fixed_scratch_mu;
-static void *g_fixed_scratch_ptr[64] = {};
-
-// Device address of g_fixed_scratch on the current device (looked up on the
-// first call for that device), or nullptr on failure.
-static void *fixed_scratch_current_device()
+// Device address of g_fixed_scratch on the current device, or nullptr (with the
+// CUDA error in *err) on failure.
+static void *fixed_scratch_current_device(cudaError_t *err)
 {
-    int dev = -1;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-    std::lock_guard<std::mutex> lock(g_fixed_scratch_mu);
-    if (!g_fixed_scratch_ptr[dev]) {
-        void *ptr = nullptr;
-        if (cudaGetSymbolAddress(&ptr, g_fixed_scratch) != cudaSuccess || !ptr) return nullptr;
-        g_fixed_scratch_ptr[dev] = ptr;
-    }
-    return g_fixed_scratch_ptr[dev];
+    void *ptr = nullptr;
+    *err = cudaGetSymbolAddress(&ptr, g_fixed_scratch);
+    if (*err == cudaSuccess && !ptr) *err = cudaErrorInvalidSymbol;
+    return *err == cudaSuccess ? ptr : nullptr;
 }
 
 }  // namespace sats
@@ -340,21 +333,31 @@ sats_status sats_sparse_mlp(const sats_layer *layer, const void *x, int B, float
 }
 
 sats_status sats_sparse_mlp_fixed_scratch(const sats_layer *layer, const void *x, int B, float t_l, float *y,
-                                          int32_t *active_idx, int32_t *active_cnt, void *stream)
+                                          int32_t *active_idx, int32_t *active_cnt, int32_t *dev_status,
+                                          void *stream)
 {
     if (!layer || B < 0) return SATS_EINVAL;
     if (ws_layout(layer->H, layer->N, B).total > kFixedScratchBytes) return SATS_ENOSPACE;
     if (bad_threshold(t_l)) return SATS_EINVAL;
     if ((active_idx == nullptr) != (active_cnt == nullptr)) return SATS_EINVAL;
+    if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return SATS_EINVAL;
     if (B == 0) return SATS_OK;
     if (!x || !y || !aligned16(x) || !aligned16(y)) return SATS_EINVAL;
-    void *ws = fixed_scratch_current_device();
-    if (!ws) return cuda_fail(cudaErrorInvalidSymbol, "fixed scratch lookup");
+    cudaError_t el = cudaSuccess;
+    void *ws = fixed_scratch_current_device(&el);
+    if (!ws) return cuda_fail(el, "fixed scratch lookup");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
     // the array keeps the previous call's contents: the control words
     // (scheduling counters, status) must start at zero
-    const cudaError_t ez = clear_fused_state(ws, layer->H, layer->N, B, static_cast<cudaStream_t>(stream));
+    const cudaError_t ez = clear_fused_state(ws, layer->H, layer->N, B, st);
     if (ez != cudaSuccess) return cuda_fail(ez, "fixed scratch clear");
-    return sparse_common(layer, kXBf16, x, B, t_l, y, active_idx, active_cnt, ws, kFixedScratchBytes, stream);
+    const sats_status s = sparse_common(layer, kXBf16, x, B, t_l, y, active_idx, active_cnt, ws,
+                                        kFixedScratchBytes, stream);
+    if (s != SATS_OK || !dev_status) return s;
+    // this call's device status word (cleared above, so it holds this call's errors only)
+    const int32_t *word = static_cast<const int32_t *>(ws) + kCtlStatus;   // the control block starts the scratch
+    return from_cuda(cudaMemcpyAsync(dev_status, word, sizeof(int32_t), cudaMemcpyDeviceToDevice, st),
+                     "fixed scratch status copy");
 }
 
 int sats_uses_tensor_cores(int H, int B) { return use_tc_path(H, B) ? 1 : 0; }

@@ -51,7 +51,7 @@ def lib() -> ctypes.CDLL:
             "sats_workspace_init": (I, [P, Z, P]),
             "sats_sparse_mlp": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_sparse_mlp_f32": (I, [P, P, I, F, P, P, P, P, Z, P]),
-            "sats_sparse_mlp_fixed_scratch": (I, [P, P, I, F, P, P, P, P]),
+            "sats_sparse_mlp_fixed_scratch": (I, [P, P, I, F, P, P, P, P, P]),
             "sats_sparse_mlp_union": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_sparse_mlp_union_f32": (I, [P, P, I, F, P, P, P, P, Z, P]),
             "sats_lora_create": (I, [P, P, P, P, P, P, P, I, F, P, ctypes.POINTER(P)]),
@@ -253,12 +253,14 @@ def sparse_mlp_union(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor,
 
 def sparse_mlp_fixed_scratch(layer: Layer, x: torch.Tensor, t_l: float, y: torch.Tensor,
                              active_idx: Optional[torch.Tensor] = None, active_cnt: Optional[torch.Tensor] = None,
-                             stream: Optional[torch.cuda.Stream] = None):
-    """sats_sparse_mlp without a workspace (the library's fixed 256 KiB device scratch)."""
+                             dev_status: Optional[torch.Tensor] = None, stream: Optional[torch.cuda.Stream] = None):
+    """sats_sparse_mlp without a workspace (the library's fixed 256 KiB device scratch); dev_status, a
+    device int32 [1], receives the call's device status word (read it with get_status_word)."""
     B = x.shape[0]
     _check(lib().sats_sparse_mlp_fixed_scratch(layer.handle, _ptr(x, "x", 2), B, float(t_l), _ptr(y, "y", 4),
                                                _ptr(active_idx, "active_idx", 4), _ptr(active_cnt, "active_cnt", 4),
-                                               _stream(stream)), "sats_sparse_mlp_fixed_scratch")
+                                               _ptr(dev_status, "dev_status", 4), _stream(stream)),
+           "sats_sparse_mlp_fixed_scratch")
 
 
 def uses_tensor_cores(H: int, B: int) -> bool:

@@ -77,7 +77,7 @@ def test_every_entry_rejects_missing_arguments_before_any_cuda_call(libsats):
     out = ctypes.c_void_p()
     f, d = ctypes.c_float(), ctypes.c_double()
     assert L.sats_sparse_mlp_f32(None, None, 1, 0.5, None, None, None, None, 0, None) == E
-    assert L.sats_sparse_mlp_fixed_scratch(None, None, 1, 0.5, None, None, None, None) == E
+    assert L.sats_sparse_mlp_fixed_scratch(None, None, 1, 0.5, None, None, None, None, None) == E
     assert L.sats_sparse_mlp_union(None, None, 4, 0.5, None, None, None, None, 0, None) == E
     assert L.sats_sparse_mlp_union_f32(None, None, 4, 0.5, None, None, None, None, 0, None) == E
     assert L.sats_lora_create(None, None, None, None, None, None, None, 16, 1.0, None, ctypes.byref(out)) == E

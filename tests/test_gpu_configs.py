@@ -105,6 +105,12 @@ def test_config2_llama_layer_256_calibration_vectors(sats, oracle):
         y_ref, a_ref, keep_ref, _ = oracle.sparse_mlp(x64, hg, hu, hd, t, keep_hint=keep_gpu, band_rel=P.BAND_REL)
         P.assert_keep_match(keep_gpu, keep_ref, a_ref, t)
         P.assert_close(y.cpu().numpy(), y_ref)
+        # and with no decision taken from the kernel: the oracle's own mask at t, held to the
+        # task's tolerance (a neuron decided the other way inside the band would move y by one
+        # neuron's contribution)
+        y_own, _, keep_own, _ = oracle.sparse_mlp(x64, hg, hu, hd, t)
+        P.assert_close(y.cpu().numpy(), y_own, tight=False)
+        assert int((keep_own != keep_gpu).sum()) <= int(P.band_mask(a_ref, t).sum())
         assert abs((1.0 - keep_gpu.mean()) - k) < 0.05
     layer.close()
 

@@ -9,7 +9,8 @@
   (for a candidate that is itself some neuron's |a|, between the oracle's
   values just below and just above it); the guardrail threshold is the
   oracle's percentile at the target; and the choice of b*, T*(b*) is the
-  oracle's Eqs. 7-10 applied to the same table.
+  oracle's Eqs. 7-10 applied to the same table; the fine candidates are the
+  oracle's (the same coarse choice, the same placement between its neighbours).
 """
 import numpy as np
 import pytest
@@ -99,5 +100,10 @@ def test_sats_calibrate_matches_oracle_step_by_step(sats, oracle):
     assert b2 == r["b"]
     np.testing.assert_allclose(t2[:L - 1], t_sel[:L - 1], rtol=0, atol=0)
     assert abs(r["S"] - s_tar) < 0.1
+    # the fine candidates (coarse-to-fine, step 5): the oracle's, placed between the coarse
+    # neighbours of the same coarse choice, to the fp32 rounding of the candidates
+    r_or = oracle.sats_calibrate(x.astype(np.float64), [w.Wg for w in ws_], [w.Wu for w in ws_],
+                                 [w.Wd for w in ws_], nw, eps, s_tar, K0=K0, K1=K1, guardrail=True)
+    np.testing.assert_allclose(tt[:, Kc:], r_or["fine"][0][:, Kc:], rtol=1e-4)
     for l in layers:
         l.close()

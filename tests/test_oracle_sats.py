@@ -187,7 +187,114 @@ def test_calibrate_hits_the_target_within_the_candidate_spacing(oracle):
     for l in range(L - 1):
         adm = t_all[l][e_all[l] <= r["b"]]
         assert r["t"][l] == (adm.max() if adm.size else 0.0)
-    # the fine candidates sit strictly between coarse neighbours of the coarse choice
+    # the coarse candidates are increasing percentiles (their fine neighbours are pinned below)
     coarse_t = r["coarse"][0]
     assert np.all(np.diff(coarse_t, axis=1) >= 0.0)
     assert abs(r["S"] - 0.5) < 0.1
+
+
+# ---------------------------------------------------------------- coarse-to-fine: the fine candidates
+#
+# A one-block stack worked by hand (H = 1, N = 2, two calibration tokens, RMSNorm with eps = 0 and
+# gain 1, so the block inputs are n = +1 and n = -1; W_gate = [1, 2], W_up = [1, 1],
+# W_down = [1, 1]^T, so y = n * sum_j keep_j a_j).  The four post-gate magnitudes are
+#   |SiLU(-2)| = 2 / (1 + e^2),  |SiLU(-1)| = 1 / (1 + e),  SiLU(1) = 1 / (1 + e^-1),  SiLU(2) = 2 / (1 + e^-2)
+# in increasing order.  With K0 = 4 the coarse candidates are the Eq. 3 percentiles at 1/4, 2/4, 3/4:
+# the first three magnitudes (m = ceil(k n) = k of n = 4 values).  Eq. 6 at each (token 0 keeps both
+# neurons below SiLU(1); token 1 loses |SiLU(-2)| at the second and both at the third):
+#   t1: err 0,                                        sp 0
+#   t2: err (0 + |SiLU(-2)| / (|SiLU(-1)| + |SiLU(-2)|)) / 2,  sp 1/4
+#   t3: err (0 + 1) / 2,                              sp 1/2
+# Eqs. 7-10 then pick t2 for s_tar = 0.3, t3 for 0.45 and t1 for 0, and step 5 places K1 = 3
+# candidates at lo + (hi - lo) k / 4 between the coarse neighbours of that choice: (t1, t3), (t2, max|a|)
+# and (0, t2) respectively.
+
+def _silu(z):
+    import math
+    return z / (1.0 + math.exp(-z))
+
+
+def _worked_block():
+    bits = lambda v: (np.asarray(v, np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    Wg = bits([[1.0, 2.0]])
+    Wu = bits([[1.0, 1.0]])
+    Wd = bits([[1.0], [1.0]])
+    x = np.array([[1.0], [-1.0]])
+    return x, Wg, Wu, Wd, [np.ones(1, np.float32)]
+
+
+@pytest.mark.parametrize("s_tar,lo,hi", [
+    (0.3, lambda m: m[0], lambda m: m[2]),
+    (0.45, lambda m: m[1], lambda m: m[3]),
+    (0.0, lambda m: 0.0, lambda m: m[1]),
+])
+def test_fine_candidates_of_a_worked_block(oracle, s_tar, lo, hi):
+    x, Wg, Wu, Wd, nw = _worked_block()
+    mags = [abs(_silu(-2.0)), abs(_silu(-1.0)), _silu(1.0), _silu(2.0)]   # increasing
+    r = oracle.sats_calibrate(x, [Wg], [Wu], [Wd], nw, 0.0, s_tar, K0=4, K1=3, guardrail=False, err_eps=0.0)
+    cand, err0, sp0 = r["coarse"]
+    np.testing.assert_allclose(cand[0], mags[:3], rtol=1e-14)
+    e2 = 0.5 * mags[0] / (mags[0] + mags[1])
+    np.testing.assert_allclose(err0[0], [0.0, e2, 0.5], rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(sp0[0], [0.0, 0.25, 0.5], rtol=0, atol=0)
+    fine = r["fine"][0][0, 3:]
+    expect = [lo(mags) + (hi(mags) - lo(mags)) * k / 4.0 for k in (1, 2, 3)]
+    np.testing.assert_allclose(fine, expect, rtol=1e-13)
+
+
+def test_final_choice_can_be_a_fine_candidate(oracle):
+    # s_tar = 0.7: the coarse S(b) takes 0, 1/4 and 1/2, so the coarse choice is t3 = SiLU(1) and the
+    # fine candidates lie between t2 and SiLU(2):
+    #   f1 = t2 + (SiLU(2) - t2) / 4  (below SiLU(1): token 0 keeps both, token 1 none: err 1/2, sp 1/2)
+    #   f2, f3 above SiLU(1): token 0 also loses SiLU(1): err (SiLU(1) / (SiLU(1) + SiLU(2)) + 1) / 2, sp 3/4
+    # Over coarse and fine candidates S(b) takes 0, 1/4, 1/2 (at b = 1/2, t*(1/2) = t3, which is
+    # larger than f1) and 3/4 (at b = that error: t* = f3, the largest admissible); 3/4 is the
+    # closest to 0.7, so the block takes f3.  At s_tar = 0.45 the same table gives 1/2 and t3.
+    x, Wg, Wu, Wd, nw = _worked_block()
+    m = [abs(_silu(-2.0)), abs(_silu(-1.0)), _silu(1.0), _silu(2.0)]
+    r = oracle.sats_calibrate(x, [Wg], [Wu], [Wd], nw, 0.0, 0.7, K0=4, K1=3, guardrail=False, err_eps=0.0)
+    f3 = m[1] + (m[3] - m[1]) * 3.0 / 4.0
+    e_hi = 0.5 * (m[2] / (m[2] + m[3]) + 1.0)
+    t_all, e_all, s_all = r["fine"]
+    np.testing.assert_allclose(e_all[0, 3:], [0.5, e_hi, e_hi], rtol=1e-12)
+    np.testing.assert_allclose(s_all[0, 3:], [0.5, 0.75, 0.75], rtol=0, atol=0)
+    assert r["t"][0] == pytest.approx(f3, rel=1e-13)
+    assert r["b"] == pytest.approx(e_hi, rel=1e-12) and r["S"] == 0.75
+    r = oracle.sats_calibrate(x, [Wg], [Wu], [Wd], nw, 0.0, 0.45, K0=4, K1=3, guardrail=False, err_eps=0.0)
+    assert r["t"][0] == pytest.approx(m[2], rel=1e-13) and r["S"] == 0.5
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("s_tar", [0.5, 0.97])
+def test_fine_candidates_sit_evenly_between_the_coarse_neighbours(oracle, s_tar):
+    # on a random 3-block stack: for every block but the guardrail block, the K1 fine candidates are
+    # evenly spaced and strictly inside (lower, upper), where lower is the largest coarse candidate
+    # below the coarse choice t*_l (0 if none) and upper the smallest above it (else the block's
+    # largest |a| on its dense-stack inputs).  At s_tar = 0.97, above every coarse sparsity, each
+    # block's coarse choice is its largest candidate, so upper is that block's own largest |a|.
+    L, H, N, C, K0, K1 = 3, 32, 64, 6, 10, 6
+    ws, nw = _stack(L, H, N)
+    x = _x(C, H, seed=11)
+    r = oracle.sats_calibrate(x, [w.Wg for w in ws], [w.Wu for w in ws], [w.Wd for w in ws], nw, 1e-5, s_tar,
+                              K0=K0, K1=K1, guardrail=True)
+    cand, err0, sp0 = r["coarse"]
+    g_t, g_sp = r["guard"]
+    _, t0, _ = oracle.sats_select(cand, err0, sp0, s_tar, L - 1, g_t, g_sp)
+    if s_tar > 0.9:
+        assert np.all(t0[:L - 1] == cand[:L - 1, -1])
+    fine = r["fine"][0][:, K0 - 1:]
+    xs = x.copy()
+    for l in range(L):
+        n = oracle.rmsnorm(xs, nw[l], 1e-5)
+        amax = float(np.abs(oracle.gate_act(n, ws[l].Wg)).max())
+        xs = xs + oracle.dense_mlp(n, ws[l].Wg, ws[l].Wu, ws[l].Wd)
+        if l == L - 1:
+            continue
+        below = cand[l][cand[l] < t0[l]]
+        above = cand[l][cand[l] > t0[l]]
+        lower = below.max() if below.size else 0.0
+        upper = above.min() if above.size else amax
+        f = fine[l]
+        assert np.all(f > lower) and np.all(f < upper)
+        step = (upper - lower) / (K1 + 1)
+        np.testing.assert_allclose(np.diff(np.concatenate([[lower], f, [upper]])), step, rtol=1e-9)
