@@ -12,10 +12,17 @@ than the 129 MB L2).
 The line also carries, under "batched", the same layer at decode-batch and
 prefill sizes (8, 64, 256 and 2048 tokens per call, 50 % threshold), which run
 on the tensor-core path: microseconds per call, tokens/s, weight-stream GB/s
-and dense-equivalent TFLOP/s against the measured bf16 peak.
+and dense-equivalent TFLOP/s against the measured bf16 peak; and, under
+"configs", the other four workloads at full size (the small layer, the
+32-block Llama stack, the 36-block routed Qwen stack at 1 / 8 / 32 / 64 tokens
+per step, the routed prefill block at 256 / 2048 tokens and 40 / 90 %), with
+thresholds from the library's own Eq. 3 kernels.  The CPU oracle is timed on
+one core and over all host cores (threshold recipe as the GPU arm: 256
+calibration vectors).
 
 Prints one JSON line.  `--impl reference` times the CPU oracle instead (the
-reference arm of this comparison), on a bounded sample of the same workload.
+reference arm of this comparison), on a bounded sample of the same workload,
+one decode token per host core at a time.
 """
 from __future__ import annotations
 
@@ -171,57 +178,88 @@ def _us_per_token(total_ms: float, steps: int, calls: int, world: int) -> float:
 
 
 # ---------------------------------------------------------------------------- CPU oracle arm
-def _oracle_sample(budget_s: float, max_calls: int = 64):
-    """Times the oracle on the workload: one token through the layer per call, cycling sparsity levels."""
+def _headline_config(world: int):
+    """The headline workload's config, shared by the GPU arm and the oracle arm."""
+    H, N = inputs.LLAMA_H, inputs.LLAMA_N
+    return {"workload": WORKLOAD, "hidden": H, "intermediate": N, "tokens": 1, "sparsity": list(SPARSITY),
+            "calibration_vectors": N_CALIB,
+            "l2": "inputs larger than L2: %d rotating device copies of the layer (%.2f GB)"
+                  % (LAYER_COPIES, LAYER_COPIES * 6.0 * H * N / 1e9),
+            "parallelism": "replicas" if world > 1 else "single"}
+
+
+def _host_threads() -> int:
+    try:
+        return max(1, len(os.sched_getaffinity(0)))
+    except AttributeError:
+        return max(1, os.cpu_count() or 1)
+
+
+def _oracle_setup():
+    """The oracle's inputs for the headline workload: the layer, decode tokens, and the Eq. 3
+    thresholds at 50 / 70 / 90 % from the same 256 calibration vectors the GPU arm uses (their
+    gate activations computed on a thread pool over the host cores; setup, not timed)."""
+    import concurrent.futures
+
     import oracle
     oracle.build()
     H, N = inputs.LLAMA_H, inputs.LLAMA_N
     w = inputs.mlp_weights(H, N)
-    x = oracle.bf16_to_f64(inputs.activations_bf16(1, H))
-    cal = oracle.bf16_to_f64(inputs.activations_bf16(4, H, seed=inputs.SEED_CALIB))
-    a_cal = oracle.gate_act(cal, w.Wg)
+    cal = oracle.bf16_to_f64(inputs.activations_bf16(N_CALIB, H, seed=inputs.SEED_CALIB))
+    with concurrent.futures.ThreadPoolExecutor(_host_threads()) as ex:   # the C oracle releases the GIL
+        parts = list(ex.map(lambda c: oracle.gate_act(cal[c:c + 4], w.Wg), range(0, N_CALIB, 4)))
+    a_cal = np.concatenate(parts)
     ts = [oracle.percentile_threshold(a_cal, s) for s in SPARSITY]
+    return oracle, w, ts
+
+
+def _oracle_one_core(orc, w, ts, budget_s: float, max_calls: int = 64):
+    """The oracle on one core: one token through the layer per call, sparsity levels cycling."""
+    x = orc.bf16_to_f64(inputs.activations_bf16(1, inputs.LLAMA_H))
     times = []
     t_all = time.perf_counter()
     i = 0
     while i < max_calls and (i < len(SPARSITY) or time.perf_counter() - t_all < budget_s):
         t0 = time.perf_counter()
-        oracle.sparse_mlp(x, w.Wg, w.Wu, w.Wd, ts[i % len(SPARSITY)])
+        orc.sparse_mlp(x, w.Wg, w.Wu, w.Wd, ts[i % len(SPARSITY)])
         times.append(time.perf_counter() - t0)
         i += 1
     us = 1e6 * sum(times) / len(times)
-    return us, len(times), "%d single-token calls (hidden 4096, intermediate 14336, thresholds at %s " \
-                           "sparsity from 4 calibration vectors)" % (len(times), "/".join(str(s) for s in SPARSITY))
+    sample = ("%d single-token calls on one core (hidden 4096, intermediate 14336, thresholds at %s sparsity "
+              "from 256 calibration vectors)" % (len(times), "/".join(str(s) for s in SPARSITY)))
+    return us, sample
+
+
+def _oracle_all_cores(orc, w, ts, rounds: int, threads: int):
+    """The oracle over the host cores: `threads` decode tokens at a time, one per thread (the C
+    oracle releases the GIL), sparsity levels cycling over the tokens; us per token of wall time."""
+    import concurrent.futures
+    T = rounds * threads
+    xs = orc.bf16_to_f64(inputs.activations_bf16(T, inputs.LLAMA_H, seed=inputs.SEED_X + 9))
+    with concurrent.futures.ThreadPoolExecutor(threads) as ex:
+        t0 = time.perf_counter()
+        list(ex.map(lambda i: orc.sparse_mlp(xs[i:i + 1], w.Wg, w.Wu, w.Wd, ts[i % len(SPARSITY)]), range(T)))
+        el = time.perf_counter() - t0
+    return 1e6 * el / T, el
 
 
 def run_reference(args):
-    ws, rank, _ = _dist_env()
+    world, rank, _ = _dist_env()
     if rank != 0:
         return
-    import oracle
-    oracle.build()
-    H, N = inputs.LLAMA_H, inputs.LLAMA_N
-    w = inputs.mlp_weights(H, N)
-    x = oracle.bf16_to_f64(inputs.activations_bf16(1, H))
-    cal = oracle.bf16_to_f64(inputs.activations_bf16(4, H, seed=inputs.SEED_CALIB))
-    a_cal = oracle.gate_act(cal, w.Wg)
-    ts = [oracle.percentile_threshold(a_cal, s) for s in SPARSITY]
-    # one step = one token through the layer at one sparsity level (cycling), a bounded sample
-    for i in range(args.warmup):
-        oracle.sparse_mlp(x, w.Wg, w.Wu, w.Wd, ts[i % 3])
-    t0 = time.perf_counter()
-    for i in range(args.steps):
-        oracle.sparse_mlp(x, w.Wg, w.Wu, w.Wd, ts[i % 3])
-    el = time.perf_counter() - t0
-    us = 1e6 * el / args.steps
-    sample = "%d single-token calls of the layer, sparsity cycling %s" % (args.steps, "/".join(map(str, SPARSITY)))
+    orc, w, ts = _oracle_setup()
+    threads = _host_threads()
+    # one step = one decode token per host core, all at once (sparsity levels cycling); a bounded sample
+    _oracle_all_cores(orc, w, ts, max(args.warmup, 1), threads)
+    us, el = _oracle_all_cores(orc, w, ts, args.steps, threads)
+    sample = ("%d steps of %d single-token calls in parallel (one per host core), sparsity cycling %s, thresholds "
+              "from 256 calibration vectors" % (args.steps, threads, "/".join(map(str, SPARSITY))))
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": us, "unit": "us/token", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
         "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": WORKLOAD, "hidden": H, "intermediate": N, "tokens": 1,
-                                        "sparsity": list(SPARSITY)},
-        "cpu_baseline": {"value": us, "unit": "us/token", "cores": 1, "kind": "oracle", "sample": sample},
+        "data": "synthetic", "config": _headline_config(world),
+        "cpu_baseline": {"value": us, "unit": "us/token", "cores": threads, "kind": "oracle", "sample": sample},
         "e2e": {"value": us, "unit": "us/token", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 
@@ -418,6 +456,29 @@ def run_gpu(args):
     stream.synchronize()
     e2e_us = 1e3 * e2e_s.elapsed_time(e2e_e) / (Ke * nc)
 
+    # the other four workloads at their full sizes, compact (one GPU; not part of the headline value)
+    configs = {}
+    if not args.no_configs and world == 1:
+        for l in layers:
+            l.close()
+        layers = []
+        hbm_peak, peak_kind = _peaks()
+        bf16_peak, bf16_kind = _bf16_peak()
+        t_cfg = time.perf_counter()
+        clk_cfg = Clocks(local)
+        clk_cfg.start()
+        with torch.cuda.stream(stream):
+            configs["small_layer_512x1408_b1"] = _wl_small_layer(sats, dev, stream, 200)
+            configs["llama_stack_32x4096x14336_b1x128"] = _wl_llama_stack(sats, dev, stream, 128, hbm_peak,
+                                                                          peak_kind)
+            torch.cuda.empty_cache()
+            configs["qwen_stack_36x4096x12288_routed"] = _wl_qwen_stack(sats, dev, stream, [1, 8, 32, 64], 10)
+            torch.cuda.empty_cache()
+            configs["llama_layer_prefill_routed"] = _wl_prefill(sats, dev, stream, [0.4, 0.9], [256, 2048], 10,
+                                                                bf16_peak, bf16_kind)
+        configs["clocks"] = clk_cfg.stop()
+        configs["seconds"] = time.perf_counter() - t_cfg
+
     # aggregate over ranks (replicas): max time
     total_ms, e2e_us = _max_over_ranks([total_ms, e2e_us], world, device=dev)
     if rank == 0:
@@ -440,11 +501,7 @@ def run_gpu(args):
             "metric": METRIC, "value": value, "unit": "us/token", "n_gpus": world, "steps": K,
             "warmup": max(args.warmup, 3), "ms_per_step": total_ms / K, "higher_is_better": False,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "hidden": H, "intermediate": N, "tokens": 1,
-                       "sparsity": list(SPARSITY), "calibration_vectors": N_CALIB,
-                       "l2": "inputs larger than L2: %d rotating device copies of the layer (%.2f GB)"
-                             % (LAYER_COPIES, LAYER_COPIES * 6.0 * H * N / 1e9),
-                       "parallelism": "replicas" if world > 1 else "single"},
+            "config": _headline_config(world),
             "per_sparsity": per,
             "dense": {"us": dense_us},
             "batched": batched,
@@ -458,9 +515,18 @@ def run_gpu(args):
             "gpu_launches": K * len(calls),
             "clocks": clk,
         }
+        if configs:
+            line["configs"] = configs
         if not args.no_cpu_baseline:
-            us, n, sample = _oracle_sample(args.cpu_seconds)
+            orc, w_or, ts_or = _oracle_setup()
+            us, sample = _oracle_one_core(orc, w_or, ts_or, args.cpu_seconds)
             line["cpu_baseline"] = {"value": us, "unit": "us/token", "cores": 1, "kind": "oracle", "sample": sample}
+            threads = _host_threads()
+            us_all, _ = _oracle_all_cores(orc, w_or, ts_or, 2, threads)
+            line["cpu_baseline_all_cores"] = {
+                "value": us_all, "unit": "us/token", "cores": threads, "os_cpu_count": os.cpu_count(),
+                "kind": "oracle", "sample": "%d single-token calls, %d at a time (one per host core)"
+                                            % (2 * threads, threads)}
         print(json.dumps(line))
     for l in layers:
         l.close()
@@ -469,27 +535,27 @@ def run_gpu(args):
 
 
 # ---------------------------------------------------------------------------- other workloads
-def _calibrate_stack(sats, layers, nws, targets, eps, xc, ws, stream, N):
-    """Per-layer thresholds for the bench (setup, not timed, not a parity input): bisection on t
-    until the kept fraction of the calibration vectors, carried through the earlier blocks,
-    meets the layer's target sparsity (the Eq. 3 percentile, found through the library)."""
+def _eq3_stack_thresholds(sats, layers, nws, targets, eps, xc, stream):
+    """Per-block thresholds for the bench (setup, not timed, not a parity input): the Eq. 3
+    percentile of the post-gate magnitudes of fp32 calibration vectors carried through the
+    earlier, already thresholded blocks, computed with the library's own RMSNorm, gate and
+    percentile kernels."""
     import torch
-    C = xc.shape[0]
-    trace = torch.empty((1, C, N), dtype=torch.uint8, device=xc.device)
+    C, H = xc.shape
+    N = layers[0].N
+    x = xc.clone()
+    n = torch.empty_like(x)
+    a = torch.empty(C, N, dtype=torch.float32, device=x.device)
+    sel = torch.empty(sats.select_workspace_bytes(), dtype=torch.uint8, device=x.device)
+    ws = sats.Workspace(H, N, C, device=x.device, stream=stream)
     ts = []
     for l, layer in enumerate(layers):
-        lo, hi = 0.0, 16.0
-        for _ in range(24):
-            mid = 0.5 * (lo + hi)
-            xt = xc.clone()
-            sats.mlp_stack([layer], [nws[l]], [mid], eps, xt, ws, keep_trace=trace, stream=stream)
-            sp = 1.0 - float(trace.float().mean())
-            if sp < targets[l]:
-                lo = mid
-            else:
-                hi = mid
-        ts.append(hi)
-        sats.mlp_stack([layer], [nws[l]], [hi], eps, xc, ws, stream=stream)
+        sats.rmsnorm(x, nws[l], eps, n, stream=stream)
+        sats.gate_act_f32(layer, n, a, stream=stream)
+        t = sats.percentile_threshold(a, float(targets[l]), sel, stream=stream)
+        ts.append(t)
+        sats.mlp_stack([layer], [nws[l]], [t], eps, x, ws, stream=stream)
+    stream.synchronize()
     return ts
 
 
@@ -502,6 +568,192 @@ def _timed(stream, fn, reps):
     e1.record(stream)
     e1.synchronize()
     return 1e3 * e0.elapsed_time(e1) / reps
+
+
+def _graph_timed(stream, fn, n_calls, reps):
+    """Device time per call of `n_calls` calls captured once into a CUDA graph and replayed
+    `reps` times back to back (for calls shorter than the host's launch time)."""
+    import torch
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(n_calls):
+            fn(i)
+    stream.synchronize()
+    with torch.cuda.stream(stream):
+        g.replay()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+    e1.synchronize()
+    return 1e3 * e0.elapsed_time(e1) / (reps * n_calls)
+
+
+def _wl_small_layer(sats, dev, stream, steps):
+    """Hidden 512 / intermediate 1408, one decode token, t at the 50th percentile of 64 calibration
+    vectors; 64 rotating copies of the layer (184 MB, weights from HBM) and one copy (L2-resident)."""
+    import torch
+    spec = inputs.WORKLOADS["small_layer_512x1408_b1"]
+    H, N = spec["H"], spec["N"]
+    layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l), stream=stream) for l in range(64)]
+    ws = sats.Workspace(H, N, 1, device=dev, stream=stream)
+    xc = torch.from_numpy(inputs.activations_bf16(spec["calib"], H, seed=inputs.SEED_CALIB).view(np.int16)).to(dev)
+    a = torch.empty(spec["calib"], N, dtype=torch.float32, device=dev)
+    sats.gate_act(layers[0], xc, a, stream=stream)
+    sel = torch.empty(sats.select_workspace_bytes(), dtype=torch.uint8, device=dev)
+    t = sats.percentile_threshold(a, 0.5, sel, stream=stream)
+    x = torch.from_numpy(inputs.activations_bf16(1, H).view(np.int16)).to(dev)
+    y = torch.empty(1, H, dtype=torch.float32, device=dev)
+    idx = torch.empty(1, N, dtype=torch.int32, device=dev)
+    cnt = torch.empty(1, dtype=torch.int32, device=dev)
+    call = lambda i: sats.sparse_mlp(layers[i % 64], x, t, y, ws, idx, cnt, stream=stream)
+    for i in range(64):
+        call(i)
+    stream.synchronize()
+    kept = int(cnt.item())
+    # a call of this layer is shorter than the host's launch time: the device time comes from
+    # 64 calls (one per copy) captured in a CUDA graph and replayed; the eagerly launched loop
+    # is reported beside it
+    us_cold = _graph_timed(stream, call, 64, max(4, steps // 64))
+    us_hot = _graph_timed(stream, lambda i: call(0), 64, max(4, steps // 64))
+    us_eager = _timed(stream, call, steps)
+    if sats.get_error(ws, stream=stream) != sats.OK:
+        raise RuntimeError("device status after the small-layer calls")
+    for l in layers:
+        l.close()
+    algo = 2.0 * H * N + 4.0 * H * kept + 2.0 * H + 4.0 * H + 4.0 * kept + 4.0
+    return {"us_per_token": us_cold, "us_l2_resident": us_hot, "us_per_token_eager_launches": us_eager,
+            "timing": "64 calls (64 rotating layer copies, 184 MB) in a CUDA graph, replayed back to back",
+            "realised_sparsity": 1.0 - kept / N, "algo_bytes": algo, "achieved_gbs": algo / us_cold / 1e3,
+            "calls": 64 * max(4, steps // 64)}
+
+
+def _wl_llama_stack(sats, dev, stream, tokens, hbm_peak, hbm_kind):
+    """32 Llama-3.1-8B-shaped blocks (RMSNorm -> MLP -> residual), `tokens` decode tokens one per
+    call, per-block targets evenly spread over [55 %, 85 %] (mean 70 %)."""
+    import torch
+    spec = inputs.WORKLOADS["llama_stack_32x4096x14336_b1x128"]
+    H, N, L, eps = spec["H"], spec["N"], spec["L"], spec["eps"]
+    targets = list(inputs.stack_sparsity_targets(L, *spec["sparsity_range"]))
+    layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l), stream=stream) for l in range(L)]
+    nws = [torch.from_numpy(inputs.norm_weight(H, layer=l)).to(dev) for l in range(L)]
+    xc = torch.from_numpy(inputs.activations_f32(64, H, seed=inputs.SEED_CALIB)).to(dev)
+    ts = _eq3_stack_thresholds(sats, layers, nws, targets, eps, xc, stream)
+    x0 = torch.from_numpy(inputs.activations_f32(tokens, H, seed=inputs.SEED_X + 3)).to(dev)
+    ws = sats.Workspace(H, N, 1, device=dev, stream=stream)
+    trace = torch.empty((L, 1, N), dtype=torch.uint8, device=dev)
+    kept_sum = torch.zeros(L, dtype=torch.float64, device=dev)
+    x = x0.clone()
+    for tok in range(tokens):      # keep masks of every token (untimed), for the realised sparsity
+        sats.mlp_stack(layers, nws, ts, eps, x[tok:tok + 1], ws, keep_trace=trace, stream=stream)
+        with torch.cuda.stream(stream):
+            kept_sum += trace[:, 0].sum(dim=1).double()
+    stream.synchronize()
+    kept = (kept_sum / tokens).cpu().numpy()          # [L] mean kept neurons per token
+    del trace
+    x = x0.clone()
+    step = lambda i: sats.mlp_stack(layers, nws, ts, eps, x[i % tokens:i % tokens + 1], ws, stream=stream)
+    for i in range(3):
+        step(i)
+    x.copy_(x0)
+    us = _timed(stream, step, tokens)      # every token once through the stack
+    if sats.get_error(ws, stream=stream) != sats.OK:
+        raise RuntimeError("device status after the stack calls")
+    for l in layers:
+        l.close()
+    algo = float(sum(2.0 * H * N + 4.0 * H * k + 12.0 * H for k in kept))
+    return {"us_per_token": us, "tokens_per_s": 1e6 / us, "tokens": tokens,
+            "realised_sparsity_mean": float(1.0 - kept.mean() / N),
+            "realised_sparsity_range": [float(1.0 - kept.max() / N), float(1.0 - kept.min() / N)],
+            "algo_bytes_per_token": algo, "achieved_gbs": algo / us / 1e3,
+            "frac_of_%s" % hbm_kind: algo / us / 1e3 / hbm_peak}
+
+
+def _wl_qwen_stack(sats, dev, stream, batches, reps_max):
+    """36 Qwen3-8B-shaped blocks with routing over a 151936-entry table (30 % dense), decode
+    batches of uniform token ids, sparse path at 50 % per block."""
+    import torch
+    spec = inputs.WORKLOADS["qwen_stack_36x4096x12288_routed"]
+    H, N, L, V, eps = spec["H"], spec["N"], spec["L"], spec["V"], spec["eps"]
+    layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l, seed=inputs.SEED_WEIGHTS + 100), stream=stream)
+              for l in range(L)]
+    nws = [torch.from_numpy(inputs.norm_weight(H, layer=l)).to(dev) for l in range(L)]
+    xc = torch.from_numpy(inputs.activations_f32(64, H, seed=inputs.SEED_CALIB)).to(dev)
+    ts = _eq3_stack_thresholds(sats, layers, nws, [spec["sparsity"]] * L, eps, xc, stream)
+    lut = torch.from_numpy(inputs.routing_lut(V, spec["p_dense"])).to(dev)
+    res = {}
+    for B in batches:
+        x0 = torch.from_numpy(inputs.activations_f32(B, H, seed=inputs.SEED_X + 40 + B)).to(dev)
+        ids = torch.from_numpy(inputs.token_ids_uniform(B, V, seed=inputs.SEED_IDS + B)).to(dev)
+        ws = sats.Workspace(H, N, B, device=dev, stream=stream)
+        reps = reps_max
+        xs = x0.repeat(reps + 3, 1, 1)        # a fresh copy of the batch per step
+        step = lambda i: sats.mlp_stack(layers, nws, ts, eps, xs[i], ws, token_ids=ids, lut=lut, stream=stream)
+        for i in range(3):
+            step(reps + i)
+        us = _timed(stream, step, reps)
+        if sats.get_error(ws, stream=stream) != sats.OK:
+            raise RuntimeError("device status after the routed stack calls")
+        res[str(B)] = {"us_per_step": us, "tokens_per_s": B / (us * 1e-6),
+                       "dense_tokens": int(lut[ids.long()].sum()),
+                       "path": "tensor cores" if sats.uses_tensor_cores(H, B) else "fused",
+                       "weight_gbs_if_all_weights_read": L * 6.0 * H * N / us / 1e3}
+        del xs, ws
+    for l in layers:
+        l.close()
+    return res
+
+
+def _wl_prefill(sats, dev, stream, sparsities, batches, reps_max, bf16_peak, bf16_kind):
+    """One Llama-shaped block with routing (20 % of a 128256-entry table dense, Zipf(1.1) ids) at
+    prefill sizes; dense-equivalent and method-work (algorithmic) FLOP rates."""
+    import torch
+    spec = inputs.WORKLOADS["llama_layer_prefill_routed"]
+    H, N, V = inputs.LLAMA_H, inputs.LLAMA_N, spec["V"]
+    eps = 1e-5
+    layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l, seed=inputs.SEED_WEIGHTS + 200), stream=stream)
+              for l in range(2)]
+    nw = torch.from_numpy(inputs.norm_weight(H)).to(dev)
+    lut = torch.from_numpy(inputs.routing_lut(V, spec["p_dense"], seed=inputs.SEED_LUT + 5)).to(dev)
+    xc = torch.from_numpy(inputs.activations_f32(256, H, seed=inputs.SEED_CALIB)).to(dev)
+    res = {}
+    for k in sparsities:
+        t = _eq3_stack_thresholds(sats, layers[:1], [nw], [k], eps, xc, stream)[0]
+        for B in batches:
+            ids = torch.from_numpy(inputs.token_ids_zipf(B, V, seed=inputs.SEED_IDS + B)).to(dev)
+            x0 = torch.from_numpy(inputs.activations_f32(B, H, seed=inputs.SEED_X + 50 + B)).to(dev)
+            ws = sats.Workspace(H, N, B, device=dev, stream=stream)
+            dense = lut[ids.long()].bool()
+            trace = torch.empty((1, B, N), dtype=torch.uint8, device=dev)
+            xt = x0.clone()
+            sats.mlp_stack([layers[0]], [nw], [t], eps, xt, ws, token_ids=ids, lut=lut, keep_trace=trace,
+                           stream=stream)
+            kept_sparse = float(trace[0][~dense].double().mean()) if bool((~dense).any()) else 0.0
+            nd = int(dense.sum())
+            del trace, xt
+            reps = max(4, min(reps_max, int(2e4 / B)))
+            xs = x0.repeat(reps + 3, 1, 1)
+            step = lambda i: sats.mlp_stack([layers[i % 2]], [nw], [t], eps, xs[i], ws, token_ids=ids, lut=lut,
+                                            stream=stream)
+            for i in range(3):
+                step(reps + i)
+            us = _timed(stream, step, reps)
+            if sats.get_error(ws, stream=stream) != sats.OK:
+                raise RuntimeError("device status after the prefill calls")
+            flops = 6.0 * B * H * N
+            method = nd * 6.0 * H * N + (B - nd) * (2.0 + 4.0 * kept_sparse) * H * N
+            res["%s@%d" % (k, B)] = {"us_per_call": us, "tokens_per_s": B / (us * 1e-6),
+                                     "tflops_dense_equivalent": flops / us / 1e6,
+                                     "tensor_frac_of_%s" % bf16_kind: flops / us / 1e6 / bf16_peak,
+                                     "method_tflops": method / us / 1e6,
+                                     "method_frac_of_%s" % bf16_kind: method / us / 1e6 / bf16_peak,
+                                     "dense_fraction_of_tokens": nd / B,
+                                     "sparse_tokens_realised_sparsity": 1.0 - kept_sparse}
+            del xs, ws
+    for l in layers:
+        l.close()
+    return res
 
 
 def run_workload(args):
@@ -524,125 +776,27 @@ def run_workload(args):
     clocks = Clocks(0)
     with torch.cuda.stream(stream):
         if wl == "small_layer_512x1408_b1":
-            H, N = spec["H"], spec["N"]
-            layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l)) for l in range(64)]
-            ws = sats.Workspace(H, N, 1, device=dev)
-            xc = torch.from_numpy(inputs.activations_bf16(64, H, seed=inputs.SEED_CALIB).view(np.int16)).to(dev)
-            a = torch.empty(64, N, dtype=torch.float32, device=dev)
-            sats.gate_act(layers[0], xc, a, stream=stream)
-            sel = torch.empty(sats.select_workspace_bytes(), dtype=torch.uint8, device=dev)
-            t = sats.percentile_threshold(a, 0.5, sel, stream=stream)
-            x = torch.from_numpy(inputs.activations_bf16(1, H).view(np.int16)).to(dev)
-            y = torch.empty(1, H, dtype=torch.float32, device=dev)
-            idx = torch.empty(1, N, dtype=torch.int32, device=dev)
-            cnt = torch.empty(1, dtype=torch.int32, device=dev)
-            call = lambda i: sats.sparse_mlp(layers[i % 64], x, t, y, ws, idx, cnt, stream=stream)
-            for i in range(64):
-                call(i)
-            stream.synchronize()
-            kept = int(cnt.item())
             clocks.start()
-            us_cold = _timed(stream, call, args.steps)       # 64 rotating copies (184 MB): weights from HBM
-            us_hot = _timed(stream, lambda i: call(0), args.steps)   # one copy, L2-resident
+            r = _wl_small_layer(sats, dev, stream, args.steps)
             clk = clocks.stop()
-            algo = 2.0 * H * N + 4.0 * H * kept + 2.0 * H + 4.0 * H + 4.0 * kept + 4.0
-            out.update({"metric": "us/token (one layer)", "value": us_cold, "unit": "us/token",
-                        "us_l2_resident": us_hot, "realised_sparsity": 1.0 - kept / N, "algo_bytes": algo,
-                        "achieved_gbs": algo / us_cold / 1e3, "clocks": clk})
-        elif wl in ("llama_stack_32x4096x14336_b1x128", "qwen_stack_36x4096x12288_routed"):
-            H, N, L, eps = spec["H"], spec["N"], spec["L"], spec["eps"]
-            if wl.startswith("llama"):
-                targets = list(inputs.stack_sparsity_targets(L, *spec["sparsity_range"]))
-                seed = inputs.SEED_WEIGHTS
-            else:
-                targets = [spec["sparsity"]] * L
-                seed = inputs.SEED_WEIGHTS + 100
-            layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l, seed=seed)) for l in range(L)]
-            nws = [torch.from_numpy(inputs.norm_weight(H, layer=l)).to(dev) for l in range(L)]
-            xc = torch.from_numpy(inputs.activations_f32(8, H, seed=inputs.SEED_CALIB)).to(dev)
-            wsc = sats.Workspace(H, N, 8, device=dev)
-            ts = _calibrate_stack(sats, layers, nws, targets, eps, xc, wsc, stream, N)
-            if wl.startswith("llama"):
-                T = spec["tokens"]
-                x0 = torch.from_numpy(inputs.activations_f32(T, H, seed=inputs.SEED_X + 3)).to(dev)
-                ws = sats.Workspace(H, N, 1, device=dev)
-                trace = torch.empty((L, 1, N), dtype=torch.uint8, device=dev)
-                kept = []
-                x = x0.clone()
-                for tok in range(T):
-                    sats.mlp_stack(layers, nws, ts, eps, x[tok:tok + 1], ws, keep_trace=trace, stream=stream)
-                    kept.append(trace.sum(dim=(1, 2)).double())
-                kept = torch.stack(kept).mean(dim=0).cpu().numpy()          # [L] mean kept neurons
-                x = x0.clone()
-                step = lambda i: sats.mlp_stack(layers, nws, ts, eps, x[i:i + 1], ws, stream=stream)
-                for i in range(3):
-                    step(i)
-                x.copy_(x0)
-                clocks.start()
-                us = _timed(stream, step, T)        # the 128 decode tokens, each once through the stack
-                clk = clocks.stop()
-                algo = float(sum(2.0 * H * N + 4.0 * H * k + 12.0 * H for k in kept))
-                out.update({"metric": "us/token through the %d-block stack (decode, one token per call)" % L,
-                            "value": us, "unit": "us/token", "tokens_per_s": 1e6 / us,
-                            "realised_sparsity_mean": float(1.0 - kept.mean() / N),
-                            "realised_sparsity_range": [float(1.0 - kept.max() / N), float(1.0 - kept.min() / N)],
-                            "algo_bytes_per_token": algo, "achieved_gbs": algo / us / 1e3,
-                            "frac_of_%s" % hbm_kind: algo / us / 1e3 / hbm_peak, "clocks": clk})
-            else:
-                V = spec["V"]
-                lut = torch.from_numpy(inputs.routing_lut(V, spec["p_dense"])).to(dev)
-                res = {}
-                clocks.start()
-                for B in spec["batches"]:
-                    x0 = torch.from_numpy(inputs.activations_f32(B, H, seed=inputs.SEED_X + 40 + B)).to(dev)
-                    ids = torch.from_numpy(inputs.token_ids_uniform(B, V, seed=inputs.SEED_IDS + B)).to(dev)
-                    ws = sats.Workspace(H, N, B, device=dev)
-                    reps = max(10, args.steps // 4)
-                    xs = x0.repeat(reps + 3, 1, 1)        # a fresh copy of the batch per step
-                    step = lambda i: sats.mlp_stack(layers, nws, ts, eps, xs[i], ws, token_ids=ids, lut=lut,
-                                                    stream=stream)
-                    for i in range(3):
-                        step(reps + i)
-                    us = _timed(stream, step, reps)
-                    tc = sats.uses_tensor_cores(H, B)
-                    wbytes = L * (6.0 * H * N)
-                    res[str(B)] = {"us_per_step": us, "tokens_per_s": B / (us * 1e-6), "path":
-                                   "tensor cores" if tc else "fused",
-                                   "weight_gbs_if_all_weights_read": wbytes / us / 1e3}
-                clk = clocks.stop()
-                out.update({"metric": "us per decode step through the %d-block routed stack" % L,
-                            "value": res[str(spec["batches"][-1])]["us_per_step"], "unit": "us/step",
-                            "per_batch": res, "thresholds_mean": float(np.mean(ts)), "clocks": clk})
-        elif wl == "llama_layer_prefill_routed":
-            H, N, V = inputs.LLAMA_H, inputs.LLAMA_N, spec["V"]
-            eps = 1e-5
-            layers = [sats.Layer(*inputs.mlp_weights_device(H, N, layer=l, seed=inputs.SEED_WEIGHTS + 200))
-                      for l in range(2)]
-            nw = torch.from_numpy(inputs.norm_weight(H)).to(dev)
-            lut = torch.from_numpy(inputs.routing_lut(V, spec["p_dense"], seed=inputs.SEED_LUT + 5)).to(dev)
-            xc = torch.from_numpy(inputs.activations_f32(8, H, seed=inputs.SEED_CALIB)).to(dev)
-            wsc = sats.Workspace(H, N, 8, device=dev)
-            res = {}
+            out.update({"metric": "us/token (one layer)", "value": r["us_per_token"], "unit": "us/token",
+                        "clocks": clk, **r})
+        elif wl == "llama_stack_32x4096x14336_b1x128":
             clocks.start()
-            for k in spec["sparsity"]:
-                t = _calibrate_stack(sats, layers[:1], [nw], [k], eps, xc.clone(), wsc, stream, N)[0]
-                for B in spec["batches"]:
-                    ids = torch.from_numpy(inputs.token_ids_zipf(B, V, seed=inputs.SEED_IDS + B)).to(dev)
-                    x0 = torch.from_numpy(inputs.activations_f32(B, H, seed=inputs.SEED_X + 50 + B)).to(dev)
-                    ws = sats.Workspace(H, N, B, device=dev)
-                    reps = max(6, min(args.steps, int(4e4 / B)))
-                    xs = x0.repeat(reps + 3, 1, 1)
-                    step = lambda i: sats.mlp_stack([layers[i % 2]], [nw], [t], eps, xs[i], ws, token_ids=ids,
-                                                    lut=lut, stream=stream)
-                    for i in range(3):
-                        step(reps + i)
-                    us = _timed(stream, step, reps)
-                    flops = 6.0 * B * H * N
-                    res["%s@%d" % (k, B)] = {"us_per_call": us, "tokens_per_s": B / (us * 1e-6),
-                                             "tflops_dense_equivalent": flops / us / 1e6,
-                                             "tensor_frac_of_%s" % bf16_kind: flops / us / 1e6 / bf16_peak,
-                                             "dense_fraction_of_tokens":
-                                                 float(lut[ids.long()].float().mean())}
+            r = _wl_llama_stack(sats, dev, stream, spec["tokens"], hbm_peak, hbm_kind)
+            clk = clocks.stop()
+            out.update({"metric": "us/token through the %d-block stack (decode, one token per call)" % spec["L"],
+                        "value": r["us_per_token"], "unit": "us/token", "clocks": clk, **r})
+        elif wl == "qwen_stack_36x4096x12288_routed":
+            clocks.start()
+            res = _wl_qwen_stack(sats, dev, stream, spec["batches"], max(10, args.steps // 4))
+            clk = clocks.stop()
+            out.update({"metric": "us per decode step through the %d-block routed stack" % spec["L"],
+                        "value": res[str(spec["batches"][-1])]["us_per_step"], "unit": "us/step",
+                        "per_batch": res, "clocks": clk})
+        elif wl == "llama_layer_prefill_routed":
+            clocks.start()
+            res = _wl_prefill(sats, dev, stream, spec["sparsity"], spec["batches"], args.steps, bf16_peak, bf16_kind)
             clk = clocks.stop()
             out.update({"metric": "us per prefill call (one routed block)", "value": res["0.6@2048"]["us_per_call"],
                         "unit": "us/call", "per_case": res, "clocks": clk})
@@ -802,6 +956,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-batched", action="store_true", help="skip the batched tensor-core measurements")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the compact measurements of the other four workloads in the headline line")
     ap.add_argument("--workload", default=WORKLOAD, choices=sorted(inputs.WORKLOADS),
                     help="the headline workload (default) or one of the other four, reported on their own line")
     ap.add_argument("--profile-batch", type=int, default=0,
@@ -812,6 +968,7 @@ def main():
     if args.profile or args.profile_batch:
         args.no_cpu_baseline = True
         args.no_batched = True
+        args.no_configs = True
     if args.impl == "reference":
         run_reference(args)
     elif args.workload != WORKLOAD:

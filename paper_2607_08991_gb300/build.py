@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libsats.so")
-SOURCES = ["fused_mlp.cu", "gemm_tc.cu", "union_mlp.cu", "aux_kernels.cu", "calib.cu", "api.cu"]
+SOURCES = ["fused_mlp.cu", "small_mlp.cu", "gemm_tc.cu", "union_mlp.cu", "aux_kernels.cu", "calib.cu", "api.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

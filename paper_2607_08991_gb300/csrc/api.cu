@@ -62,8 +62,8 @@ static sats_status from_cuda(cudaError_t e, const char *where = "CUDA call")
 static bool bad_threshold(float t) { return std::isnan(t) || t < 0.0f; }
 
 // Runs one block over B tokens: on the tensor cores when the batch is larger
-// than one pass of the fused kernel, else the fused kernel in passes of
-// fused_tokens_per_pass(H) tokens.
+// than one pass of the fused kernel, else in passes of fused_tokens_per_pass(H)
+// tokens of the fused kernel (of the small-layer kernel for small layers).
 sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B, const float *t_per_pass_l,
                       const float *norm_w, float eps, const uint8_t *dense_flags, int out_mode, float *out,
                       int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws, cudaStream_t stream,
@@ -109,6 +109,11 @@ sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B,
             p.lora_r = lora->r;
             p.lora_scale = lora->scale;
             p.lora_z = reinterpret_cast<float *>(base + L.lora_z);
+        }
+        if (!lora && use_small_path(H, N, p.nb)) {
+            const cudaError_t e = launch_small(p, stream);
+            if (e != cudaSuccess) return cuda_fail(e, "small-layer kernel launch");
+            continue;
         }
         const cudaError_t e = launch_fused(p, stream);
         if (e != cudaSuccess) return cuda_fail(e, "fused kernel launch");

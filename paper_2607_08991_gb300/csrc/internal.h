@@ -106,6 +106,11 @@ sats_status cuda_fail(cudaError_t e, const char *where);
 int fused_grid(int nchunks);
 int fused_tokens_per_pass(int H);
 cudaError_t launch_fused(const FusedParams &p, cudaStream_t stream);
+// small_mlp.cu: a pass of nb <= 2 tokens on a small layer (hidden <= 1024, a few thousand
+// neurons; use_small_path says which) runs as one thread-block cluster with no workspace use
+// beyond the status word.
+bool use_small_path(int H, int N, int nb);
+cudaError_t launch_small(const FusedParams &p, cudaStream_t stream);
 
 cudaError_t launch_pack(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd, int H, int N,
                         uint16_t *wg_t, uint16_t *w_ud, cudaStream_t stream);
