@@ -23,8 +23,8 @@ WsLayout ws_layout(int H, int N, int B)
     off += align256(kCtlInts * sizeof(int));
     L.lora_z = off;   // cleared with the control words; the fused kernel's last CTA clears it after a LoRA call
     off += align256((size_t)kLoraZCopies * kMaxTokensPerPass * 2 * kMaxLoraRank * sizeof(float));
-    L.flags = off;   // one 64-bit word per chunk of kChunk neurons, then one per CTA of the fused grid
-    off += align256(((size_t)nchunks_of(N) + kMaxGrid) * sizeof(uint64_t));
+    L.flags = off;   // one 64-bit word per chunk of kChunk neurons (the fused kernel's index-list words)
+    off += align256((size_t)nchunks_of(N) * sizeof(uint64_t));
     L.route_perm = off;
     off += align256((size_t)(B > 0 ? B : 1) * sizeof(int32_t));
     L.route_flags = off;

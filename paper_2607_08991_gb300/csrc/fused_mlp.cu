@@ -29,13 +29,13 @@
 //     applies SiLU (Eq. 2) and the mask (Eqs. 4-5) per token, publishes the
 //     chunk's kept counts, frees the buffer, and streams the W_ud rows of the
 //     kept neurons into the W_ud ring (4 slots of 32 KB).
-//   * index warp: turns the kept rows of its CTA's slice of consecutive chunks
-//     into their entries of the ascending index lists.  A chunk's place in the
-//     list is the number of neurons kept in all earlier chunks: the slice's
-//     counts are summed from its chunks' published words, and the counts of the
-//     slices before it found by a decoupled look-back over the slice words (each
-//     holds a slice's own counts, then its inclusive prefix once known), so the
-//     lists are complete soon after every chunk's gate work is done.
+//   * index warp: waits until every CTA has cleared its chunk words (the words
+//     are then this call's) and tells the gate warps.  Once their stream has
+//     ended, the gate warps turn the kept rows of the CTA's slice of consecutive
+//     chunks into their entries of the ascending index lists: a chunk's place in
+//     the list is the number of neurons kept in all earlier chunks, summed
+//     directly from those chunks' published words (256 threads, one round of
+//     loads once the words are there), so no CTA waits on another's sums.
 //   * 8 up/down warps: thread t owns vectors t, t + 256, ... of the up and
 //     down halves of each W_ud row and keeps its y columns in registers.  The
 //     up dot products of a stage are reduced across these warps through a
@@ -81,28 +81,15 @@ constexpr int kTailLag = 2;                                // ... only kTailLag 
 constexpr int kPendingChunks = 16;                        // chunk words held back until every CTA has cleared its flags
 constexpr int kMaxUdRows = 8;                              // W_ud rows per stage (small H)
 
-// Index-list words (the flags region: nchunks chunk words, then one slice word
-// per CTA; CTA c's slice is chunks [c per, (c + 1) per), per = ceil(nchunks / G)).
-// Chunk word: [63:62] status (0: not yet published this call, kChunkKept:
-// published), [8b + 7:8b] the rows of the chunk kept for token b.  Slice word:
-// [63:62] status (0, kFlagAgg: the slice's own kept counts, kFlagInc: the kept
-// counts of slices 0..c), [61:31] token 1's count, [30:0] token 0's count.
-// Every CTA clears its chunk words and its slice word before it passes its
-// prologue, and the words are written and read only after every CTA has passed
-// it.  A word holds its whole payload, so the accesses are relaxed; a word only
-// moves from 0 to its final value (slice words through kFlagAgg), and every
-// writer of a slice's kFlagInc writes the same value (the prefix is unique).
+// Index-list words (the flags region: one word per chunk; CTA c's slice of the
+// lists is chunks [c per, (c + 1) per), per = ceil(nchunks / G)).  Chunk word:
+// [63:62] status (0: not yet published this call, kChunkKept: published),
+// [8b + 7:8b] the rows of the chunk kept for token b.  Every CTA clears the words
+// of its slice before it passes its prologue, and the words are written and read
+// only after every CTA has passed it.  A word holds its whole payload and moves
+// only from 0 to its final value, so the accesses are relaxed.
 constexpr uint64_t kChunkKept = 1ull << 62;
-constexpr uint64_t kFlagAgg = 1ull << 62;
-constexpr uint64_t kFlagInc = 2ull << 62;
-constexpr uint64_t kFlagPayload = (1ull << 62) - 1ull;   // payloads add field by field (sums stay below 2^31)
-constexpr int kLookWords = kMaxGrid / 32;                 // slice words per lane: one look-back step covers the grid
 
-__device__ __forceinline__ uint64_t make_flag(uint64_t status, uint32_t v0, uint32_t v1)
-{
-    return status | ((uint64_t)(v1 & 0x7FFFFFFFu) << 31) | (uint64_t)(v0 & 0x7FFFFFFFu);
-}
-__device__ __forceinline__ uint32_t flag_value(uint64_t f, int b) { return (uint32_t)(f >> (31 * b)) & 0x7FFFFFFFu; }
 __device__ __forceinline__ uint32_t flag_state(uint64_t f) { return (uint32_t)(f >> 62); }
 __device__ __forceinline__ uint32_t chunk_rows(uint64_t f, int b) { return (uint32_t)(f >> (8 * b)) & 0xFFu; }
 
@@ -140,7 +127,8 @@ struct Shared {
     int pend_chunk[kPendingChunks];
     int abort;
     int seen;                   // the list producer has seen every CTA past its prologue
-    int lend;                   // the list producer has published its last chunk word
+    int flags_ready;            // index warp: 1 once every CTA has cleared its chunk words, -1 if that wait gave up
+    uint32_t ired[kGateWarps][2];   // per-warp kept counts of the chunks before this CTA's slice
     int quiet;                  // roles past their last use of the counters (list producer, index warp)
     int ldone;                  // chunks whose W_ud rows the list producer has issued (read by the gate producer)
 };
@@ -397,6 +385,141 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
     }
 }
 
+// ------------------------------------------------------------------ index lists
+// The chunks [k0, k1) whose index-list entries CTA c writes.
+__device__ __forceinline__ void list_slice(int nch, int &k0, int &k1)
+{
+    const int per = (nch + gridDim.x - 1) / gridDim.x;
+    k0 = min(nch, (int)blockIdx.x * per);
+    k1 = min(nch, k0 + per);
+}
+
+// Waits (bounded, with backoff) until chunk word k is published; returns it, or 0
+// if the wait gave up.
+template <int BT>
+__device__ uint64_t await_word(const FusedParams &p, Shared<BT> &S, int k, unsigned long long t0)
+{
+    uint64_t w;
+    uint32_t ns = 64;
+    while (flag_state(w = ld_relaxed_gpu_u64(p.flags + k)) == 0u) {
+        if (global_ns() - t0 > kWaitLimitNs || *(volatile int *)&S.abort) return 0ull;
+        __nanosleep(ns);
+        ns = min(ns * 2u, 512u);
+    }
+    return w;
+}
+
+// The gate warps, after their stream: the entries of this CTA's slice of the
+// ascending index lists.  The entries of chunk k start at the number of neurons
+// kept in chunks [0, k):
+//   1. every thread sums the kept rows of its chunk words before the slice
+//      (words t, t + 256, ...; eight loads in flight; an unpublished word is
+//      awaited before the thread goes on), then the sums are reduced over the
+//      gate warps;
+//   2. the first gate warp writes the slice's entries from a warp scan of its
+//      chunks' counts, 32 chunks at a time, and the last slice the counts.
+// Chunks are taken in increasing order, so the words before a slice are mostly
+// published by the time this CTA's stream ends; the slices need no word but the
+// chunks', and no CTA waits for another CTA's sums.
+template <int BT>
+__device__ void slice_index_lists(const FusedParams &p, Shared<BT> &S, GroupSync &gs, int t, int lane, int warp)
+{
+    static_assert(BT <= 2, "chunk words carry two tokens' rows");
+    const int N = p.N, nch = p.nchunks;
+    int k0, k1;
+    list_slice(nch, k0, k1);
+    if (k0 >= k1) return;
+    const unsigned long long t0 = global_ns();
+    int ready;
+    while ((ready = *(volatile int *)&S.flags_ready) == 0) {
+        if (global_ns() - t0 > kWaitLimitNs || *(volatile int *)&S.abort) {
+            ready = -1;
+            break;
+        }
+        __nanosleep(64);
+    }
+    bool ok = ready > 0;
+    // 1.
+    uint32_t pre0 = 0, pre1 = 0;
+    for (int k = t; ok && k < k0;) {
+        uint64_t w[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int kk = k + kGateThreads * i;
+            w[i] = kk < k0 ? ld_relaxed_gpu_u64(p.flags + kk) : kChunkKept;
+        }
+        int n = 8;   // the words before the first unpublished one are counted now
+#pragma unroll
+        for (int i = 7; i >= 0; --i)
+            if (flag_state(w[i]) == 0u) n = i;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            if (i < n && k + kGateThreads * i < k0) {
+                pre0 += (uint32_t)__popc(chunk_rows(w[i], 0));
+                if (BT > 1) pre1 += (uint32_t)__popc(chunk_rows(w[i], 1));
+            }
+        }
+        k += kGateThreads * n;
+        if (n < 8 && k < k0) ok = await_word<BT>(p, S, k, t0) != 0ull;
+    }
+    pre0 = (uint32_t)__reduce_add_sync(0xffffffffu, pre0);
+    pre1 = (uint32_t)__reduce_add_sync(0xffffffffu, pre1);
+    if (lane == 0) {
+        S.ired[warp][0] = pre0;
+        S.ired[warp][1] = pre1;
+    }
+    if (!__all_sync(0xffffffffu, ok) && lane == 0) {
+        S.abort = 1;
+        flag_status(p.ctl, kStatusTimeout);
+    }
+    if (!gs(lane, &S.abort) || warp != 0) return;
+    // 2.
+    uint32_t run[2] = {0u, 0u};
+#pragma unroll
+    for (int w = 0; w < kGateWarps; ++w) {
+        run[0] += S.ired[w][0];
+        run[1] += S.ired[w][1];
+    }
+    for (int base = k0; base < k1; base += 32) {
+        const int k = base + lane;
+        uint64_t f = 0ull;
+        bool good = true;
+        if (k < k1) {
+            f = ld_relaxed_gpu_u64(p.flags + k);
+            if (flag_state(f) == 0u) good = (f = await_word<BT>(p, S, k, t0)) != 0ull;
+        }
+        if (!__all_sync(0xffffffffu, good)) {
+            if (lane == 0) {
+                S.abort = 1;
+                flag_status(p.ctl, kStatusTimeout);
+            }
+            return;
+        }
+#pragma unroll
+        for (int b = 0; b < BT; ++b) {
+            uint32_t m = k < k1 ? chunk_rows(f, b) : 0u;
+            const uint32_t cnt = (uint32_t)__popc(m);
+            uint32_t pre = cnt;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t v = __shfl_up_sync(0xffffffffu, pre, o);
+                if (lane >= o) pre += v;
+            }
+            uint32_t pos = run[b] + pre - cnt;
+            for (; m; m &= m - 1u, ++pos) {
+                if (pos < (uint32_t)N) p.active_idx[(size_t)b * N + pos] = k * kChunk + __ffs(m) - 1;
+                else flag_status(p.ctl, kStatusInternal);
+            }
+            run[b] += __shfl_sync(0xffffffffu, pre, 31);
+        }
+    }
+    if (k1 == nch && lane == 0 && p.active_cnt) {
+#pragma unroll
+        for (int b = 0; b < BT; ++b)
+            if (b < p.nb) p.active_cnt[b] = (int)run[b];
+    }
+}
+
 // ------------------------------------------------------------------ gate warps
 template <int BT, int VPT>
 __device__ void gate_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *gring)
@@ -521,6 +644,7 @@ __device__ void gate_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *g
         for (int k = 0; k < adv; ++k)
             if (++stage == kGateStages) { stage = 0; phase ^= 1u; }
     }
+    if (p.active_idx) slice_index_lists<BT>(p, S, gs, t, lane, warp);
 }
 
 // Waits (bounded) until every CTA has passed its prologue.
@@ -644,11 +768,10 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
             reinterpret_cast<float4 *>(p.out)[q] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
     if (p.active_idx) {
-        // clear this CTA's chunk words and slice word (read and written only after every prologue)
-        const int per = (p.nchunks + gridDim.x - 1) / gridDim.x;
-        const int j1 = min(p.nchunks, (int)(blockIdx.x + 1) * per);
-        for (int j = blockIdx.x * per + lane; j < j1; j += 32) p.flags[j] = 0ull;
-        if (lane == 0) p.flags[p.nchunks + blockIdx.x] = 0ull;
+        // clear the chunk words of this CTA's slice (read and written only after every prologue)
+        int j0, j1;
+        list_slice(p.nchunks, j0, j1);
+        for (int j = j0 + lane; j < j1; j += 32) p.flags[j] = 0ull;
     }
     __threadfence();
     bool ok = mbar_wait(&S.xloaded, 0u, &S.abort);
@@ -770,7 +893,6 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         if (lane == 0 && npend > 0) good = publish(-1, 0ull, true) ? 1 : 0;
         ok = __shfl_sync(0xffffffffu, good, 0) != 0;
     }
-    if (lane == 0) *(volatile int *)&S.lend = 1;   // the index warp may poll harder: the stream is ending
     if (ok && mbar_wait(&S.uempty[stage], phase ^ 1u, &S.abort)) {
         if (lane == 0) {
             S.udesc[stage].kind = kEnd;
@@ -790,190 +912,21 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
 }
 
 // ------------------------------------------------------------------ index warp
-// Lane 0 waits (bounded, with backoff, one load at a time so that the words'
-// L2 lines are not flooded) until word w is published; warp-uniform result.
-template <int BT>
-__device__ __forceinline__ bool wait_word(const uint64_t *w, Shared<BT> &S, unsigned long long t0, int lane)
-{
-    int good = 1;
-    if (lane == 0) {
-        uint32_t ns = 64;
-        while (flag_state(ld_relaxed_gpu_u64(w)) == 0u) {
-            if (global_ns() - t0 > kWaitLimitNs || *(volatile int *)&S.abort) {
-                good = 0;
-                break;
-            }
-            __nanosleep(ns);
-            ns = min(ns * 2u, 1024u);
-        }
-    }
-    return __shfl_sync(0xffffffffu, good, 0) != 0;
-}
-
-// The ascending per-token index lists, one slice of chunks per CTA.  The
-// entries of a chunk start at the number of neurons kept in all earlier chunks:
-//   1. the slice's kept counts, summed once each of its chunk words is published
-//      (slices are contiguous in chunk order, and chunks are taken in increasing
-//      order, so slices complete in about that order during the call);
-//   2. the slice's prefix, by a decoupled look-back over the slice words of
-//      the CTAs before it in one step (kMaxGrid words, kLookWords per lane): the
-//      counts of the slices after the nearest published prefix; it publishes its
-//      own prefix and those of the slices it summed;
-//   3. each chunk's entries, from a warp scan of the chunks' counts.
+// Index warp: its only use of the counters is to wait (bounded) until every CTA
+// has cleared its chunk words; it then tells the gate warps (S.flags_ready) and
+// releases the counters.
 template <int BT, bool LORA>
 __device__ void index_warp(const FusedParams &p, Shared<BT> &S, int lane)
 {
-    static_assert(BT <= 2, "slice words carry two tokens' counts");
-    const int N = p.N, nch = p.nchunks, c = blockIdx.x;
-    const int per = (nch + gridDim.x - 1) / gridDim.x;
-    const int k0 = c * per, k1 = min(nch, k0 + per);
+    int k0, k1;
+    list_slice(p.nchunks, k0, k1);
     // the control words and index words belong to the previous call until it has ended
     grid_dependency_wait();
-    // no lists, or no chunks (only slices after the last chunk are empty)
-    const bool work = p.active_idx != nullptr && k0 < k1;
-    int go = 1;
     if (lane == 0) {
-        if (work) go = wait_prologues(p.ctl) ? 1 : 0;   // every word is cleared for this call
-        counters_released<BT, LORA>(p, S);                   // the index warp's only counter read is above
-    }
-    if (!work) return;
-    if (!__shfl_sync(0xffffffffu, go, 0)) {
-        if (lane == 0) S.abort = 1;
-        return;
-    }
-    const unsigned long long t0 = global_ns();
-    uint64_t *sw = p.flags + nch;   // slice words
-    bool ok = true;
-    // 1.
-    uint64_t own = 0, f_first = 0;   // f_first: the words of the slice's first 32 chunks, kept for step 3
-    uint64_t lw[kLookWords];         // step 2's words, read early once this CTA's list producer is done
-    bool have_lw = false;
-    for (int base = k0; base < k1 && ok; base += 32) {
-        const int k = base + lane;
-        uint64_t f;
-        for (;;) {
-            // once this CTA's stream has ended few CTAs still poll: the last reload of the
-            // slice's words also reads the look-back words (one round trip fewer at the end)
-            have_lw = c > 0 && base + 32 >= k1 && *(volatile int *)&S.lend != 0;
-            f = k < k1 ? ld_relaxed_gpu_u64(p.flags + k) : kChunkKept;
-            if (have_lw) {
-#pragma unroll
-                for (int i = 0; i < kLookWords; ++i) {
-                    const int j = c - 1 - (32 * i + lane);
-                    lw[i] = j >= 0 ? ld_relaxed_gpu_u64(p.flags + nch + j) : kFlagInc;
-                }
-            }
-            const uint32_t missing = __ballot_sync(0xffffffffu, flag_state(f) == 0u);
-            if (!missing) break;
-            if (!wait_word<BT>(p.flags + base + __ffs(missing) - 1, S, t0, lane)) { ok = false; break; }
-        }
-        if (base == k0) f_first = f;
-        if (k < k1) own += make_flag(0, __popc(chunk_rows(f, 0)), BT > 1 ? __popc(chunk_rows(f, 1)) : 0u);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) own += __shfl_xor_sync(0xffffffffu, own, o);
-    // 2.
-    uint64_t excl = 0;
-    if (ok && lane == 0) st_relaxed_gpu_u64(sw + c, (c == 0 ? kFlagInc : kFlagAgg) | own);
-    if (ok && c > 0) {
-        // slice c-1-d for d = 32 i + lane
-        uint64_t f[kLookWords];
-#pragma unroll
-        for (int i = 0; i < kLookWords; ++i) {
-            const int j = c - 1 - (32 * i + lane);
-            f[i] = have_lw ? lw[i] : j >= 0 ? ld_relaxed_gpu_u64(sw + j) : kFlagInc;   // before slice 0: 0
-        }
-        for (;;) {
-            int first = 32 * kLookWords, missing = 32 * kLookWords;
-#pragma unroll
-            for (int i = kLookWords - 1; i >= 0; --i) {
-                const uint32_t inc = __ballot_sync(0xffffffffu, flag_state(f[i]) == 2u);
-                const uint32_t unready = __ballot_sync(0xffffffffu, flag_state(f[i]) == 0u);
-                if (inc) first = 32 * i + __ffs(inc) - 1;
-                if (unready) missing = 32 * i + __ffs(unready) - 1;
-            }
-            // first <= c always (the words before slice 0 read as prefix 0); wait for
-            // every unpublished word before the nearest prefix at once (each lane polls
-            // its own, bounded, with backoff) and keep the values the polls read
-            if (missing < first) {
-                bool wait_ok = true;
-#pragma unroll
-                for (int i = 0; i < kLookWords; ++i) {
-                    const int d = 32 * i + lane;
-                    int good = 1;
-                    if (d < first && flag_state(f[i]) == 0u) {
-                        uint32_t ns = 32;
-                        while (flag_state(f[i] = ld_relaxed_gpu_u64(sw + (c - 1 - d))) == 0u) {
-                            if (global_ns() - t0 > kWaitLimitNs || *(volatile int *)&S.abort) { good = 0; break; }
-                            __nanosleep(ns);
-                            ns = min(ns * 2u, 256u);
-                        }
-                    }
-                    wait_ok = __all_sync(0xffffffffu, good) && wait_ok;
-                }
-                if (!wait_ok) { ok = false; break; }
-                continue;
-            }
-            uint64_t part = 0;
-#pragma unroll
-            for (int i = 0; i < kLookWords; ++i)
-                if (32 * i + lane <= first) part += f[i] & kFlagPayload;
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-            excl = part;
-            if (lane == 0) st_relaxed_gpu_u64(sw + c, kFlagInc | (excl + own));
-            // slice c-1-d (d < first) ends at excl minus the slices after it
-            uint64_t after = 0;
-#pragma unroll
-            for (int i = 0; i < kLookWords; ++i) {
-                const int d = 32 * i + lane;
-                const uint64_t v = d < first ? (f[i] & kFlagPayload) : 0ull;
-                uint64_t incl = v;
-#pragma unroll
-                for (int o = 1; o < 32; o <<= 1) {
-                    const uint64_t t = __shfl_up_sync(0xffffffffu, incl, o);
-                    if (lane >= o) incl += t;
-                }
-                if (d < first) st_relaxed_gpu_u64(sw + (c - 1 - d), kFlagInc | (excl - (after + incl - v)));
-                after += __shfl_sync(0xffffffffu, incl, 31);
-            }
-            break;
-        }
-    }
-    if (!ok) {
-        if (lane == 0) {
-            S.abort = 1;
-            flag_status(p.ctl, kStatusTimeout);
-        }
-        return;
-    }
-    // 3.
-    uint32_t run[2] = {flag_value(excl, 0), flag_value(excl, 1)};
-    for (int base = k0; base < k1; base += 32) {
-        const int k = base + lane;
-        const uint64_t f = k >= k1 ? 0ull : (base == k0 ? f_first : ld_relaxed_gpu_u64(p.flags + k));
-#pragma unroll
-        for (int b = 0; b < BT; ++b) {
-            uint32_t m = k < k1 ? chunk_rows(f, b) : 0u;
-            const uint32_t cnt = (uint32_t)__popc(m);
-            uint32_t pre = cnt;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const uint32_t t = __shfl_up_sync(0xffffffffu, pre, o);
-                if (lane >= o) pre += t;
-            }
-            uint32_t pos = run[b > 0 ? 1 : 0] + pre - cnt;
-            for (; m; m &= m - 1u, ++pos) {
-                if (pos < (uint32_t)N) p.active_idx[(size_t)b * N + pos] = k * kChunk + __ffs(m) - 1;
-                else flag_status(p.ctl, kStatusInternal);
-            }
-            run[b > 0 ? 1 : 0] += __shfl_sync(0xffffffffu, pre, 31);
-        }
-    }
-    if (k1 == nch && lane == 0 && p.active_cnt) {
-#pragma unroll
-        for (int b = 0; b < BT; ++b)
-            if (b < p.nb) p.active_cnt[b] = (int)run[b > 0 ? 1 : 0];
+        int ready = 1;
+        if (p.active_idx && k0 < k1) ready = wait_prologues(p.ctl) ? 1 : -1;
+        *(volatile int *)&S.flags_ready = ready;
+        counters_released<BT, LORA>(p, S);
     }
 }
 
@@ -1269,7 +1222,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
         mbar_init(&S.ubar, kUdWarps);
         S.abort = 0;
         S.seen = 0;
-        S.lend = 0;
+        S.flags_ready = 0;
         S.quiet = 0;
         S.ldone = 0;
         mbar_init_fence();

@@ -87,7 +87,7 @@ struct FusedParams {
     int out_mode;
     float *out;                   // kOutY: y [nb][H]; kOutResid: residual [nb][H] (+=)
     int *ctl;                     // workspace control block
-    uint64_t *flags;              // [nchunks + kMaxGrid]: index-list words (index output only)
+    uint64_t *flags;              // [nchunks]: index-list words (index output only)
     int32_t *active_idx;          // [nb][N] or nullptr
     int32_t *active_cnt;          // [nb] or nullptr
     uint8_t *keep_trace;          // [nb][N] or nullptr
