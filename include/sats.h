@@ -28,6 +28,17 @@
  *     sats_get_error.  No call aborts, throws, or traps on the device.
  *   - Calls never allocate device memory, except sats_layer_create.
  *   - Requirements: H a multiple of 8 and 8 <= H <= 8192; N >= 1; B >= 0.
+ *   - SM occupancy: the single-token / two-token decode kernel (the small-batch
+ *     path of sats_sparse_mlp and the calls built on it) runs one CTA on every
+ *     SM (about 216 KB of shared memory each) and its CTAs wait, bounded, for
+ *     one another's prologue.  It needs every SM to become free while it runs:
+ *     a kernel on another stream that holds SMs for longer than 2 s (a
+ *     persistent kernel, or one spinning on a flag) makes the call give up with
+ *     SATS_ETIMEOUT from sats_get_error, and y and the index lists are then
+ *     incomplete.  Ordinary kernels on other streams only delay the call.  The
+ *     kernel is not launched cooperatively: that guarantees co-residency but
+ *     stops the next call from starting on SMs this call frees, which measured
+ *     8 us slower per call on the Llama-shaped layer.
  */
 #ifndef SATS_H
 #define SATS_H
