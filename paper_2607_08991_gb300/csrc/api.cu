@@ -67,13 +67,14 @@ static bool bad_threshold(float t) { return std::isnan(t) || t < 0.0f; }
 sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B, const float *t_per_pass_l,
                       const float *norm_w, float eps, const uint8_t *dense_flags, int out_mode, float *out,
                       int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws, cudaStream_t stream,
-                      const sats_lora *lora)
+                      const sats_lora *lora, const int32_t *perm, const int32_t *n_dense)
 {
     const int H = layer->H, N = layer->N;
     const WsLayout L = ws_layout(H, N, B);
     char *base = static_cast<char *>(ws);
     if (!lora && use_tc_path(H, B)) {   // the LoRA variant runs in passes of the fused kernel at any batch
-        const cudaError_t e = run_tc_layer(layer, x_mode, x, B, *t_per_pass_l, norm_w, eps, dense_flags, out_mode,
+        const cudaError_t e = run_tc_layer(layer, x_mode, x, B, *t_per_pass_l, norm_w, eps, perm ? nullptr : dense_flags,
+                                           perm, n_dense, out_mode,
                                            out, active_idx, active_cnt, keep_trace, base + L.tc,
                                            reinterpret_cast<int *>(base + L.ctl), stream);
         return e == cudaSuccess ? SATS_OK : SATS_ECUDA;   // run_tc_layer recorded the failing step
@@ -392,7 +393,7 @@ static sats_status union_common(const sats_layer *layer, int x_mode, const void 
     if (!x || !y || !aligned16(x) || !aligned16(y)) return SATS_EINVAL;
     const WsLayout L = ws_layout(layer->H, layer->N, B);
     char *base = static_cast<char *>(ws);
-    const cudaError_t e = run_tc_layer(layer, x_mode, x, B, t_l, nullptr, 0.f, nullptr, kOutY, y, active_idx,
+    const cudaError_t e = run_tc_layer(layer, x_mode, x, B, t_l, nullptr, 0.f, nullptr, nullptr, nullptr, kOutY, y, active_idx,
                                        active_cnt, nullptr, base + L.tc, reinterpret_cast<int *>(base + L.ctl),
                                        static_cast<cudaStream_t>(stream), true);
     return e == cudaSuccess ? SATS_OK : SATS_ECUDA;   // run_tc_layer recorded the failing step
@@ -447,16 +448,22 @@ sats_status sats_mlp_stack(const sats_layer *const *layers, const float *const *
     const WsLayout W = ws_layout(H, N, B);
     char *base = static_cast<char *>(ws);
     int *ctl = reinterpret_cast<int *>(base + W.ctl);
+    // Routing once for every block (Eq. 13 through the table): the per-token flags serve the
+    // fused passes (B <= 2), the permutation (base-path tokens first) and its count the
+    // tensor-core path, which gathers the tokens in that order and scatters the results back.
     uint8_t *flags = nullptr;
+    int32_t *perm = nullptr;
+    const int32_t *n_dense = nullptr;
     if (token_ids) {
         flags = reinterpret_cast<uint8_t *>(base + W.route_flags);
-        cudaError_t e = launch_route(token_ids, B, lut, V, reinterpret_cast<int32_t *>(base + W.route_perm),
-                                     ctl + kCtlNDense, flags, ctl + kCtlStatus, st);
+        perm = reinterpret_cast<int32_t *>(base + W.route_perm);
+        n_dense = ctl + kCtlNDense;
+        cudaError_t e = launch_route(token_ids, B, lut, V, perm, ctl + kCtlNDense, flags, ctl + kCtlStatus, st);
         if (e != cudaSuccess) return cuda_fail(e, "route kernel launch");
     }
     for (int l = 0; l < L; ++l) {
         s = run_layer(layers[l], kXResidNorm, x, B, &t[l], norm_w[l], eps, flags, kOutResid, x, nullptr, nullptr,
-                      keep_trace ? keep_trace + (size_t)l * B * N : nullptr, ws, st);
+                      keep_trace ? keep_trace + (size_t)l * B * N : nullptr, ws, st, nullptr, perm, n_dense);
         if (s != SATS_OK) return s;
     }
     return SATS_OK;

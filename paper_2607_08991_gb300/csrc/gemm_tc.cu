@@ -12,6 +12,14 @@
 // the same accumulator, so that the gate values keep ~fp32 accuracy.  h goes
 // to the second GEMM the same way, as a bf16 high part and a bf16 low part
 // (about 16 significant bits), so that errors do not build up along a stack.
+// (Rounding h, or x for the up projection, to bf16 alone was measured to put a
+// Llama-shaped layer's output 2.9e-2 off the fp64 result in the worst element,
+// beyond the 2e-2 output tolerance, so both GEMMs keep both parts.)
+//
+// Routing (Sec. 3.2, Fig. 2): with the routing kernel's permutation (base-path
+// tokens first, n_dense of them, read on the device, so no host round trip),
+// row i of the packed activations is token perm[i], rows below n_dense take
+// threshold 0, and outputs, keep traces and kept lists go back to token perm[i].
 //
 // Two orientations:
 //  - skinny (M <= 256 tokens, bandwidth-bound): the weights are the MMA's A
@@ -35,14 +43,16 @@ namespace tc {
 namespace {
 
 // ---------------------------------------------------------------------- activations
-// Row m of X (fp32, optionally RMS-normalised with gain w) -> bf16 hi + lo.
+// Row m of X = row perm[m] of x (row m without a permutation), fp32, optionally
+// RMS-normalised with gain w -> bf16 hi + lo.
 __global__ void __launch_bounds__(256) split_kernel(const float *__restrict__ x, int H, const float *__restrict__ w,
-                                                    float eps, uint16_t *__restrict__ hi, uint16_t *__restrict__ lo)
+                                                    float eps, uint16_t *__restrict__ hi, uint16_t *__restrict__ lo,
+                                                    const int32_t *__restrict__ perm)
 {
     grid_dependency_wait();   // x may be the residual written by the preceding kernel
     grid_launch_dependents();
     const int m = blockIdx.x;
-    const float *xr = x + (size_t)m * H;
+    const float *xr = x + (size_t)(perm ? perm[m] : m) * H;
     __shared__ float red[8];
     float inv = 1.0f;
     if (w) {
@@ -128,6 +138,8 @@ struct SkinnyGuParams {
     int merge;                    // split and NT <= 128: one MMA of N = 2 NT over both parts
     float t_l;                    // threshold of sparse-path tokens
     const uint8_t *dense_flags;   // [M] (1 = base path, threshold 0) or nullptr
+    const int32_t *perm;          // routed order: row j is token perm[j], rows j < *n_dense on the base path; or nullptr
+    const int32_t *n_dense;
     uint16_t *hact;               // [M][ldh] bf16: h rounded to bf16
     uint16_t *hact_lo;            // [M][ldh] bf16: h minus that rounding
     int ldh;
@@ -249,6 +261,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // epilogue: thread = neuron r of the tile, columns = tokens
         const bool ok = mbar_wait(acc_full, 0u, &abort_flag);
         tc_fence_after();
+        const int nd = p.perm ? *p.n_dense : 0;
         const int lb = 32 * (warp & 3);
         const int r = lb + lane, n = t * R + r;
         const bool row_ok = ok && r < R && n < p.N;
@@ -292,7 +305,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int e = 0; e < 16; ++e) {
                 const int j = c0 + e;
                 if (j < p.M) {
-                    const float thr = (p.dense_flags && p.dense_flags[j]) ? 0.f : p.t_l;
+                    const bool base = p.perm ? j < nd : (p.dense_flags && p.dense_flags[j]);
+                    const float thr = base ? 0.f : p.t_l;
                     const float a = g[e] / (1.0f + expf(-g[e]));   // SiLU, Eq. 2
                     const bool keep = fabsf(a) >= thr;             // Eqs. 4-5
                     const float h = keep ? a * u[e] : 0.f;
@@ -300,7 +314,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     p.hact[(size_t)j * p.ldh + n] = hb;
                     p.hact_lo[(size_t)j * p.ldh + n] = bf16_bits(h - __uint_as_float((uint32_t)hb << 16));
                     if (p.keep) p.keep[(size_t)j * p.keep_stride + n] = keep ? 1 : 0;
-                    if (p.keep_trace) p.keep_trace[(size_t)j * p.N + n] = keep ? 1 : 0;
+                    if (p.keep_trace) p.keep_trace[(size_t)(p.perm ? p.perm[j] : j) * p.N + n] = keep ? 1 : 0;
                 }
             }
         }
@@ -321,6 +335,7 @@ struct SkinnyDownParams {
     const uint16_t *w;            // wd_blk
     int M, H, NT, KBn, units;     // units = tc_dt * KBn (hidden tile, neuron block) pairs
     float *out;                   // [M][H] fp32, added to with L2 reductions
+    const int32_t *perm;          // routed order: column j of h is token perm[j]; or nullptr
     int *ctl;
     int stages, stage_bytes, a_bytes;
     int merge;                    // NT <= 128: one MMA of N = 2 NT over h's high and low parts
@@ -458,7 +473,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!ok || h >= p.H) continue;
 #pragma unroll
                 for (int e = 0; e < 16; ++e)
-                    if (c0 + e < p.M) atomicAdd(p.out + (size_t)(c0 + e) * p.H + h, v[e]);
+                    if (c0 + e < p.M) atomicAdd(p.out + (size_t)(p.perm ? p.perm[c0 + e] : c0 + e) * p.H + h, v[e]);
             }
             tc_fence_before();
             mbar_arrive(&acc_empty[buf]);
@@ -489,6 +504,8 @@ struct WideGuParams {
     int split;
     float t_l;
     const uint8_t *dense_flags;
+    const int32_t *perm;          // routed order (see the file comment) or nullptr
+    const int32_t *n_dense;
     uint16_t *hact, *hact_lo;     // h as bf16 high and low parts
     int ldh;
     uint8_t *keep;
@@ -613,7 +630,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const bool row_ok = ok && m < p.M;
             float thr = INFINITY;
-            if (row_ok) thr = (p.dense_flags && p.dense_flags[m]) ? 0.f : p.t_l;
+            if (row_ok) thr = (p.perm ? m < *p.n_dense : (p.dense_flags && p.dense_flags[m])) ? 0.f : p.t_l;
             const uint32_t dg = tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * 2 * R);
             for (int c0 = 0; c0 < R; c0 += 16) {
                 float g[16], u[16];
@@ -655,7 +672,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 if (p.keep_trace) {
-                    uint8_t *trow = p.keep_trace + (size_t)m * p.N + n;
+                    uint8_t *trow = p.keep_trace + (size_t)(p.perm ? p.perm[m] : m) * p.N + n;
 #pragma unroll
                     for (int e = 0; e < 16; ++e)
                         if (n + e < p.N) trow[e] = (uint8_t)(kw[e / 4] >> (8 * (e & 3)));
@@ -690,6 +707,7 @@ struct WideDownParams {
     int atomic_out;       // 1: add into out with L2 reductions (split K); 0: one writer per element
     int add_residual;     // with atomic_out == 0: out += tile, else out = tile
     float *out;           // [M][H] fp32
+    const int32_t *perm;  // routed order: row m of h is token perm[m]; or nullptr
     int *ctl;
     int stages, stage_bytes;
 };
@@ -778,7 +796,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_ld_wait();
             const int h = d0 * BM + c0;
             if (!row_ok || h >= p.H) continue;
-            float *dst = p.out + (size_t)m * p.H + h;
+            float *dst = p.out + (size_t)(p.perm ? p.perm[m] : m) * p.H + h;
             const bool vec = h + 16 <= p.H;   // H is a multiple of 8: dst is 16-byte aligned
             if (p.atomic_out) {
                 if (vec) {
@@ -818,13 +836,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ---------------------------------------------------------------------- kept lists
-// Token m's ascending kept list from its keep bytes (one CTA per token).
+// Row m's ascending kept list from its keep bytes (one CTA per row), written as
+// the list of token perm[m] (token m without a permutation).
 __global__ void __launch_bounds__(512) keep_list_kernel(const uint8_t *__restrict__ keep, int stride, int N,
-                                                        int32_t *__restrict__ idx, int32_t *__restrict__ cnt)
+                                                        int32_t *__restrict__ idx, int32_t *__restrict__ cnt,
+                                                        const int32_t *__restrict__ perm)
 {
     grid_dependency_wait();   // the keep bytes are written by the preceding kernel
     grid_launch_dependents();
     const int m = blockIdx.x;
+    const int tok = perm ? perm[m] : m;
     const uint8_t *k = keep + (size_t)m * stride;
     __shared__ int warp_sums[16];
     __shared__ int base_s;
@@ -839,7 +860,7 @@ __global__ void __launch_bounds__(512) keep_list_kernel(const uint8_t *__restric
         __syncthreads();
         int before = base_s;
         for (int i = 0; i < w; ++i) before += warp_sums[i];
-        if (f) idx[(size_t)m * N + before + __popc(bal & ((1u << lane) - 1u))] = n;
+        if (f) idx[(size_t)tok * N + before + __popc(bal & ((1u << lane) - 1u))] = n;
         __syncthreads();
         if (threadIdx.x == 0) {
             int tot = 0;
@@ -848,7 +869,7 @@ __global__ void __launch_bounds__(512) keep_list_kernel(const uint8_t *__restric
         }
         __syncthreads();
     }
-    if (threadIdx.x == 0 && cnt) cnt[m] = base_s;
+    if (threadIdx.x == 0 && cnt) cnt[tok] = base_s;
 }
 
 
@@ -938,10 +959,13 @@ size_t tc_workspace_bytes(int H, int N, int B) { return tc_layout(H, N, B).total
 //   x: bf16 [B][H] (x_mode kXBf16) or fp32 [B][H] (kXF32 / kXResidNorm, then
 //   split into bf16 hi + lo, after RMSNorm with norm_w for kXResidNorm).
 //   out: y [B][H] (kOutY) or the residual (kOutResid, += y).
+//   perm, n_dense: the routing kernel's permutation and base-path count (device), or
+//   nullptr (then dense_flags, or no token on the base path).  With a permutation x
+//   must be fp32 (it is gathered into the split parts).
 cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int B, float t_l, const float *norm_w,
-                         float eps, const uint8_t *dense_flags, int out_mode, float *out, int32_t *active_idx,
-                         int32_t *active_cnt, uint8_t *keep_trace, void *tc_ws, int *ctl, cudaStream_t stream,
-                         bool union_path)
+                         float eps, const uint8_t *dense_flags, const int32_t *perm, const int32_t *n_dense,
+                         int out_mode, float *out, int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace,
+                         void *tc_ws, int *ctl, cudaStream_t stream, bool union_path)
 {
     using namespace tc;
     auto fail = [](cudaError_t err, const char *where) {
@@ -959,12 +983,13 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
     const int kstride = (N + 15) & ~15;
     const int sms = sm_count();
     const bool split = x_mode != kXBf16;
+    if (perm && (!split || !n_dense || union_path)) return fail(cudaErrorInvalidValue, "routed batch arguments");
     const uint16_t *xa = split ? xhi : static_cast<const uint16_t *>(x);
     cudaError_t e;
 
     if (split) {
         e = launch_pdl_threads(split_kernel, dim3(B), 256, stream, static_cast<const float *>(x), H,
-                               x_mode == kXResidNorm ? norm_w : nullptr, eps, xhi, xlo);
+                               x_mode == kXResidNorm ? norm_w : nullptr, eps, xhi, xlo, perm);
         if (e != cudaSuccess) return fail(e, "split kernel launch");
     }
 
@@ -1032,6 +1057,8 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.split = split ? 1 : 0;
         gp.t_l = t_l;
         gp.dense_flags = dense_flags;
+        gp.perm = perm;
+        gp.n_dense = n_dense;
         gp.hact = hact;
         gp.hact_lo = hact_lo;
         gp.ldh = ldn;
@@ -1066,6 +1093,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         dp.KBn = layer->tc_kbn;
         dp.units = layer->tc_dt * layer->tc_kbn;
         dp.out = out;
+        dp.perm = perm;
         dp.ctl = ctl;
         dp.a_bytes = BM * kTileBytes;
         dp.stage_bytes = dp.a_bytes + 2 * NT * kTileBytes;
@@ -1098,6 +1126,8 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.split = split ? 1 : 0;
         gp.t_l = t_l;
         gp.dense_flags = dense_flags;
+        gp.perm = perm;
+        gp.n_dense = n_dense;
         gp.hact = hact;
         gp.hact_lo = hact_lo;
         gp.ldh = ldn;
@@ -1130,6 +1160,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         dp.atomic_out = splits > 1 ? 1 : 0;
         dp.add_residual = out_mode == kOutResid ? 1 : 0;
         dp.out = out;
+        dp.perm = perm;
         dp.ctl = ctl;
         dp.stage_bytes = BM * kTileBytes * (2 + dp.dtiles);
         dp.stages = stages_for(dp.stage_bytes, wide_budget());
@@ -1145,7 +1176,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
     }
     if (active_idx) {
         e = launch_pdl_threads(keep_list_kernel, dim3(B), 512, stream, static_cast<const uint8_t *>(keep), kstride, N,
-                               active_idx, active_cnt);
+                               active_idx, active_cnt, perm);
         if (e != cudaSuccess) return fail(e, "kept-list kernel launch");
     }
     return cudaSuccess;

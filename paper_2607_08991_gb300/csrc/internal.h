@@ -132,9 +132,9 @@ cudaError_t launch_union_tail(const sats_layer *layer, int B, const uint16_t *xa
                               const uint8_t *uflag, int32_t *ulist, int32_t *ucount, const float *a_keep, int lda,
                               float *u, int ldu, float *out, int *ctl, cudaStream_t stream);
 cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int B, float t_l, const float *norm_w,
-                         float eps, const uint8_t *dense_flags, int out_mode, float *out, int32_t *active_idx,
-                         int32_t *active_cnt, uint8_t *keep_trace, void *tc_ws, int *ctl, cudaStream_t stream,
-                         bool union_path = false);
+                         float eps, const uint8_t *dense_flags, const int32_t *perm, const int32_t *n_dense,
+                         int out_mode, float *out, int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace,
+                         void *tc_ws, int *ctl, cudaStream_t stream, bool union_path = false);
 cudaError_t launch_wait_timeout(int *ctl, cudaStream_t stream);
 cudaError_t launch_route(const int32_t *ids, int B, const uint8_t *lut, int V, int32_t *perm,
                          int32_t *n_dense, uint8_t *flags, int32_t *status, cudaStream_t stream);
@@ -144,10 +144,13 @@ cudaError_t launch_gate_act_f32(const sats_layer *layer, const float *x, int B, 
 
 // One block over B tokens (fused kernel or tensor cores), as the C ABI calls run it
 // (api.cu).  ws: a workspace of ws_layout(H, N, B).total bytes with zeroed control words.
+// dense_flags (per token, original order) serve the fused passes; perm / n_dense (the
+// routing kernel's output) serve the tensor-core path, which then works in routed order.
 sats_status run_layer(const sats_layer *layer, int x_mode, const void *x, int B, const float *t_l,
                       const float *norm_w, float eps, const uint8_t *dense_flags, int out_mode, float *out,
                       int32_t *active_idx, int32_t *active_cnt, uint8_t *keep_trace, void *ws, cudaStream_t stream,
-                      const sats_lora *lora = nullptr);
+                      const sats_lora *lora = nullptr, const int32_t *perm = nullptr,
+                      const int32_t *n_dense = nullptr);
 size_t select_ws_bytes();
 cudaError_t launch_select(const float *a, int64_t n, int64_t m, void *ws, float *t_dev,
                           cudaStream_t stream);

@@ -104,6 +104,22 @@ def test_routed_stack_matches_oracle(sats, oracle, B):
     assert keep[:, dense].all()
 
 
+@pytest.mark.parametrize("B,p_dense", [(300, 0.4), (8, 1.0), (8, 0.0), (300, 1.0), (300, 0.0)])
+def test_routed_stack_tensor_core_groups(sats, oracle, B, p_dense):
+    """Batches on the tensor cores work in routed order (base-path tokens first, gathered
+    by the routing permutation, results scattered back): a mixed batch beyond one 128-token
+    tile, and the all-base / all-sparse tables, which must equal the static dense and sparse
+    paths."""
+    L, H, N = 2, 512, 1408
+    keep, ids, lut = _stack(sats, oracle, L, H, N, B, [0.6] * L, 1e-6, routed=True, p_dense=p_dense, seed=B + 1)
+    dense = lut[ids] == 1
+    assert keep[:, dense].all()
+    if p_dense == 1.0:
+        assert keep.all()
+    if p_dense == 0.0:
+        assert abs((1.0 - keep.mean()) - 0.6) < 0.1
+
+
 def test_llama_shaped_stack_two_layers(sats, oracle):
     """Two Llama-3.1-8B-shaped blocks (4096 / 14336), one decode token."""
     _stack(sats, oracle, 2, inputs.LLAMA_H, inputs.LLAMA_N, 1, [0.6, 0.8], 1e-5)
