@@ -80,6 +80,7 @@ constexpr int kTailChunks = 4;                             // the last kTailChun
 constexpr int kTailLag = 2;                                // ... only kTailLag chunks ahead of the W_ud rows
 constexpr int kPendingChunks = 16;                        // chunk words held back until every CTA has cleared its flags
 constexpr int kMaxUdRows = 8;                              // W_ud rows per stage (small H)
+constexpr int kSliceWords = 64;                            // a slice's chunk words kept in shared memory
 
 // Index-list words (the flags region: one word per chunk; CTA c's slice of the
 // lists is chunks [c per, (c + 1) per), per = ceil(nchunks / G)).  Chunk word:
@@ -129,6 +130,7 @@ struct Shared {
     int seen;                   // the list producer has seen every CTA past its prologue
     int flags_ready;            // index warp: 1 once every CTA has cleared its chunk words, -1 if that wait gave up
     uint32_t ired[kGateWarps][2];   // per-warp kept counts of the chunks before this CTA's slice
+    uint64_t sword[kSliceWords];    // the chunk words of this CTA's slice (slices of up to kSliceWords chunks)
     int quiet;                  // roles past their last use of the counters (list producer, index warp)
     int ldone;                  // chunks whose W_ud rows the list producer has issued (read by the gate producer)
 };
@@ -285,7 +287,7 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
     constexpr int kStatic = kStaticChunks<LORA>;
     const int nstatic = kStatic * G;
     auto static_chunk = [&](int s) { return (int)blockIdx.x + s * G; };
-    {
+    auto prefetch_fixed = [&]() {
         // The weights do not depend on the previous call: while it finishes (its tail
         // leaves HBM mostly idle), start moving this CTA's fixed chunks past the first
         // (which the gate ring takes) into L2.
@@ -304,7 +306,7 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
                 bytes -= nbytes;
             }
         }
-    }
+    };
     int next_k = -1;       // a claimed chunk not yet started
     bool waited = false;   // the claim counter belongs to the previous call until that call has ended
     auto claim = [&]() {
@@ -359,6 +361,16 @@ __device__ void gate_producer(const FusedParams &p, Shared<BT> &S, uint8_t *grin
             if (++stage == kGateStages) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
+        if (seq == 0) {
+            // Only once the first chunk's rows have landed: issued together, every CTA's
+            // prefetch of later chunks queued ahead of other CTAs' first rows in HBM, and the
+            // first chunk's mask came 1.3 us after the dependency was released (instrumented).
+            // (each ring slot on the latest phase this loop issued: only this thread re-arms a slot)
+            for (int s2 = 0; s2 < kGateStages && ok; ++s2)
+                if (S.gissued[s2] > 0) ok = mbar_wait(&S.gfull[s2], (uint32_t)(S.gissued[s2] - 1), &S.abort);
+            if (!ok) break;
+            prefetch_fixed();
+        }
         // the next chunk is a claimed one: claim it while this chunk's rows stream.  Near the
         // end of the chunks, first let the list producer catch up (its W_ud rows issued up to
         // kTailLag chunks behind this one): a CTA whose kept rows pile up takes no more chunks,
@@ -412,10 +424,11 @@ __device__ uint64_t await_word(const FusedParams &p, Shared<BT> &S, int k, unsig
 // The gate warps, after their stream: the entries of this CTA's slice of the
 // ascending index lists.  The entries of chunk k start at the number of neurons
 // kept in chunks [0, k):
-//   1. every thread sums the kept rows of its chunk words before the slice
-//      (words t, t + 256, ...; eight loads in flight; an unpublished word is
-//      awaited before the thread goes on), then the sums are reduced over the
-//      gate warps;
+//   1. every thread reads its chunk words up to the slice's end (words t,
+//      t + 256, ...; eight loads in flight; an unpublished word is awaited
+//      before the thread goes on), sums the kept rows of those before the slice
+//      and leaves the slice's own words in shared memory; the sums are reduced
+//      over the gate warps;
 //   2. the first gate warp writes the slice's entries from a warp scan of its
 //      chunks' counts, 32 chunks at a time, and the last slice the counts.
 // Chunks are taken in increasing order, so the words before a slice are mostly
@@ -440,27 +453,32 @@ __device__ void slice_index_lists(const FusedParams &p, Shared<BT> &S, GroupSync
     }
     bool ok = ready > 0;
     // 1.
+    const bool own_in_smem = k1 - k0 <= kSliceWords;
+    const int kend = own_in_smem ? k1 : k0;
     uint32_t pre0 = 0, pre1 = 0;
-    for (int k = t; ok && k < k0;) {
+    for (int k = t; ok && k < kend;) {
         uint64_t w[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
             const int kk = k + kGateThreads * i;
-            w[i] = kk < k0 ? ld_relaxed_gpu_u64(p.flags + kk) : kChunkKept;
+            w[i] = kk < kend ? ld_relaxed_gpu_u64(p.flags + kk) : kChunkKept;
         }
-        int n = 8;   // the words before the first unpublished one are counted now
+        int n = 8;   // the words before the first unpublished one are taken now
 #pragma unroll
         for (int i = 7; i >= 0; --i)
             if (flag_state(w[i]) == 0u) n = i;
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-            if (i < n && k + kGateThreads * i < k0) {
+            const int kk = k + kGateThreads * i;
+            if (i < n && kk < k0) {
                 pre0 += (uint32_t)__popc(chunk_rows(w[i], 0));
                 if (BT > 1) pre1 += (uint32_t)__popc(chunk_rows(w[i], 1));
+            } else if (i < n && kk < kend) {
+                S.sword[kk - k0] = w[i];
             }
         }
         k += kGateThreads * n;
-        if (n < 8 && k < k0) ok = await_word<BT>(p, S, k, t0) != 0ull;
+        if (n < 8 && k < kend) ok = await_word<BT>(p, S, k, t0) != 0ull;
     }
     pre0 = (uint32_t)__reduce_add_sync(0xffffffffu, pre0);
     pre1 = (uint32_t)__reduce_add_sync(0xffffffffu, pre1);
@@ -484,7 +502,9 @@ __device__ void slice_index_lists(const FusedParams &p, Shared<BT> &S, GroupSync
         const int k = base + lane;
         uint64_t f = 0ull;
         bool good = true;
-        if (k < k1) {
+        if (k < k1 && own_in_smem) {
+            f = S.sword[k - k0];
+        } else if (k < k1) {
             f = ld_relaxed_gpu_u64(p.flags + k);
             if (flag_state(f) == 0u) good = (f = await_word<BT>(p, S, k, t0)) != 0ull;
         }
