@@ -947,6 +947,97 @@ def run_workload(args):
     print(json.dumps(out))
 
 
+PROFILE_CASES = ("route", "batch64", "union", "lora", "small", "stack")
+
+
+def run_profile_case(args):
+    """Small capture cases for ncu, one kernel group each, `warmup + steps` launches of it:
+    route (the routing kernel at 64 and 2048 tokens over the Qwen-shaped vocabulary),
+    batch64 (the Llama-shaped layer at 64 tokens with index lists: the skinny tensor-core pair
+    and the kept-list kernel), union (the union path at 8 tokens, 90 %), lora (the LoRA-aware
+    decode kernel at rank 16, one token, 70 %), small (the small-layer cluster kernel) and stack
+    (one Llama-shaped block of a routed stack at 64 tokens: the RMSNorm/split kernel with the
+    routing gather, then the skinny pair).  Prints one JSON line."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_08991_gb300 import sats
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    stream = torch.cuda.Stream(device=dev)
+    n_calls = max(args.warmup, 1) + args.steps
+    case = args.profile_case
+
+    def threshold(layer, H, N, k, n_cal=64):
+        xc = torch.from_numpy(inputs.activations_bf16(n_cal, H, seed=inputs.SEED_CALIB).view(np.int16)).to(dev)
+        a = torch.empty(n_cal, N, dtype=torch.float32, device=dev)
+        sats.gate_act(layer, xc, a, stream=stream)
+        sel = torch.empty(sats.select_workspace_bytes(), dtype=torch.uint8, device=dev)
+        return sats.percentile_threshold(a, k, sel, stream=stream)
+
+    info = {"profile_case": case, "calls": n_calls}
+    with torch.cuda.stream(stream):
+        if case == "route":
+            V = inputs.QWEN_V
+            lut = torch.from_numpy(inputs.routing_lut(V, 0.3)).to(dev)
+            for B in (64, 2048):
+                ids = torch.from_numpy(inputs.token_ids_zipf(B, V, seed=inputs.SEED_IDS + B)).to(dev)
+                perm = torch.empty(B, dtype=torch.int32, device=dev)
+                nd = torch.empty(1, dtype=torch.int32, device=dev)
+                st = torch.zeros(1, dtype=torch.int32, device=dev)
+                for _ in range(n_calls):
+                    sats.route(ids, lut, perm, nd, st, stream=stream)
+                stream.synchronize()
+                info["n_dense_%d" % B] = int(nd.item())
+            ok = True
+        elif case in ("batch64", "union", "lora", "small", "stack"):
+            H, N = (inputs.SMALL_H, inputs.SMALL_N) if case == "small" else (inputs.LLAMA_H, inputs.LLAMA_N)
+            layer = sats.Layer(*inputs.mlp_weights_device(H, N), stream=stream)
+            B = {"batch64": 64, "union": 8, "lora": 1, "small": 1, "stack": 64}[case]
+            k = {"batch64": 0.5, "union": 0.9, "lora": 0.7, "small": 0.5, "stack": 0.5}[case]
+            t = threshold(layer, H, N, k)
+            ws = sats.Workspace(H, N, B, device=dev, stream=stream)
+            y = torch.empty(B, H, dtype=torch.float32, device=dev)
+            idx = torch.empty(B, N, dtype=torch.int32, device=dev)
+            cnt = torch.empty(B, dtype=torch.int32, device=dev)
+            xb = torch.from_numpy(inputs.activations_bf16(B, H).view(np.int16)).to(dev)
+            if case == "lora":
+                r = 16
+                ad = [torch.from_numpy(m.view(np.int16)).to(dev) for m in inputs.lora_adapter(H, N, r)]
+                lora = sats.Lora(layer, *ad, scale=1.0, stream=stream)
+                for _ in range(n_calls):
+                    sats.sparse_mlp_lora(layer, lora, xb, t, y, ws, idx, cnt, stream=stream)
+            elif case == "union":
+                for _ in range(n_calls):
+                    sats.sparse_mlp_union(layer, xb, t, y, ws, idx, cnt, stream=stream)
+            elif case == "stack":
+                V = inputs.LLAMA_V
+                lut = torch.from_numpy(inputs.routing_lut(V, 0.2, seed=inputs.SEED_LUT + 5)).to(dev)
+                ids = torch.from_numpy(inputs.token_ids_zipf(B, V, seed=inputs.SEED_IDS + B)).to(dev)
+                nw = torch.from_numpy(inputs.norm_weight(H)).to(dev)
+                x = torch.from_numpy(inputs.activations_f32(B, H)).to(dev)
+                for _ in range(n_calls):
+                    sats.mlp_stack([layer], [nw], [t], 1e-5, x, ws, token_ids=ids, lut=lut, stream=stream)
+            else:
+                for _ in range(n_calls):
+                    sats.sparse_mlp(layer, xb, t, y, ws, idx, cnt, stream=stream)
+            stream.synchronize()
+            ok = sats.get_error(ws, stream=stream) == sats.OK
+            info.update({"hidden": H, "intermediate": N, "tokens": B, "target_sparsity": k,
+                         "tensor_cores": sats.uses_tensor_cores(H, B)})
+            if case != "stack":
+                info["kept_token0"] = int(cnt[0].item())
+            if case == "lora":
+                lora.close()
+            layer.close()
+        else:
+            raise SystemExit("unknown profile case " + case)
+    info["status_ok"] = ok
+    print(json.dumps(info))
+    if not ok:
+        raise RuntimeError("device status after the profile case")
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -964,7 +1055,12 @@ def main():
                     help="small capture case for ncu: `warmup + steps` calls at this batch size on one layer copy")
     ap.add_argument("--profile", action="store_true",
                     help="small capture case for ncu: one layer copy, timed calls only, no CPU baseline")
+    ap.add_argument("--profile-case", default="", choices=("",) + PROFILE_CASES,
+                    help="small capture case for ncu of one kernel group (see run_profile_case)")
     args = ap.parse_args()
+    if args.profile_case:
+        run_profile_case(args)
+        return
     if args.profile or args.profile_batch:
         args.no_cpu_baseline = True
         args.no_batched = True
