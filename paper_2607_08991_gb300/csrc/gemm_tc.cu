@@ -837,7 +837,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ---------------------------------------------------------------------- kept lists
 // Row m's ascending kept list from its keep bytes (one CTA per row), written as
-// the list of token perm[m] (token m without a permutation).
+// the list of token perm[m] (token m without a permutation).  Thread t takes the
+// 16-byte vectors [t per, (t + 1) per) of the row: it counts their kept bytes, a
+// block scan gives its first position, and it writes its entries in order.  Two
+// passes over the row in all (the second from L1/L2), one block scan.
 __global__ void __launch_bounds__(512) keep_list_kernel(const uint8_t *__restrict__ keep, int stride, int N,
                                                         int32_t *__restrict__ idx, int32_t *__restrict__ cnt,
                                                         const int32_t *__restrict__ perm)
@@ -846,30 +849,43 @@ __global__ void __launch_bounds__(512) keep_list_kernel(const uint8_t *__restric
     grid_launch_dependents();
     const int m = blockIdx.x;
     const int tok = perm ? perm[m] : m;
-    const uint8_t *k = keep + (size_t)m * stride;
+    const uint4 *k = reinterpret_cast<const uint4 *>(keep + (size_t)m * stride);   // stride: a multiple of 16
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+    const int nv = (N + 15) >> 4;
+    const int per = (nv + 511) >> 9;
+    const int v0 = t * per, v1 = min(nv, v0 + per);
+    // the kept bytes (0 or 1) of vector v as a 16-bit mask; bytes at or past N are not counted
+    auto mask16 = [&](int v) {
+        const uint4 q = k[v];
+        const uint32_t wq[4] = {q.x, q.y, q.z, q.w};
+        uint32_t bits = 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            bits |= ((wq[i] & 1u) | ((wq[i] >> 7) & 2u) | ((wq[i] >> 14) & 4u) | ((wq[i] >> 21) & 8u)) << (4 * i);
+        const int rest = N - 16 * v;
+        return rest >= 16 ? bits : bits & ((1u << rest) - 1u);
+    };
+    int c = 0;
+    for (int v = v0; v < v1; ++v) c += __popc(mask16(v));
     __shared__ int warp_sums[16];
-    __shared__ int base_s;
-    if (threadIdx.x == 0) base_s = 0;
-    __syncthreads();
-    for (int c0 = 0; c0 < N; c0 += 512) {
-        const int n = c0 + threadIdx.x;
-        const int f = (n < N && k[n]) ? 1 : 0;
-        const uint32_t bal = __ballot_sync(0xffffffffu, f);
-        const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-        if (lane == 0) warp_sums[w] = __popc(bal);
-        __syncthreads();
-        int before = base_s;
-        for (int i = 0; i < w; ++i) before += warp_sums[i];
-        if (f) idx[(size_t)tok * N + before + __popc(bal & ((1u << lane) - 1u))] = n;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            int tot = 0;
-            for (int i = 0; i < 16; ++i) tot += warp_sums[i];
-            base_s += tot;
-        }
-        __syncthreads();
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int x = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += x;
     }
-    if (threadIdx.x == 0 && cnt) cnt[tok] = base_s;
+    if (lane == 31) warp_sums[w] = incl;
+    __syncthreads();
+    int pos = incl - c, total = 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        if (i < w) pos += warp_sums[i];
+        total += warp_sums[i];
+    }
+    int32_t *out = idx + (size_t)tok * N;
+    for (int v = v0; v < v1; ++v)
+        for (uint32_t bits = mask16(v); bits; bits &= bits - 1u) out[pos++] = 16 * v + __ffs(bits) - 1;
+    if (t == 0 && cnt) cnt[tok] = total;
 }
 
 
