@@ -15,11 +15,11 @@
 //      rows' gate dot products from shared memory (paired FP32 FMAs, all its
 //      rows in one transposed warp reduction), SiLU (Eq. 2) and the mask
 //      |a| >= t per token (Eqs. 4-5);
-//   3. once every warp is past the gate rows, each warp brings the W_ud rows
-//      of its kept neurons only (a skipped neuron costs no bytes beyond its
-//      gate row) into its own slots of shared memory, one bulk copy per row,
-//      all in flight at once; then up dot product, h = a u, and the down
-//      projection h W_down[j, :] into its y columns;
+//   3. each warp reads the W_ud rows of its kept neurons only (a skipped
+//      neuron costs no bytes beyond its gate row) straight into registers,
+//      each lane the 16-byte vectors it multiplies, two rows' loads in flight
+//      at a time; then up dot product, h = a u, and the down projection
+//      h W_down[j, :] into its y columns;
 //   4. the warps' y partials are summed through shared memory into the CTA's
 //      partial y, whose column slice s is stored into CTA s's shared memory
 //      (distributed shared memory); the CTA's kept count per token is stored
@@ -40,9 +40,19 @@ namespace sats {
 namespace {
 
 constexpr int kSmMaxH = 1024;
-constexpr size_t kSmMaxRowBytes = 192 * 1024;     // a CTA's W_ud rows (twice its gate rows) in shared memory
+constexpr size_t kSmMaxRowBytes = 192 * 1024;     // a CTA's gate rows in shared memory
 constexpr size_t kSmMaxSmem = kSmMaxRowBytes + 9216;
 constexpr uint32_t kSmCopyBytes = 32768;          // bytes per bulk copy of gate rows
+
+// 16-byte load of read-once data (the W_ud rows): not kept in L1.
+__device__ __forceinline__ uint4 ld_stream_v4(const uint4 *p)
+{
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
 
 __device__ __forceinline__ uint32_t cluster_ctarank()
 {
@@ -101,11 +111,10 @@ __device__ __forceinline__ float warp_sum8_transposed(const float (&p)[8], int l
     return d;
 }
 
-// Layout of the dynamic shared memory: R W_ud row slots of 4H bytes (the
-// first half holds the gate rows until every warp is past them; the slots
-// then hold the warps' y partials once every warp is past its W_ud rows), then
-// the receive buffer of this CTA's slice of the y columns, [C][BT][per] float4
-// groups.
+// Layout of the dynamic shared memory: the CTA's R gate rows of 2H bytes (the
+// region then holds the warps' y partials once every warp is past the gate
+// rows), then the receive buffer of this CTA's slice of the y columns,
+// [C][BT][per] float4 groups.
 struct SmallLayout {
     size_t rows, recv, total;
     int per;   // float4 column groups per CTA slice
@@ -114,7 +123,7 @@ struct SmallLayout {
 __host__ __device__ inline SmallLayout small_layout(int H, int R, int NW, int BT, int C)
 {
     SmallLayout L{};
-    const size_t row_bytes = (size_t)R * H * 4;
+    const size_t row_bytes = (size_t)R * H * 2;
     const size_t red_bytes = (size_t)NW * BT * H * 4;
     L.per = ((H >> 2) + C - 1) / C;
     L.rows = 0;
@@ -127,7 +136,6 @@ __host__ __device__ inline SmallLayout small_layout(int H, int R, int NW, int BT
 template <int BT, int NW>
 struct SmallState {
     uint64_t gfull;               // the gate rows have landed
-    uint64_t wfull[NW];           // warp w's W_ud rows have landed
     uint32_t keepw[BT][32];       // the CTA's keep words per token (bit j of word i = neuron 32 i + j of the CTA)
     int wpre[BT][32];             // kept neurons of the CTA in the words before word i
     int cnt_recv[BT][16];         // kept counts of the CTAs before this one (stored by them)
@@ -164,16 +172,14 @@ __global__ void __launch_bounds__(NW * 32, 1) small_mlp_kernel(const FusedParams
     const int c0 = (int)rank * R;                  // the CTA's first neuron
     const int cn = max(0, min(N - c0, R));         // neurons of this CTA
     const SmallLayout Ls = small_layout(H, R, NW, BT, (int)C);
-    uint8_t *rows_s = smem + Ls.rows;              // gate rows [R][2H bytes], then W_ud slots [R][4H bytes]
+    uint8_t *rows_s = smem + Ls.rows;              // gate rows [R][2H bytes]
     float *red_s = reinterpret_cast<float *>(smem + Ls.rows);    // [NW][BT][H], last
     float4 *recv = reinterpret_cast<float4 *>(smem + Ls.recv);   // [C][BT][per]
     const int per = Ls.per;
-    const size_t ud_bytes = (size_t)H * 4;
 
     // 1. the CTA's gate rows (contiguous in Wg_t) into shared memory, before the dependency wait
     if (tid == 0) {
         mbar_init(&S.gfull, 1);
-        for (int w = 0; w < NW; ++w) mbar_init(&S.wfull[w], 1);
         mbar_init_fence();
     }
     for (int i = tid; i < BT * 32; i += kThreads) S.keepw[i / 32][i % 32] = 0u;
@@ -298,17 +304,13 @@ __global__ void __launch_bounds__(NW * 32, 1) small_mlp_kernel(const FusedParams
             if (keep) atomicOr(&S.keepw[b][(w0 + myr) >> 5], 1u << ((w0 + myr) & 31));
         }
     }
-    __syncthreads();   // every warp is past the gate rows: the slots may be filled from here on
+    __syncthreads();   // every warp is past the gate rows: the region may hold the y partials from here on
     if (!S.ok) kept = 0u;
 
-    // 3. the warp's kept W_ud rows into its slots [w0, w0 + RW) of 4H bytes, one bulk copy each
-    if (lane == 0) mbar_arrive_expect_tx(&S.wfull[warp], (uint32_t)__popc(kept) * (uint32_t)ud_bytes);
-    __syncwarp();
-    if (lane < RW && ((kept >> lane) & 1u)) {
-        const int slot = w0 + __popc(kept & ((1u << lane) - 1u));
-        bulk_load(rows_s + (size_t)slot * ud_bytes, p.w_ud + (size_t)(c0 + w0 + lane) * 2 * H, (uint32_t)ud_bytes,
-                  &S.wfull[warp], pol);
-    }
+    // 3. the warp's kept W_ud rows, read straight into registers: lane takes the 16-byte vectors
+    //    lane + 32 i of each kept row's up half and down half, two rows' loads in flight at a time.
+    //    (One bulk copy per 2H-byte row had queued on the SM's copy engine: with about fifty rows
+    //    per CTA the last warp's rows landed 2.3 us after the first's.)
     f32x2 yp[BT][VPL][4];
 #pragma unroll
     for (int b = 0; b < BT; ++b)
@@ -316,36 +318,39 @@ __global__ void __launch_bounds__(NW * 32, 1) small_mlp_kernel(const FusedParams
         for (int i = 0; i < VPL; ++i)
 #pragma unroll
             for (int e = 0; e < 4; ++e) yp[b][i][e] = 0ull;
-    if (!mbar_wait(&S.wfull[warp], 0u, &never)) {
-        if (lane == 0) {
-            S.ok = 0;
-            atomicOr(p.ctl + kCtlStatus, kStatusTimeout);
-        }
-        (void)mbar_wait(&S.wfull[warp], 0u, &never);   // once more, bounded: copies still in flight land first
-        kept = 0u;
-    }
-    for (uint32_t todo = kept; todo; todo &= todo - 1u) {
-        const int r = __ffs(todo) - 1;
-        const uint8_t *row = rows_s + (size_t)(w0 + __popc(kept & ((1u << r) - 1u))) * ud_bytes;
+    for (uint32_t todo = kept; todo;) {
+        int rr[2];
+        uint4 wu[2][VPL], wd[2][VPL];
 #pragma unroll
-        for (int b = 0; b < BT; ++b) {
-            f32x2 u2 = 0ull;
+        for (int k = 0; k < 2; ++k) {
+            rr[k] = todo ? __ffs(todo) - 1 : -1;
+            if (todo) todo &= todo - 1u;
+            const uint4 *row = rr[k] >= 0 ? reinterpret_cast<const uint4 *>(p.w_ud + (size_t)(c0 + w0 + rr[k]) * 2 * H)
+                                          : nullptr;
 #pragma unroll
             for (int i = 0; i < VPL; ++i) {
                 const int v = lane + 32 * i;
-                if (v < HV) u2 = dot8_acc(reinterpret_cast<const uint4 *>(row)[v], xp[b][i], u2);
+                const bool in = row != nullptr && v < HV;
+                wu[k][i] = in ? ld_stream_v4(row + v) : make_uint4(0u, 0u, 0u, 0u);
+                wd[k][i] = in ? ld_stream_v4(row + HV + v) : make_uint4(0u, 0u, 0u, 0u);
             }
-            const float u = warp_sum(hsum2(u2));
-            const float h = __shfl_sync(0xffffffffu, am[b], kLead * r) * u;   // CATS_t(a) (x W_up), Eqs. 1, 5
-            const f32x2 hh = pack2(h, h);
+        }
 #pragma unroll
-            for (int i = 0; i < VPL; ++i) {
-                const int v = lane + 32 * i;
-                if (v < HV) axpy8(reinterpret_cast<const uint4 *>(row + (size_t)H * 2)[v], hh, yp[b][i]);
+        for (int k = 0; k < 2; ++k) {
+            if (rr[k] < 0) break;
+#pragma unroll
+            for (int b = 0; b < BT; ++b) {
+                f32x2 u2 = 0ull;
+#pragma unroll
+                for (int i = 0; i < VPL; ++i) u2 = dot8_acc(wu[k][i], xp[b][i], u2);
+                const float u = warp_sum(hsum2(u2));
+                const float h = __shfl_sync(0xffffffffu, am[b], kLead * rr[k]) * u;   // CATS_t(a) (x W_up), Eqs. 1, 5
+                const f32x2 hh = pack2(h, h);
+#pragma unroll
+                for (int i = 0; i < VPL; ++i) axpy8(wd[k][i], hh, yp[b][i]);
             }
         }
     }
-    __syncthreads();   // every warp is past its W_ud rows: the slots hold the y partials from here on
 
     // 4. the CTA's y: each warp with kept rows writes its partial, the columns are summed over the
     //    warps, and column slice s goes to CTA s; the kept counts go to the CTAs after this one
@@ -502,7 +507,7 @@ SmallPlan plan_small(int H, int N)
     if (RW > Sh::MR) return pl;
     const int R = RW * Sh::NW;
     const SmallLayout L = small_layout(H, R, Sh::NW, BT, C);
-    if ((size_t)R * H * 4 > kSmMaxRowBytes || L.total > kSmMaxSmem || R > 32 * 32) return pl;
+    if ((size_t)R * H * 2 > kSmMaxRowBytes || L.total > kSmMaxSmem || R > 32 * 32) return pl;
     pl.C = C;
     pl.R = R;
     pl.RW = RW;
