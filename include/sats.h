@@ -157,7 +157,7 @@ SATS_API sats_status sats_sparse_mlp(const sats_layer *layer, const void *x, int
  * sats_workspace_bytes(H, N, B) > 256 KiB, is rejected with SATS_ENOSPACE
  * before anything is enqueued.  On the fused small-batch kernel (B <= 2 for
  * H <= 4096, B = 1 above) the workspace is one 64-bit word per 8 neurons plus
- * about 17 KB, which admits N up to about 243,000; a batch on the tensor-core
+ * about 17 KB, which admits N up to about 245,000; a batch on the tensor-core
  * path (sats_uses_tensor_cores) also needs its staging (activations, h and
  * keep bytes per token, and padding to whole tiles), so only small layers fit
  * there: for example N <= 5504 at H = 8192, B = 2, and N <= 1008 at H = 4096,
