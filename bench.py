@@ -370,6 +370,19 @@ def run_gpu(args):
         e1.record(stream)
         e1.synchronize()
         mean_us.append(1e3 * e0.elapsed_time(e1) / K)
+    # the same without index lists (y only), outside the timed region: what the lists cost
+    nolist_us = []
+    if not args.profile:
+        for si, t in calls:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for k in range(K):
+                layer = layers[copy[0] % len(layers)]
+                copy[0] += 1
+                sats.sparse_mlp(layer, x, t, y, ws, stream=stream)
+            e1.record(stream)
+            e1.synchronize()
+            nolist_us.append(1e3 * e0.elapsed_time(e1) / K)
     torch.cuda.synchronize(dev)
     if world > 1:
         dist.barrier()
@@ -492,6 +505,8 @@ def run_gpu(args):
             per[str(s)] = {"us": mean_us[i], "realised_sparsity": realised[i], "algo_bytes": algo,
                            "achieved_gbs": gbs, "frac_of_%s" % peak_kind: gbs / hbm_peak,
                            "frac_of_8tbs": gbs / NOMINAL_HBM_GBS, "speedup_vs_dense": dense_us / mean_us[i]}
+            if nolist_us:
+                per[str(s)]["us_without_index_lists"] = nolist_us[i]
             bytes_all += algo
             us_all += mean_us[i]
         achieved = bytes_all / (us_all * 1e-6) / 1e9
