@@ -75,6 +75,8 @@ def _run(sats, oracle, H, N, B, k, seed=0, f32=False, want_lists=True):
     (4096, 640, 4, 0.5),        # two vectors per consumer thread
     (6144, 300, 3, 0.5),        # four vectors per consumer thread, passes of two
     (8192, 130, 2, 0.5),        # the largest hidden size
+    (64, 100003, 1, 0.7),       # slices of more than 64 chunks (index words re-read, not kept in shared memory)
+    (64, 100003, 2, 0.5),
 ])
 def test_sparse_mlp_matches_oracle(sats, oracle, H, N, B, k):
     keep, _ = _run(sats, oracle, H, N, B, k)
