@@ -563,6 +563,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp == 0 && lane == 0) {
         const uint32_t load_bytes = (uint32_t)(wofs + 2 * R * kTileBytes);
+        // L2 prefetch of the weight stage kWidePrefetch loads ahead (this CTA's own sequence of
+        // tiles); of the CTAs that share a weight tile, those of its first two token tiles ask
+        int pq = blockIdx.x, pkb = 0;
+        auto prefetch_ahead = [&]() {
+            if (pq >= p.tiles) return;
+            if (pq % p.mtiles < 2)
+                bulk_prefetch_l2(p.w + (size_t)((pq / p.mtiles) * KBh + pkb) * 2 * R * BK,
+                                 (uint32_t)(2 * R * kTileBytes));
+            if (++pkb == KBh) {
+                pkb = 0;
+                pq += gridDim.x;
+            }
+        };
+        for (int j = 0; j < kWidePrefetch; ++j) prefetch_ahead();
         int i = 0, s = 0, ph = 0;
         bool stop = false;
         for (int q = blockIdx.x; q < p.tiles && !stop; q += gridDim.x) {
@@ -579,6 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (p.split) tma_load(st + kA, &tmX2, kb * BK, m0, &full[s]);
                 bulk_load_shared(st + wofs, p.w + (size_t)(t * KBh + kb) * 2 * R * BK, (uint32_t)(2 * R * kTileBytes),
                                  &full[s]);
+                prefetch_ahead();
                 if (++s == S) { s = 0; ph ^= 1; }
             }
         }
@@ -752,6 +767,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp == 0 && lane == 0) {
         const uint32_t load_bytes = (uint32_t)(2 * kA + BN * kTileBytes);
+        // L2 prefetch kWidePrefetch stages ahead: the weight tiles by the CTAs of the first two
+        // token tiles, the h tiles by every fourth hidden-tile column of CTAs
+        int pkb = kb0;
+        auto prefetch_ahead = [&]() {
+            if (pkb >= kb1) return;
+            if (blockIdx.x < 2)
+                for (int q = 0; q < p.dtiles; ++q)
+                    bulk_prefetch_l2(p.w + ((size_t)(d0 + q) * p.KBn + pkb) * BM * BK, (uint32_t)kA);
+            if (blockIdx.y % 4 == 0) {
+                tma_prefetch_l2(&tmH, pkb * BK, m0);
+                tma_prefetch_l2(&tmH2, pkb * BK, m0);
+            }
+            ++pkb;
+        };
+        for (int j = 0; j < kWidePrefetch; ++j) prefetch_ahead();
         int i = 0;
         for (int s = 0, ph = 0; kb0 + i < kb1; ++i) {
             if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
@@ -763,6 +793,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int q = 0; q < p.dtiles; ++q)
                 bulk_load_shared(st + 2 * kA + q * kA, p.w + ((size_t)(d0 + q) * p.KBn + kb) * BM * BK,
                                  (uint32_t)kA, &full[s]);
+            prefetch_ahead();
             if (++s == S) { s = 0; ph ^= 1; }
         }
         issued_s = i;

@@ -30,6 +30,10 @@ constexpr int kMaxStages = 8;
 constexpr int kMaxSkinny = 256;      // largest batch on the skinny orientation (MMA N <= 256)
 constexpr int kMaxUnion = 8;         // largest batch on the union path (sparse-path tokens only)
 constexpr int kTileBytes = BK * 2;   // bytes of one tile row
+// The prefill kernels bring their weight stages into L2 this many stages ahead of
+// the loads: every weight stage is read by the CTAs of all token tiles at about
+// the same time, and a ring of four or five stages does not cover a miss to HBM.
+constexpr int kWidePrefetch = 16;
 
 // ---------------------------------------------------------------------- device helpers
 // Shared-memory matrix descriptor of a K-major bf16 tile written by TMA with
@@ -116,6 +120,14 @@ __device__ __forceinline__ void tma_load(void *dst, const CUtensorMap *map, int 
         "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
         ::"r"(smem_addr(dst)), "l"(map), "r"(c0), "r"(c1), "r"(smem_addr(bar))
         : "memory");
+}
+
+// Starts bringing one TMA box (inner coordinate c0, row c1) of the tensor into L2;
+// no completion to wait for.
+__device__ __forceinline__ void tma_prefetch_l2(const CUtensorMap *map, int c0, int c1)
+{
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(map), "r"(c0), "r"(c1)
+                 : "memory");
 }
 
 __device__ __forceinline__ uint16_t bf16_bits(float v)
