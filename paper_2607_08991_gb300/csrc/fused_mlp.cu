@@ -913,6 +913,13 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         if (lane == 0 && npend > 0) good = publish(-1, 0ull, true) ? 1 : 0;
         ok = __shfl_sync(0xffffffffu, good, 0) != 0;
     }
+    if (lane == 0) {
+        // the CTA adds into y only after every CTA has read its activations; the up/down
+        // warps read this with the end marker below
+        if (!flags_open && !*(volatile int *)&S.abort) flags_open = wait_prologues(p.ctl);
+        S.seen = flags_open ? 1 : 0;
+    }
+    __syncwarp();
     if (ok && mbar_wait(&S.uempty[stage], phase ^ 1u, &S.abort)) {
         if (lane == 0) {
             S.udesc[stage].kind = kEnd;
@@ -922,12 +929,7 @@ __device__ void list_producer(const FusedParams &p, Shared<BT> &S, uint8_t *urin
         S.abort = 1;
         flag_status(p.ctl, kStatusTimeout);
     }
-    if (lane == 0) {
-        // the CTA adds into y only after every CTA has read its activations
-        if (!flags_open && !*(volatile int *)&S.abort) flags_open = wait_prologues(p.ctl);
-        S.seen = flags_open ? 1 : 0;
-        counters_released<BT, LORA>(p, S);
-    }
+    if (lane == 0) counters_released<BT, LORA>(p, S);
     __syncwarp();
 }
 
@@ -994,8 +996,9 @@ __device__ __forceinline__ void down_stage(const FusedParams &p, Shared<BT> &S, 
     if (lane == 0) mbar_arrive(&S.uempty[st]);
 }
 
+// Returns true once the end marker has been taken and this thread's y columns are final.
 template <int BT, int VPT, bool LORA>
-__device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *uring, f32x2 (&yp)[BT][VPT][4])
+__device__ bool updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *uring, f32x2 (&yp)[BT][VPT][4])
 {
     float wacc[BT];   // LoRA: this lane's column of sum_j h_j A_down[j, :] (first warp only)
 #pragma unroll
@@ -1022,7 +1025,7 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
     if (!loaded) {
         S.abort = 1;
         flag_status(p.ctl, kStatusTimeout);
-        return;
+        return false;
     }
     if constexpr (LORA) {
         // While no W_ud row can arrive yet (the first one follows the first chunk's mask, which
@@ -1076,7 +1079,7 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
         if (!us(lane, &S.abort)) {
             S.abort = 1;
             flag_status(p.ctl, kStatusTimeout);
-            return;
+            return false;
         }
         if (t < BT * r2) {
             const int b = t / r2, c = t % r2;
@@ -1090,7 +1093,7 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
         if (!us(lane, &S.abort)) {
             S.abort = 1;
             flag_status(p.ctl, kStatusTimeout);
-            return;
+            return false;
         }
         if (t == 0) mbar_arrive(&L.zdone);
     }
@@ -1103,7 +1106,7 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
         if (!mbar_wait(&S.ufull[stage], phase, &S.abort)) {
             S.abort = 1;
             flag_status(p.ctl, kStatusTimeout);
-            return;
+            return false;
         }
         const UdDesc<BT> &d = S.udesc[stage];
         if (d.kind == kEnd) {
@@ -1151,7 +1154,7 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
         if (!us.wait(&S.abort)) {
             S.abort = 1;
             flag_status(p.ctl, kStatusTimeout);
-            return;
+            return false;
         }
         pend_stage = (int)stage;
         pend_nr = nr;
@@ -1169,7 +1172,7 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
         if (!us(lane, &S.abort)) {
             S.abort = 1;
             flag_status(p.ctl, kStatusTimeout);
-            return;
+            return false;
         }
         // four rank columns at a time, their B_down loads issued together (the rank is a multiple of 8)
         for (int q0 = 0; q0 < p.lora_r; q0 += 4) {
@@ -1197,6 +1200,7 @@ __device__ void updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
             }
         }
     }
+    return true;
 }
 
 // Bounded wait for every bulk copy still in flight (only on the error path).
@@ -1210,6 +1214,30 @@ __device__ void drain_copies(Shared<BT> &S)
         if (S.uissued[s] > 0) (void)mbar_wait(&S.ufull[s], (uint32_t)(S.uissued[s] - 1), &never);
 }
 
+
+// Adds up/down thread t's y columns into the output with L2 vector reductions.  Only
+// once every CTA has passed its prologue (has read its activations, which the output
+// may alias, and zeroed its slice of y).
+template <int BT, int VPT>
+__device__ __forceinline__ void add_partial_y(const FusedParams &p, const f32x2 (&yp)[BT][VPT][4], int t)
+{
+    const int HV = p.H >> 3;
+#pragma unroll
+    for (int b = 0; b < BT; ++b) {
+        if (b >= p.nb) break;
+#pragma unroll
+        for (int i = 0; i < VPT; ++i) {
+            const int v = t + i * kUdThreads;
+            if (v < HV) {
+                float *dst = p.out + (size_t)b * p.H + (size_t)v * 8;
+                const float2 y0 = unpack2(yp[b][i][0]), y1 = unpack2(yp[b][i][1]);
+                const float2 y2 = unpack2(yp[b][i][2]), y3 = unpack2(yp[b][i][3]);
+                red_add_v4(dst, y0.x, y0.y, y1.x, y1.y);
+                red_add_v4(dst + 4, y2.x, y2.y, y3.x, y3.y);
+            }
+        }
+    }
+}
 
 template <int BT, int VPT, bool LORA>
 __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParams p)
@@ -1253,10 +1281,16 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
     grid_launch_dependents();
 
     f32x2 yp[BT][VPT][4];
+    bool y_added = false;
     if (warp < kGateWarps) {
         gate_warps<BT, VPT>(p, S, gring);
     } else if (warp < kGateProducerWarp) {
-        updown_warps<BT, VPT, LORA>(p, S, uring, yp);
+        // the CTA's partial y goes out as soon as its last stage is done, while the gate warps
+        // may still be writing the CTA's slice of the index lists
+        if (updown_warps<BT, VPT, LORA>(p, S, uring, yp) && S.seen) {
+            add_partial_y<BT, VPT>(p, yp, tid - kGateThreads);
+            y_added = true;
+        }
     } else if (warp == kGateProducerWarp) {
         if (lane == 0) gate_producer<BT, LORA>(p, S, gring);
         __syncwarp();
@@ -1268,27 +1302,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_mlp_kernel(const FusedParam
     __syncthreads();
     if (tid == 0 && S.abort) drain_copies<BT>(S);
 
-    // add this CTA's partial y into the output: the list producer has seen every
-    // CTA past its prologue (every CTA has read its activations and zeroed its slice of y)
-    if (S.seen && warp >= kGateWarps && warp < kGateProducerWarp) {
-        const int t = tid - kGateThreads;
-        const int HV = p.H >> 3;
-#pragma unroll
-        for (int b = 0; b < BT; ++b) {
-            if (b >= p.nb) break;
-#pragma unroll
-            for (int i = 0; i < VPT; ++i) {
-                const int v = t + i * kUdThreads;
-                if (v < HV) {
-                    float *dst = p.out + (size_t)b * p.H + (size_t)v * 8;
-                    const float2 y0 = unpack2(yp[b][i][0]), y1 = unpack2(yp[b][i][1]);
-                    const float2 y2 = unpack2(yp[b][i][2]), y3 = unpack2(yp[b][i][3]);
-                    red_add_v4(dst, y0.x, y0.y, y1.x, y1.y);
-                    red_add_v4(dst + 4, y2.x, y2.y, y3.x, y3.y);
-                }
-            }
-        }
-    }
+    // otherwise (a role gave up early) the partial y is added here, if the list producer has
+    // seen every CTA past its prologue
+    if (!y_added && S.seen && warp >= kGateWarps && warp < kGateProducerWarp)
+        add_partial_y<BT, VPT>(p, yp, tid - kGateThreads);
 }
 
 template <int BT, int VPT, bool LORA>
