@@ -425,8 +425,8 @@ __device__ uint64_t await_word(const FusedParams &p, Shared<BT> &S, int k, unsig
 // ascending index lists.  The entries of chunk k start at the number of neurons
 // kept in chunks [0, k):
 //   1. every thread reads its chunk words up to the slice's end (words t,
-//      t + 256, ...; eight loads in flight; an unpublished word is awaited
-//      before the thread goes on), sums the kept rows of those before the slice
+//      t + 256, ...; eight loads in flight; an unpublished word is awaited,
+//      and taken as the wait read it), sums the kept rows of those before the slice
 //      and leaves the slice's own words in shared memory; the sums are reduced
 //      over the gate warps;
 //   2. the first gate warp writes the slice's entries from a warp scan of its
@@ -456,29 +456,33 @@ __device__ void slice_index_lists(const FusedParams &p, Shared<BT> &S, GroupSync
     const bool own_in_smem = k1 - k0 <= kSliceWords;
     const int kend = own_in_smem ? k1 : k0;
     uint32_t pre0 = 0, pre1 = 0;
-    for (int k = t; ok && k < kend;) {
+    for (int k = t; ok && k < kend; k += kGateThreads * 8) {
         uint64_t w[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
             const int kk = k + kGateThreads * i;
             w[i] = kk < kend ? ld_relaxed_gpu_u64(p.flags + kk) : kChunkKept;
         }
-        int n = 8;   // the words before the first unpublished one are taken now
-#pragma unroll
-        for (int i = 7; i >= 0; --i)
-            if (flag_state(w[i]) == 0u) n = i;
+        // every published word is taken now; an unpublished one is awaited and then taken
+        // as the wait read it (no second load)
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
             const int kk = k + kGateThreads * i;
-            if (i < n && kk < k0) {
+            if (kk >= kend || !ok) continue;
+            if (flag_state(w[i]) == 0u) {
+                w[i] = await_word<BT>(p, S, kk, t0);
+                if (w[i] == 0ull) {
+                    ok = false;
+                    continue;
+                }
+            }
+            if (kk < k0) {
                 pre0 += (uint32_t)__popc(chunk_rows(w[i], 0));
                 if (BT > 1) pre1 += (uint32_t)__popc(chunk_rows(w[i], 1));
-            } else if (i < n && kk < kend) {
+            } else {
                 S.sword[kk - k0] = w[i];
             }
         }
-        k += kGateThreads * n;
-        if (n < 8 && k < kend) ok = await_word<BT>(p, S, k, t0) != 0ull;
     }
     pre0 = (uint32_t)__reduce_add_sync(0xffffffffu, pre0);
     pre1 = (uint32_t)__reduce_add_sync(0xffffffffu, pre1);
