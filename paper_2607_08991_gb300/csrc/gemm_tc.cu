@@ -160,8 +160,10 @@ struct SkinnyGuParams {
 
 // One tile of R neurons (gate and up) against all M tokens: D[r][j] in TMEM
 // lane r, column j (gate) and NT + j (up).  Grid: tc_T CTAs.  In gate-only mode
-// only the gate rows are read and multiplied.
-__global__ void __launch_bounds__(kThreads, 1)
+// only the gate rows are read and multiplied.  The epilogue runs once all MMAs
+// are done, on G groups of four warps (blockDim 64 + 128 G): group g takes the
+// 16-token column blocks g, g + G, ... of every row (G = 1 in gate-only mode).
+__global__ void __launch_bounds__(kSkinnyMaxThreads, 1)
     gu_skinny_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmX2,
                      const SkinnyGuParams p)
 {
@@ -256,17 +258,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int per = (((p.zero_count + (int)gridDim.x - 1) / (int)gridDim.x) + 7) & ~7;
             const int z0 = (int)blockIdx.x * per, z1 = min(p.zero_count, z0 + per);
             float4 *z = reinterpret_cast<float4 *>(p.zero);
-            for (int i = z0 / 4 + (int)threadIdx.x - 64; i < z1 / 4; i += 128) z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int i = z0 / 4 + (int)threadIdx.x - 64; i < z1 / 4; i += (int)blockDim.x - 64)
+                z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
         }
         // epilogue: thread = neuron r of the tile, columns = tokens
         const bool ok = mbar_wait(acc_full, 0u, &abort_flag);
         tc_fence_after();
         const int nd = p.perm ? *p.n_dense : 0;
         const int lb = 32 * (warp & 3);
+        const int G = ((int)blockDim.x - 64) / 128, grp = (warp - 2) >> 2;
         const int r = lb + lane, n = t * R + r;
         const bool row_ok = ok && r < R && n < p.N;
         bool any = false;   // gate-only mode: some token keeps neuron n
-        for (int c0 = 0; c0 < NT; c0 += 16) {
+        for (int c0 = 16 * grp; c0 < NT; c0 += 16 * G) {
             float g[16], u[16], lo[16];
             tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)c0, g);
             if (p.merge) {
@@ -451,7 +455,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         consumed_s = i;
         mma_commit(mma_done);
     } else if (warp >= 2) {
+        // a warp's 32 rows x 16 tokens go through shared memory, so that each lane adds four
+        // vectors of four consecutive hidden units of one token (vector reductions in L2)
+        __shared__ float tr[4][16][33];
+        float(*T)[33] = tr[warp & 3];
         const int lb = 32 * (warp & 3);
+        const int te = lane >> 1, r0 = (lane & 1) * 16;   // this lane's token in the block, first row
         int q = 0;
         for (int u = u0; u < u1; ++q) {
             const int d = u / KBn;
@@ -459,7 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int buf = q & 1;
             const bool ok = mbar_wait(&acc_full[buf], (uint32_t)((q >> 1) & 1), &abort_flag);
             tc_fence_after();
-            const int h = d * BM + lb + lane;
+            const int h0 = d * BM + lb + r0;
             for (int c0 = 0; c0 < NT; c0 += 16) {
                 float v[16], lo[16];
                 tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * NX + c0), v);
@@ -470,10 +479,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int e = 0; e < 16; ++e) v[e] += lo[e];
                 }
                 tmem_ld_wait();
-                if (!ok || h >= p.H) continue;
 #pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    if (c0 + e < p.M) atomicAdd(p.out + (size_t)(p.perm ? p.perm[c0 + e] : c0 + e) * p.H + h, v[e]);
+                for (int e = 0; e < 16; ++e) T[e][lane] = v[e];
+                __syncwarp();
+                const int j = c0 + te;
+                if (ok && j < p.M) {
+                    float *dst = p.out + (size_t)(p.perm ? p.perm[j] : j) * p.H + h0;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k)   // H is a multiple of 8: a vector is in range or not at all
+                        if (h0 + 4 * k < p.H)
+                            red_add_v4(dst + 4 * k, T[te][r0 + 4 * k], T[te][r0 + 4 * k + 1], T[te][r0 + 4 * k + 2],
+                                       T[te][r0 + 4 * k + 3]);
+                }
+                __syncwarp();
             }
             tc_fence_before();
             mbar_arrive(&acc_empty[buf]);
@@ -1083,7 +1101,8 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.tmem_cols = tmem_cols_for(gp.merge ? 2 * NT : NT);
         if ((e = set_smem(gu_skinny_kernel, smem_for(1, gp.ring_bytes), cfg_gu_skinny)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
-        e = launch_pdl(gu_skinny_kernel, dim3(layer->tc_T), smem_for(1, gp.ring_bytes), stream, mX, mX2, gp);
+        e = launch_pdl_cfg(gu_skinny_kernel, dim3(layer->tc_T), 64 + 128, smem_for(1, gp.ring_bytes), stream, mX, mX2,
+                           gp);
         if (e != cudaSuccess) return fail(e, "gate kernel launch");
         e = launch_union_tail(layer, B, xa, split ? xlo : nullptr, uflag, ulist, ucount, a_keep, ldn, u, ldn, out, ctl,
                               stream);
@@ -1129,7 +1148,11 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.tmem_cols = tmem_cols_for((gp.merge ? 4 : 2) * NT);
         if ((e = set_smem(gu_skinny_kernel, smem_for(1, gp.ring_bytes), cfg_gu_skinny)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
-        e = launch_pdl(gu_skinny_kernel, dim3(layer->tc_T), smem_for(1, gp.ring_bytes), stream, mX, mX2, gp);
+        // epilogue groups: one per 16-token column block, at most kSkinnyMaxGroups (the epilogue
+        // runs after the last MMA, so its time adds to the call's)
+        const int groups = NT / 16 < kSkinnyMaxGroups ? NT / 16 : kSkinnyMaxGroups;
+        e = launch_pdl_cfg(gu_skinny_kernel, dim3(layer->tc_T), 64 + 128 * groups, smem_for(1, gp.ring_bytes), stream,
+                           mX, mX2, gp);
         if (e != cudaSuccess) return fail(e, "gate/up kernel launch");
 
         SkinnyDownParams dp{};

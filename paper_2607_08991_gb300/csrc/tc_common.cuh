@@ -24,6 +24,8 @@ namespace {
 constexpr int BM = 128;              // MMA M: rows of the A operand
 constexpr int BK = 64;               // K per TMA box: one 128-byte swizzle row of bf16
 constexpr int kThreads = 192;
+constexpr int kSkinnyMaxGroups = 6;                             // epilogue groups of four warps
+constexpr int kSkinnyMaxThreads = 64 + 128 * kSkinnyMaxGroups;  // of the batched-decode gate/up kernel
 constexpr int kSmemBudget = 196608;  // stage ring (one CTA per SM)
 constexpr int kSmemWide = 225280;    // stage ring of the persistent prefill kernels, at most
 constexpr int kMaxStages = 8;
