@@ -20,15 +20,17 @@
 //      each lane the 16-byte vectors it multiplies, two rows' loads in flight
 //      at a time; then up dot product, h = a u, and the down projection
 //      h W_down[j, :] into its y columns;
-//   4. the warps' y partials are summed through shared memory into the CTA's
-//      partial y, whose column slice s is stored into CTA s's shared memory
-//      (distributed shared memory); the CTA's kept count per token is stored
-//      into the CTAs after it;
-//   5. after one cluster barrier each CTA sums the C partials of its slice of
-//      the y columns from its own shared memory and writes it (or adds it into
-//      the residual stream), and writes its entries of the ascending index
-//      lists at the offset the earlier CTAs' counts give.  Nothing reads
-//      another CTA's shared memory after the barrier.
+//   4. as soon as the masks are known, the CTA's kept count per token goes into
+//      the shared memory of the CTAs after it (distributed shared memory), the
+//      CTA clears its slice of y (a plain output), and its threads arrive on
+//      the cluster barrier - every CTA has then read its activations (the
+//      output may alias them), cleared its slice and sent its counts;
+//   5. after step 3 the threads wait on that barrier (long complete by then),
+//      write the CTA's entries of the ascending index lists at the offset the
+//      earlier CTAs' counts give, sum the warps' y partials through shared
+//      memory and add the CTA's partial y into the output with vector
+//      reductions in L2.  Nothing touches another CTA's shared memory after
+//      the barrier.
 // The only wait is the bounded one on the gate rows' bulk copies; the cluster
 // barrier is a hardware barrier of co-scheduled CTAs.
 #include <cmath>
@@ -61,27 +63,12 @@ __device__ __forceinline__ uint32_t cluster_ctarank()
     return r;
 }
 
-// All threads of the cluster: release this CTA's shared-memory writes, then
-// acquire the other CTAs'.
-__device__ __forceinline__ void cluster_sync_all()
-{
-    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
-    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
 // Address of `p` (this CTA's shared memory) in the shared memory of cluster CTA `rank`.
 __device__ __forceinline__ uint32_t dsmem_addr(const void *p, uint32_t rank)
 {
     uint32_t r;
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr(p)), "r"(rank));
     return r;
-}
-
-__device__ __forceinline__ void st_dsmem_v4(uint32_t addr, float4 v)
-{
-    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y), "f"(v.z),
-                 "f"(v.w)
-                 : "memory");
 }
 
 __device__ __forceinline__ void st_dsmem_s32(uint32_t addr, int v)
@@ -111,13 +98,12 @@ __device__ __forceinline__ float warp_sum8_transposed(const float (&p)[8], int l
     return d;
 }
 
-// Layout of the dynamic shared memory: the CTA's R gate rows of 2H bytes (the
-// region then holds the warps' y partials once every warp is past the gate
-// rows), then the receive buffer of this CTA's slice of the y columns,
-// [C][BT][per] float4 groups.
+// Layout of the dynamic shared memory: the CTA's R gate rows of 2H bytes; the
+// region then holds the warps' y partials, [NW][BT][H] floats, once every warp
+// is past the gate rows.
 struct SmallLayout {
-    size_t rows, recv, total;
-    int per;   // float4 column groups per CTA slice
+    size_t rows, total;
+    int per;   // float4 column groups of y per CTA slice (cleared by that CTA)
 };
 
 __host__ __device__ inline SmallLayout small_layout(int H, int R, int NW, int BT, int C)
@@ -127,9 +113,7 @@ __host__ __device__ inline SmallLayout small_layout(int H, int R, int NW, int BT
     const size_t red_bytes = (size_t)NW * BT * H * 4;
     L.per = ((H >> 2) + C - 1) / C;
     L.rows = 0;
-    L.recv = (row_bytes > red_bytes ? row_bytes : red_bytes);
-    L.recv = (L.recv + 127) & ~(size_t)127;
-    L.total = L.recv + (size_t)C * BT * L.per * 16;
+    L.total = ((row_bytes > red_bytes ? row_bytes : red_bytes) + 127) & ~(size_t)127;
     return L;
 }
 
@@ -174,7 +158,6 @@ __global__ void __launch_bounds__(NW * 32, 1) small_mlp_kernel(const FusedParams
     const SmallLayout Ls = small_layout(H, R, NW, BT, (int)C);
     uint8_t *rows_s = smem + Ls.rows;              // gate rows [R][2H bytes]
     float *red_s = reinterpret_cast<float *>(smem + Ls.rows);    // [NW][BT][H], last
-    float4 *recv = reinterpret_cast<float4 *>(smem + Ls.recv);   // [C][BT][per]
     const int per = Ls.per;
 
     // 1. the CTA's gate rows (contiguous in Wg_t) into shared memory, before the dependency wait
@@ -307,6 +290,30 @@ __global__ void __launch_bounds__(NW * 32, 1) small_mlp_kernel(const FusedParams
     __syncthreads();   // every warp is past the gate rows: the region may hold the y partials from here on
     if (!S.ok) kept = 0u;
 
+    // 4. the CTA's kept counts to the CTAs after it, its slice of y cleared, then the arrival
+    if (warp == 0) {
+        const int nwords = (R + 31) >> 5;
+#pragma unroll
+        for (int b = 0; b < BT; ++b) {
+            const int c = lane < nwords ? __popc(S.keepw[b][lane]) : 0;
+            int incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int t = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += t;
+            }
+            S.wpre[b][lane] = incl - c;
+            const int tot = __shfl_sync(0xffffffffu, incl, 31);
+            if (lane > (int)rank && lane < (int)C) st_dsmem_s32(dsmem_addr(&S.cnt_recv[b][rank], (uint32_t)lane), tot);
+        }
+    }
+    if (p.out_mode == kOutY) {
+        const int k0 = (int)rank * per, nk = max(0, min(H4, k0 + per) - k0);
+        for (int q = tid; q < p.nb * nk; q += kThreads)
+            reinterpret_cast<float4 *>(p.out + (size_t)(q / nk) * H)[k0 + q % nk] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+
     // 3. the warp's kept W_ud rows, read straight into registers: lane takes the 16-byte vectors
     //    lane + 32 i of each kept row's up half and down half, two rows' loads in flight at a time.
     //    (One bulk copy per 2H-byte row had queued on the SM's copy engine: with about fifty rows
@@ -352,76 +359,8 @@ __global__ void __launch_bounds__(NW * 32, 1) small_mlp_kernel(const FusedParams
         }
     }
 
-    // 4. the CTA's y: each warp with kept rows writes its partial, the columns are summed over the
-    //    warps, and column slice s goes to CTA s; the kept counts go to the CTAs after this one
-    if (kept) {
-        if (lane == 0) S.warp_any[warp] = 1;
-#pragma unroll
-        for (int b = 0; b < BT; ++b)
-#pragma unroll
-            for (int i = 0; i < VPL; ++i) {
-                const int v = lane + 32 * i;
-                if (v < HV) {
-                    float4 *dst = reinterpret_cast<float4 *>(red_s + ((size_t)warp * BT + b) * H + 8 * v);
-                    const float2 y0 = unpack2(yp[b][i][0]), y1 = unpack2(yp[b][i][1]);
-                    const float2 y2 = unpack2(yp[b][i][2]), y3 = unpack2(yp[b][i][3]);
-                    dst[0] = make_float4(y0.x, y0.y, y1.x, y1.y);
-                    dst[1] = make_float4(y2.x, y2.y, y3.x, y3.y);
-                }
-            }
-    }
-    __syncthreads();
-    for (int q = tid; q < BT * H4; q += kThreads) {
-        const int b = q / H4, k = q % H4;
-        float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int w = 0; w < NW; ++w) {
-            if (!S.warp_any[w]) continue;
-            const float4 v = reinterpret_cast<const float4 *>(red_s + ((size_t)w * BT + b) * H)[k];
-            s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
-        }
-        const int dst = k / per;
-        st_dsmem_v4(dsmem_addr(recv + ((size_t)rank * BT + b) * per + (k - dst * per), (uint32_t)dst), s);
-    }
-    if (warp == 0) {
-        const int nwords = (R + 31) >> 5;
-#pragma unroll
-        for (int b = 0; b < BT; ++b) {
-            const int c = lane < nwords ? __popc(S.keepw[b][lane]) : 0;
-            int incl = c;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int t = __shfl_up_sync(0xffffffffu, incl, o);
-                if (lane >= o) incl += t;
-            }
-            S.wpre[b][lane] = incl - c;
-            const int tot = __shfl_sync(0xffffffffu, incl, 31);
-            if (lane > (int)rank && lane < (int)C) st_dsmem_s32(dsmem_addr(&S.cnt_recv[b][rank], (uint32_t)lane), tot);
-        }
-    }
-
-    // 5. one cluster barrier: every slice and every count has arrived
-    cluster_sync_all();
-    {
-        const int k0 = (int)rank * per;
-        const int nk = max(0, min(H4, k0 + per) - k0);
-        for (int q = tid; q < BT * nk; q += kThreads) {
-            const int b = q / nk, kk = q % nk;
-            if (b >= p.nb || !S.ok) continue;
-            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (uint32_t r = 0; r < C; ++r) {
-                const float4 w = recv[((size_t)r * BT + b) * per + kk];
-                v.x += w.x; v.y += w.y; v.z += w.z; v.w += w.w;
-            }
-            float4 *dst = reinterpret_cast<float4 *>(p.out + (size_t)b * H) + k0 + kk;
-            if (p.out_mode == kOutY) {
-                *dst = v;
-            } else {   // the residual stream: every CTA read its activations before the cluster barrier
-                float4 o = *dst;
-                o.x += v.x; o.y += v.y; o.z += v.z; o.w += v.w;
-                *dst = o;
-            }
-        }
-    }
+    // 5. every CTA has sent its counts, cleared its slice of y and read its activations
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
     if (p.active_idx) {
         for (int b = 0; b < p.nb; ++b) {
             int before = 0;
@@ -440,6 +379,38 @@ __global__ void __launch_bounds__(NW * 32, 1) small_mlp_kernel(const FusedParams
                 p.active_cnt[b] = before + own;
             }
         }
+    }
+    // the CTA's partial y: each warp with kept rows writes its partial, the columns are summed over
+    // the warps and added into the output (a cleared y, or the residual stream)
+    if (kept) {
+        if (lane == 0) S.warp_any[warp] = 1;
+#pragma unroll
+        for (int b = 0; b < BT; ++b)
+#pragma unroll
+            for (int i = 0; i < VPL; ++i) {
+                const int v = lane + 32 * i;
+                if (v < HV) {
+                    float4 *dst = reinterpret_cast<float4 *>(red_s + ((size_t)warp * BT + b) * H + 8 * v);
+                    const float2 y0 = unpack2(yp[b][i][0]), y1 = unpack2(yp[b][i][1]);
+                    const float2 y2 = unpack2(yp[b][i][2]), y3 = unpack2(yp[b][i][3]);
+                    dst[0] = make_float4(y0.x, y0.y, y1.x, y1.y);
+                    dst[1] = make_float4(y2.x, y2.y, y3.x, y3.y);
+                }
+            }
+    }
+    __syncthreads();
+    if (!S.ok) return;
+    for (int q = tid; q < p.nb * H4; q += kThreads) {
+        const int b = q / H4, k = q % H4;
+        float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+        bool any = false;
+        for (int w = 0; w < NW; ++w) {
+            if (!S.warp_any[w]) continue;
+            const float4 v = reinterpret_cast<const float4 *>(red_s + ((size_t)w * BT + b) * H)[k];
+            s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
+            any = true;
+        }
+        if (any) red_add_v4(p.out + (size_t)b * H + 4 * k, s.x, s.y, s.z, s.w);
     }
 }
 
