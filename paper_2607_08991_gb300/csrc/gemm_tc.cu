@@ -540,7 +540,7 @@ struct WideGuParams {
 // Per tile, D[m][c] accumulates in TMEM lane m, column b 2R + c (gate) and
 // b 2R + R + c (up), b alternating between tiles so that one tile's epilogue
 // overlaps the next tile's MMAs; the load ring runs across tile boundaries.
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kWideMaxThreads, 1)
     gu_wide_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmX2,
                    const WideGuParams p)
 {
@@ -565,7 +565,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&acc_full[b], 1);
-            mbar_init(&acc_empty[b], 128);
+            mbar_init(&acc_empty[b], blockDim.x - 64);   // every epilogue thread
         }
         mbar_init(mma_done, 1);
         abort_flag = 0;
@@ -653,8 +653,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         consumed_s = i;
         mma_commit(mma_done);
     } else if (warp >= 2) {
-        // epilogue: thread = token row of the tile, 16 neurons at a time
+        // epilogue: thread = token row of the tile, 16 neurons at a time; group g of four warps
+        // takes the 16-neuron column blocks g, g + G, ...
         const int lb = 32 * (warp & 3);
+        const int G = ((int)blockDim.x - 64) / 128, grp = (warp - 2) >> 2;
         int it = 0;
         for (int q = blockIdx.x; q < p.tiles; q += gridDim.x, ++it) {
             const int buf = it & 1;
@@ -665,7 +667,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             float thr = INFINITY;
             if (row_ok) thr = (p.perm ? m < *p.n_dense : (p.dense_flags && p.dense_flags[m])) ? 0.f : p.t_l;
             const uint32_t dg = tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * 2 * R);
-            for (int c0 = 0; c0 < R; c0 += 16) {
+            for (int c0 = 16 * grp; c0 < R; c0 += 16 * G) {
                 float g[16], u[16];
                 tmem_ld16(dg + (uint32_t)c0, g);
                 tmem_ld16(dg + (uint32_t)(R + c0), u);
@@ -748,7 +750,7 @@ struct WideDownParams {
 // One 128-token x (128 dtiles)-column tile of Y = h W_down over one split of
 // the neuron range; h arrives as its high and low bf16 parts (two A tiles).
 // Grid: (ceil(M / 128), tc_dt / dtiles, splits).
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kWideMaxThreads, 1)
     down_wide_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmH2,
                      const WideDownParams p)
 {
@@ -836,10 +838,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp >= 2) {
         const bool ok = mbar_wait(acc_full, 0u, &abort_flag) && kb1 > kb0;
         tc_fence_after();
+        // thread = token row of the tile; group g of four warps takes the 16-column blocks g, g + G, ...
+        // (the epilogue follows the tile's last MMA, so its time adds to the CTA's)
         const int lb = 32 * (warp & 3);
+        const int G = ((int)blockDim.x - 64) / 128, grp = (warp - 2) >> 2;
         const int m = m0 + lb + lane;
         const bool row_ok = ok && m < p.M;
-        for (int c0 = 0; c0 < BN; c0 += 16) {
+        for (int c0 = 16 * grp; c0 < BN; c0 += 16 * G) {
             float v[16];
             tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)c0, v);
             tmem_ld_wait();
@@ -1210,7 +1215,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         static std::atomic<int> cfg_gu[64];
         if ((e = set_smem(gu_wide_kernel, smem_for(gp.stages, gp.stage_bytes), cfg_gu)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
-        gu_wide_kernel<<<dim3(gp.tiles < sms ? gp.tiles : sms), kThreads, smem_for(gp.stages, gp.stage_bytes),
+        gu_wide_kernel<<<dim3(gp.tiles < sms ? gp.tiles : sms), 64 + 128 * kWideGuGroups, smem_for(gp.stages, gp.stage_bytes),
                          stream>>>(mX, mX2, gp);
         if ((e = cudaGetLastError()) != cudaSuccess) return fail(e, "gate/up kernel launch");
 
@@ -1240,7 +1245,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         static std::atomic<int> cfg_dn[64];
         if ((e = set_smem(down_wide_kernel, smem_for(dp.stages, dp.stage_bytes), cfg_dn)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
-        down_wide_kernel<<<dim3(mtiles, layer->tc_dt / dp.dtiles, splits), kThreads,
+        down_wide_kernel<<<dim3(mtiles, layer->tc_dt / dp.dtiles, splits), 64 + 128 * kWideDownGroups,
                            smem_for(dp.stages, dp.stage_bytes), stream>>>(mH, mH2, dp);
         if ((e = cudaGetLastError()) != cudaSuccess) return fail(e, "down kernel launch");
     }

@@ -24,6 +24,11 @@ namespace {
 constexpr int BM = 128;              // MMA M: rows of the A operand
 constexpr int BK = 64;               // K per TMA box: one 128-byte swizzle row of bf16
 constexpr int kThreads = 192;
+// Epilogue groups of four warps in the prefill kernels: the last tile's epilogue of the
+// persistent gate/up kernel, and every tile's of the down projection, follow their MMAs.
+constexpr int kWideGuGroups = 3;     // R = 96: two 16-neuron blocks each
+constexpr int kWideDownGroups = 4;   // 256 columns: four 16-column blocks each
+constexpr int kWideMaxThreads = 64 + 128 * 4;
 constexpr int kSkinnyMaxGroups = 6;                             // epilogue groups of four warps
 constexpr int kSkinnyMaxThreads = 64 + 128 * kSkinnyMaxGroups;  // of the batched-decode gate/up kernel
 constexpr int kSmemBudget = 196608;  // stage ring (one CTA per SM)
