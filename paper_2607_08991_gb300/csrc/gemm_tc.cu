@@ -32,10 +32,12 @@
 // The weights are read from tile-contiguous copies made at layer creation
 // (gu_blk, wd_blk), so that every TMA box is one contiguous DRAM read.
 //
-// Kernel layout (192 threads): warp 0 lane 0 issues the TMA loads, warp 1 owns
-// the TMEM allocation and lane 0 issues the MMAs, warps 2-5 run the epilogue
-// (warp w reads TMEM lanes 32 (w mod 4) .. 32 (w mod 4) + 31).  Every wait is
-// bounded in time and sets the status word when it gives up.
+// Kernel layout (64 + 128 G threads): warp 0 lane 0 issues the TMA loads, warp 1
+// owns the TMEM allocation and lane 0 issues the MMAs, warps 2 .. 4 G + 1 run the
+// epilogue in G groups of four (warp w reads TMEM lanes 32 (w mod 4) .. 32 (w mod
+// 4) + 31; the groups split the accumulator's columns; G = 1 in the down kernel of
+// batched decode, up to six in its gate/up kernel, three and four in the prefill
+// kernels).  Every wait is bounded in time and sets the status word when it gives up.
 #include "tc_common.cuh"
 
 namespace sats {
