@@ -201,12 +201,33 @@ struct GroupSync {
     }
 };
 
+// The RMSNorm gains of thread `t`'s vectors t + nthreads * i (a layer constant:
+// loaded before the dependency wait, so that the normalisation does not wait for them).
+template <int VPT>
+__device__ __forceinline__ void load_norm_gains(const FusedParams &p, int t, int nthreads, float (&gw)[VPT][8])
+{
+    const int HV = p.H >> 3;
+#pragma unroll
+    for (int i = 0; i < VPT; ++i) {
+        const int v = t + i * nthreads;
+        float4 lo = make_float4(0.f, 0.f, 0.f, 0.f), hi = lo;
+        if (p.x_mode == kXResidNorm && v < HV) {
+            const float4 *gw4 = reinterpret_cast<const float4 *>(p.norm_w);
+            lo = gw4[2 * v];
+            hi = gw4[2 * v + 1];
+        }
+        gw[i][0] = lo.x; gw[i][1] = lo.y; gw[i][2] = lo.z; gw[i][3] = lo.w;
+        gw[i][4] = hi.x; gw[i][5] = hi.y; gw[i][6] = hi.z; gw[i][7] = hi.w;
+    }
+}
+
 // Activations of this pass for one warp group: thread `t` of `nthreads` owns
 // the vectors t + nthreads * i (i < VPT).  RMSNorm (kXResidNorm) reduces over
-// the group through `gs`, using red[red0 + warp-in-group].
+// the group through `gs`, using red[red0 + warp-in-group], and scales by the
+// gains `gain` (load_norm_gains).
 template <int BT, int VPT>
 __device__ bool load_activations(const FusedParams &p, Shared<BT> &S, GroupSync &gs, int t, int nthreads,
-                                 int red0, f32x2 (&xp)[BT][VPT][4])
+                                 int red0, const float (&gain)[VPT][8], f32x2 (&xp)[BT][VPT][4])
 {
     const int lane = t & 31, gw = t >> 5, nw = nthreads >> 5;
     const int H = p.H, HV = H >> 3;
@@ -256,11 +277,8 @@ __device__ bool load_activations(const FusedParams &p, Shared<BT> &S, GroupSync 
             for (int i = 0; i < VPT; ++i) {
                 const int v = t + i * nthreads;
                 if (v < HV) {
-                    const float4 *gw4 = reinterpret_cast<const float4 *>(p.norm_w);
-                    const float4 lo = gw4[2 * v], hi = gw4[2 * v + 1];
-                    const float g8[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) xv[b][i][e] = xv[b][i][e] * inv * g8[e];
+                    for (int e = 0; e < 8; ++e) xv[b][i][e] = xv[b][i][e] * inv * gain[i][e];
                 }
             }
         }
@@ -554,8 +572,10 @@ __device__ void gate_warps(const FusedParams &p, Shared<BT> &S, const uint8_t *g
     const uint4 zero4 = make_uint4(0u, 0u, 0u, 0u);
     GroupSync gs{&S.gbar, 0u};
     f32x2 xp[BT][VPT][4];
+    float gw[VPT][8];
+    load_norm_gains<VPT>(p, t, kGateThreads, gw);
     grid_dependency_wait();   // x may be the previous launch's output
-    const bool loaded = load_activations<BT, VPT>(p, S, gs, t, kGateThreads, 0, xp);
+    const bool loaded = load_activations<BT, VPT>(p, S, gs, t, kGateThreads, 0, gw, xp);
     __syncwarp();
     if (lane == 0) mbar_arrive(&S.xloaded);
     if (!loaded) {
@@ -1022,8 +1042,10 @@ __device__ bool updown_warps(const FusedParams &p, Shared<BT> &S, const uint8_t 
 #pragma unroll
             for (int e = 0; e < 4; ++e) yp[b][i][e] = 0ull;
     f32x2 xp[BT][VPT][4];
+    float gw[VPT][8];
+    load_norm_gains<VPT>(p, t, kUdThreads, gw);
     grid_dependency_wait();
-    const bool loaded = load_activations<BT, VPT>(p, S, us, t, kUdThreads, kGateWarps, xp);
+    const bool loaded = load_activations<BT, VPT>(p, S, us, t, kUdThreads, kGateWarps, gw, xp);
     __syncwarp();
     if (lane == 0) mbar_arrive(&S.xloaded);
     if (!loaded) {

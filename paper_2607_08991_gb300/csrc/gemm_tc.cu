@@ -46,33 +46,60 @@ namespace {
 
 // ---------------------------------------------------------------------- activations
 // Row m of X = row perm[m] of x (row m without a permutation), fp32, optionally
-// RMS-normalised with gain w -> bf16 hi + lo.
+// RMS-normalised with gain w -> bf16 hi + lo.  Thread t holds the float4 vectors
+// t, t + 256, ... of the row in registers (H <= 8 * 4 * 256); the gains, a layer
+// constant, are read before the dependency wait.
+constexpr int kSplitVec = kMaxH / (4 * 256);
+
 __global__ void __launch_bounds__(256) split_kernel(const float *__restrict__ x, int H, const float *__restrict__ w,
                                                     float eps, uint16_t *__restrict__ hi, uint16_t *__restrict__ lo,
                                                     const int32_t *__restrict__ perm)
 {
+    const int H4 = H >> 2, t = threadIdx.x;
+    float4 wv[kSplitVec];
+#pragma unroll
+    for (int k = 0; k < kSplitVec; ++k) {
+        const int i = t + 256 * k;
+        wv[k] = (w && i < H4) ? reinterpret_cast<const float4 *>(w)[i] : make_float4(1.f, 1.f, 1.f, 1.f);
+    }
     grid_dependency_wait();   // x may be the residual written by the preceding kernel
     grid_launch_dependents();
     const int m = blockIdx.x;
-    const float *xr = x + (size_t)(perm ? perm[m] : m) * H;
-    __shared__ float red[8];
+    const float4 *xr = reinterpret_cast<const float4 *>(x + (size_t)(perm ? perm[m] : m) * H);
+    float4 xv[kSplitVec];
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < kSplitVec; ++k) {
+        const int i = t + 256 * k;
+        xv[k] = i < H4 ? xr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+        s = fmaf(xv[k].x, xv[k].x, fmaf(xv[k].y, xv[k].y, fmaf(xv[k].z, xv[k].z, fmaf(xv[k].w, xv[k].w, s))));
+    }
     float inv = 1.0f;
     if (w) {
-        float s = 0.f;
-        for (int i = threadIdx.x; i < H; i += 256) s = fmaf(xr[i], xr[i], s);
+        __shared__ float red[8];
         s = warp_sum(s);
-        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+        if ((t & 31) == 0) red[t >> 5] = s;
         __syncthreads();
         float tot = 0.f;
         for (int i = 0; i < 8; ++i) tot += red[i];
         inv = 1.0f / sqrtf(tot / (float)H + eps);
     }
-    for (int i = threadIdx.x; i < H; i += 256) {
-        const float v = w ? xr[i] * inv * w[i] : xr[i];
-        const uint16_t h = bf16_bits(v);
-        const float hv = __uint_as_float((uint32_t)h << 16);
-        hi[(size_t)m * H + i] = h;
-        lo[(size_t)m * H + i] = bf16_bits(v - hv);
+#pragma unroll
+    for (int k = 0; k < kSplitVec; ++k) {
+        const int i = t + 256 * k;
+        if (i >= H4) break;
+        const float v[4] = {xv[k].x * inv * wv[k].x, xv[k].y * inv * wv[k].y, xv[k].z * inv * wv[k].z,
+                            xv[k].w * inv * wv[k].w};
+        uint16_t hb[4], lb[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            hb[e] = bf16_bits(v[e]);
+            lb[e] = bf16_bits(v[e] - __uint_as_float((uint32_t)hb[e] << 16));
+        }
+        reinterpret_cast<uint2 *>(hi + (size_t)m * H)[i] =
+            make_uint2((uint32_t)hb[0] | ((uint32_t)hb[1] << 16), (uint32_t)hb[2] | ((uint32_t)hb[3] << 16));
+        reinterpret_cast<uint2 *>(lo + (size_t)m * H)[i] =
+            make_uint2((uint32_t)lb[0] | ((uint32_t)lb[1] << 16), (uint32_t)lb[2] | ((uint32_t)lb[3] << 16));
     }
 }
 
