@@ -290,10 +290,11 @@ __global__ void __launch_bounds__(kSkinnyMaxThreads, 1)
             for (int i = z0 / 4 + (int)threadIdx.x - 64; i < z1 / 4; i += (int)blockDim.x - 64)
                 z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        // epilogue: thread = neuron r of the tile, columns = tokens
+        // epilogue: thread = neuron r of the tile, columns = tokens (the base-path count is read
+        // while the MMAs run)
+        const int nd = p.perm ? *p.n_dense : 0;
         const bool ok = mbar_wait(acc_full, 0u, &abort_flag);
         tc_fence_after();
-        const int nd = p.perm ? *p.n_dense : 0;
         const int lb = 32 * (warp & 3);
         const int G = ((int)blockDim.x - 64) / 128, grp = (warp - 2) >> 2;
         const int r = lb + lane, n = t * R + r;
@@ -487,7 +488,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         // a warp's 32 rows x 16 tokens go through shared memory, so that each lane adds four
         // vectors of four consecutive hidden units of one token (vector reductions in L2)
         __shared__ float tr[4][16][33];
+        __shared__ int tok_s[kMaxSkinny];   // output row of each column (the routing permutation, read early)
         float(*T)[33] = tr[warp & 3];
+        grid_dependency_wait();   // (the permutation is older than the preceding kernel; its MMAs run meanwhile)
+        for (int j = (int)threadIdx.x - 64; j < NT; j += (int)blockDim.x - 64)
+            tok_s[j] = j < p.M ? (p.perm ? p.perm[j] : j) : 0;
+        named_barrier(1, (int)blockDim.x - 64);   // the epilogue warps only
         const int lb = 32 * (warp & 3);
         const int te = lane >> 1, r0 = (lane & 1) * 16;   // this lane's token in the block, first row
         int q = 0;
@@ -513,7 +519,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 __syncwarp();
                 const int j = c0 + te;
                 if (ok && j < p.M) {
-                    float *dst = p.out + (size_t)(p.perm ? p.perm[j] : j) * p.H + h0;
+                    float *dst = p.out + (size_t)tok_s[j] * p.H + h0;
 #pragma unroll
                     for (int k = 0; k < 4; ++k)   // H is a multiple of 8: a vector is in range or not at all
                         if (h0 + 4 * k < p.H)
@@ -686,6 +692,7 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
         // takes the 16-neuron column blocks g, g + G, ...
         const int lb = 32 * (warp & 3);
         const int G = ((int)blockDim.x - 64) / 128, grp = (warp - 2) >> 2;
+        const int nd = p.perm ? *p.n_dense : 0;   // the base-path count (routed order), read once
         int it = 0;
         for (int q = blockIdx.x; q < p.tiles; q += gridDim.x, ++it) {
             const int buf = it & 1;
@@ -694,7 +701,7 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
             tc_fence_after();
             const bool row_ok = ok && m < p.M;
             float thr = INFINITY;
-            if (row_ok) thr = (p.perm ? m < *p.n_dense : (p.dense_flags && p.dense_flags[m])) ? 0.f : p.t_l;
+            if (row_ok) thr = (p.perm ? m < nd : (p.dense_flags && p.dense_flags[m])) ? 0.f : p.t_l;
             const uint32_t dg = tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * 2 * R);
             for (int c0 = 16 * grp; c0 < R; c0 += 16 * G) {
                 float g[16], u[16];
@@ -865,6 +872,8 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
         consumed_s = i;
         mma_commit(acc_full);
     } else if (warp >= 2) {
+        const int m_row = m0 + 32 * (warp & 3) + lane;   // this thread's token row, and its output row (read early)
+        const int out_row = (p.perm && m_row < p.M) ? p.perm[m_row] : m_row;
         const bool ok = mbar_wait(acc_full, 0u, &abort_flag) && kb1 > kb0;
         tc_fence_after();
         // thread = token row of the tile; group g of four warps takes the 16-column blocks g, g + G, ...
@@ -879,7 +888,7 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
             tmem_ld_wait();
             const int h = d0 * BM + c0;
             if (!row_ok || h >= p.H) continue;
-            float *dst = p.out + (size_t)(p.perm ? p.perm[m] : m) * p.H + h;
+            float *dst = p.out + (size_t)out_row * p.H + h;
             const bool vec = h + 16 <= p.H;   // H is a multiple of 8: dst is 16-byte aligned
             if (p.atomic_out) {
                 if (vec) {
