@@ -90,7 +90,11 @@ def _stack(sats, oracle, L, H, N, B, targets, eps, routed=False, V=1000, p_dense
     return keep_ref, ids, lut
 
 
-@pytest.mark.parametrize("L,H,N,B", [(3, 256, 512, 1), (4, 512, 1408, 3), (2, 1024, 333, 6)])
+@pytest.mark.parametrize("L,H,N,B", [
+    (3, 256, 512, 1), (4, 512, 1408, 3), (2, 1024, 333, 6),
+    (2, 8192, 200, 1),   # the largest hidden size: four vectors per decode-kernel thread, RMSNorm gains in registers
+    (2, 8192, 200, 3),   # ... and on the tensor cores (one token per decode pass above 4096): the split kernel's full row
+])
 def test_stack_matches_oracle(sats, oracle, L, H, N, B):
     targets = inputs.stack_sparsity_targets(L, 0.55, 0.85)
     _stack(sats, oracle, L, H, N, B, targets, 1e-5)
