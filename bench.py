@@ -988,7 +988,7 @@ def run_workload(args):
     print(json.dumps(out))
 
 
-PROFILE_CASES = ("route", "batch64", "union", "lora", "small", "stack")
+PROFILE_CASES = ("route", "batch64", "union", "lora", "small", "stack", "prefill")
 
 
 def run_profile_case(args):
@@ -996,9 +996,10 @@ def run_profile_case(args):
     route (the routing kernel at 64 and 2048 tokens over the Qwen-shaped vocabulary),
     batch64 (the Llama-shaped layer at 64 tokens with index lists: the skinny tensor-core pair
     and the kept-list kernel), union (the union path at 8 tokens, 90 %), lora (the LoRA-aware
-    decode kernel at rank 16, one token, 70 %), small (the small-layer cluster kernel) and stack
+    decode kernel at rank 16, one token, 70 %), small (the small-layer cluster kernel), stack
     (one Llama-shaped block of a routed stack at 64 tokens: the RMSNorm/split kernel with the
-    routing gather, then the skinny pair).  Prints one JSON line."""
+    routing gather, then the skinny pair) and prefill (the same block at 2048 tokens, 90 %: the
+    split kernel, then the prefill pair with fp32 activations).  Prints one JSON line."""
     import torch
     import __graft_entry__
     __graft_entry__.build()
@@ -1031,11 +1032,11 @@ def run_profile_case(args):
                 stream.synchronize()
                 info["n_dense_%d" % B] = int(nd.item())
             ok = True
-        elif case in ("batch64", "union", "lora", "small", "stack"):
+        elif case in ("batch64", "union", "lora", "small", "stack", "prefill"):
             H, N = (inputs.SMALL_H, inputs.SMALL_N) if case == "small" else (inputs.LLAMA_H, inputs.LLAMA_N)
             layer = sats.Layer(*inputs.mlp_weights_device(H, N), stream=stream)
-            B = {"batch64": 64, "union": 8, "lora": 1, "small": 1, "stack": 64}[case]
-            k = {"batch64": 0.5, "union": 0.9, "lora": 0.7, "small": 0.5, "stack": 0.5}[case]
+            B = {"batch64": 64, "union": 8, "lora": 1, "small": 1, "stack": 64, "prefill": 2048}[case]
+            k = {"batch64": 0.5, "union": 0.9, "lora": 0.7, "small": 0.5, "stack": 0.5, "prefill": 0.9}[case]
             t = threshold(layer, H, N, k)
             ws = sats.Workspace(H, N, B, device=dev, stream=stream)
             y = torch.empty(B, H, dtype=torch.float32, device=dev)
@@ -1051,7 +1052,7 @@ def run_profile_case(args):
             elif case == "union":
                 for _ in range(n_calls):
                     sats.sparse_mlp_union(layer, xb, t, y, ws, idx, cnt, stream=stream)
-            elif case == "stack":
+            elif case in ("stack", "prefill"):
                 V = inputs.LLAMA_V
                 lut = torch.from_numpy(inputs.routing_lut(V, 0.2, seed=inputs.SEED_LUT + 5)).to(dev)
                 ids = torch.from_numpy(inputs.token_ids_zipf(B, V, seed=inputs.SEED_IDS + B)).to(dev)
@@ -1066,7 +1067,7 @@ def run_profile_case(args):
             ok = sats.get_error(ws, stream=stream) == sats.OK
             info.update({"hidden": H, "intermediate": N, "tokens": B, "target_sparsity": k,
                          "tensor_cores": sats.uses_tensor_cores(H, B)})
-            if case != "stack":
+            if case not in ("stack", "prefill"):
                 info["kept_token0"] = int(cnt[0].item())
             if case == "lora":
                 lora.close()
