@@ -28,7 +28,10 @@
 //    down projection splits its 64-neuron K blocks evenly over one CTA per SM
 //    and adds partial sums into y with L2 reductions.
 //  - wide (prefill): tokens are the A operand in tiles of 128, the weights the
-//    B operand; CTAs that run together share weight tiles through L2.
+//    B operand (up to 128 neurons' gate and up rows, gathered from the packed
+//    tiles); both kernels are persistent, and CTAs that run together share
+//    weight tiles through L2.  The down projection splits the neuron range so
+//    that its units even out over the SMs, and adds every unit into the output.
 // The weights are read from tile-contiguous copies made at layer creation
 // (gu_blk, wd_blk), so that every TMA box is one contiguous DRAM read.
 //
@@ -36,8 +39,8 @@
 // owns the TMEM allocation and lane 0 issues the MMAs, warps 2 .. 4 G + 1 run the
 // epilogue in G groups of four (warp w reads TMEM lanes 32 (w mod 4) .. 32 (w mod
 // 4) + 31; the groups split the accumulator's columns; G = 1 in the down kernel of
-// batched decode, up to six in its gate/up kernel, three and four in the prefill
-// kernels).  Every wait is bounded in time and sets the status word when it gives up.
+// batched decode, up to six in its gate/up kernel, four in the prefill kernels).
+// Every wait is bounded in time and sets the status word when it gives up.
 #include "tc_common.cuh"
 
 namespace sats {
@@ -551,9 +554,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ---------------------------------------------------------------------- wide gate + up
 struct WideGuParams {
-    const uint16_t *w;            // gu_blk
-    int M, N, R, KBh;
-    int mtiles, tiles;            // token tiles; tiles = mtiles * tc_T
+    const uint16_t *w;            // gu_blk: tiles of R neurons
+    int M, N, R, KBh, T;          // T: tiles of gu_blk
+    int Rw;                       // neurons per wide tile (a multiple of 16, <= 128): MMA N = 2 Rw
+    int mtiles, tiles;            // token tiles; tiles = mtiles * ceil(N / Rw)
     int split;
     float t_l;
     const uint8_t *dense_flags;
@@ -565,15 +569,22 @@ struct WideGuParams {
     int keep_stride;              // a multiple of 16
     uint8_t *keep_trace;
     int *ctl;
+    float *zero;                  // y [M][H] to clear for the down projection's additions, or nullptr
+    int zero_count;               // M H (a multiple of 8)
     int stages, stage_bytes;
-    uint32_t tmem_cols;           // two accumulator buffers of 2R columns
+    uint32_t tmem_cols;           // two accumulator buffers of 2 Rw columns
 };
 
-// Persistent: CTA c takes tiles c, c + G, c + 2G, ... of 128 tokens x R
+// Persistent: CTA c takes tiles c, c + G, c + 2G, ... of 128 tokens x Rw
 // neurons; tile q covers token tile q mod mtiles of neuron tile q / mtiles, so
 // the CTAs running together share few weight tiles and read them through L2.
-// Per tile, D[m][c] accumulates in TMEM lane m, column b 2R + c (gate) and
-// b 2R + R + c (up), b alternating between tiles so that one tile's epilogue
+// A stage holds the x tile(s), then the tile's Rw gate rows and Rw up rows,
+// gathered from gu_blk's tiles of R neurons: every operand byte passes through
+// shared memory twice (written by the copy engine, read by the MMA), and that
+// traffic rather than the MMA rate paces the loop, so a wider weight tile (up
+// to 128 neurons, MMA N = 256) puts more work on each byte.
+// Per tile, D[m][c] accumulates in TMEM lane m, column b 2Rw + c (gate) and
+// b 2Rw + Rw + c (up), b alternating between tiles so that one tile's epilogue
 // overlaps the next tile's MMAs; the load ring runs across tile boundaries.
 __global__ void __launch_bounds__(kWideMaxThreads, 1)
     gu_wide_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmX2,
@@ -590,7 +601,7 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mma_done + 1);
     __shared__ int abort_flag, issued_s, consumed_s;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int R = p.R, S = p.stages, KBh = p.KBh;
+    const int R = p.R, Rw = p.Rw, S = p.stages, KBh = p.KBh;
     const int wofs = kA * (p.split ? 2 : 1);
 
     if (threadIdx.x == 0) {
@@ -615,25 +626,59 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
     const uint32_t tmem = *tmem_slot;
 
     if (warp == 0 && lane == 0) {
-        const uint32_t load_bytes = (uint32_t)(wofs + 2 * R * kTileBytes);
+        // a wide tile's gate (and up) rows lie in at most two tiles of gu_blk: la rows from row r0
+        // of tile t0, then lb rows from the start of tile t0 + 1 (the host keeps Rw - gcd(Rw, R)
+        // <= R).  R and Rw are multiples of 16, so each piece keeps its rows' swizzle phase.  Rows
+        // past the last packed tile are not loaded: their columns of D belong to neurons >= N,
+        // which the epilogue skips.  Offsets in rows of BK elements at K block 0, worked out
+        // once per tile: this one thread's per-stage work must stay well below a stage's MMAs.
+        struct Pieces {
+            size_t a, b;
+            int la, lb;
+        };
+        auto pieces_of = [&](int tw) {
+            const int n0 = tw * Rw, rows = min(Rw, p.T * R - n0);
+            const int t0 = n0 / R, r0 = n0 - t0 * R;
+            Pieces w;
+            w.la = min(R - r0, rows);
+            w.lb = rows - w.la;
+            w.a = (size_t)t0 * KBh * 2 * R + r0;
+            w.b = (size_t)(t0 + 1) * KBh * 2 * R;
+            return w;
+        };
+        const size_t kb_rows = (size_t)2 * R;   // rows of a gu_blk tile per K block
         // L2 prefetch of the weight stage kWidePrefetch loads ahead (this CTA's own sequence of
         // tiles); of the CTAs that share a weight tile, those of its first two token tiles ask
         int pq = blockIdx.x, pkb = 0;
+        bool pf_on = false;
+        Pieces pf{};
+        auto prefetch_tile = [&]() {
+            pf_on = pq < p.tiles && pq % p.mtiles < 2;
+            if (pf_on) pf = pieces_of(pq / p.mtiles);
+        };
+        prefetch_tile();
         auto prefetch_ahead = [&]() {
             if (pq >= p.tiles) return;
-            if (pq % p.mtiles < 2)
-                bulk_prefetch_l2(p.w + (size_t)((pq / p.mtiles) * KBh + pkb) * 2 * R * BK,
-                                 (uint32_t)(2 * R * kTileBytes));
+            if (pf_on) {
+                const size_t o = (size_t)pkb * kb_rows;
+                for (int g = 0; g < 2; ++g) {
+                    bulk_prefetch_l2(p.w + (pf.a + o + g * R) * BK, (uint32_t)(pf.la * kTileBytes));
+                    if (pf.lb) bulk_prefetch_l2(p.w + (pf.b + o + g * R) * BK, (uint32_t)(pf.lb * kTileBytes));
+                }
+            }
             if (++pkb == KBh) {
                 pkb = 0;
                 pq += gridDim.x;
+                prefetch_tile();
             }
         };
         for (int j = 0; j < kWidePrefetch; ++j) prefetch_ahead();
         int i = 0, s = 0, ph = 0;
         bool stop = false;
         for (int q = blockIdx.x; q < p.tiles && !stop; q += gridDim.x) {
-            const int m0 = (q % p.mtiles) * BM, t = q / p.mtiles;
+            const int m0 = (q % p.mtiles) * BM;
+            const Pieces pc = pieces_of(q / p.mtiles);
+            const uint32_t load_bytes = (uint32_t)(wofs + 2 * (pc.la + pc.lb) * kTileBytes);
             for (int kb = 0; kb < KBh; ++kb, ++i) {
                 if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) {
                     set_timeout(p.ctl, &abort_flag);
@@ -644,17 +689,23 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
                 mbar_arrive_expect_tx(&full[s], load_bytes);
                 tma_load(st, &tmX, kb * BK, m0, &full[s]);
                 if (p.split) tma_load(st + kA, &tmX2, kb * BK, m0, &full[s]);
-                bulk_load_shared(st + wofs, p.w + (size_t)(t * KBh + kb) * 2 * R * BK, (uint32_t)(2 * R * kTileBytes),
-                                 &full[s]);
+                const size_t o = (size_t)kb * kb_rows;
+                for (int g = 0; g < 2; ++g) {
+                    uint8_t *dst = st + wofs + g * Rw * kTileBytes;
+                    bulk_load_shared(dst, p.w + (pc.a + o + g * R) * BK, (uint32_t)(pc.la * kTileBytes), &full[s]);
+                    if (pc.lb)
+                        bulk_load_shared(dst + pc.la * kTileBytes, p.w + (pc.b + o + g * R) * BK,
+                                         (uint32_t)(pc.lb * kTileBytes), &full[s]);
+                }
                 prefetch_ahead();
                 if (++s == S) { s = 0; ph ^= 1; }
             }
         }
         issued_s = i;
     } else if (warp == 1 && lane == 0) {
-        // gate rows and up rows are adjacent in the stage: one MMA with N = 2R writes the gate
-        // accumulator to columns [0, R) and the up accumulator to [R, 2R)
-        const uint32_t idesc = instr_desc(BM, 2 * R);
+        // gate rows and up rows are adjacent in the stage: one MMA with N = 2Rw writes the gate
+        // accumulator to columns [0, Rw) and the up accumulator to [Rw, 2Rw)
+        const uint32_t idesc = instr_desc(BM, 2 * Rw);
         int i = 0, s = 0, ph = 0, it = 0;
         bool stop = false;
         for (int q = blockIdx.x; q < p.tiles && !stop; q += gridDim.x, ++it) {
@@ -664,7 +715,7 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
                 break;
             }
             tc_fence_after();
-            const uint32_t d = tmem + (uint32_t)(buf * 2 * R);
+            const uint32_t d = tmem + (uint32_t)(buf * 2 * Rw);
             for (int kb = 0; kb < KBh; ++kb, ++i) {
                 if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) {
                     set_timeout(p.ctl, &abort_flag);
@@ -688,6 +739,15 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
         consumed_s = i;
         mma_commit(mma_done);
     } else if (warp >= 2) {
+        if (p.zero) {
+            // this CTA's share of y, cleared for the down projection's additions while the first
+            // tile's MMAs run
+            const int per = (((p.zero_count + (int)gridDim.x - 1) / (int)gridDim.x) + 7) & ~7;
+            const int z0 = (int)blockIdx.x * per, z1 = min(p.zero_count, z0 + per);
+            float4 *z = reinterpret_cast<float4 *>(p.zero);
+            for (int i = z0 / 4 + (int)threadIdx.x - 64; i < z1 / 4; i += (int)blockDim.x - 64)
+                z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
         // epilogue: thread = token row of the tile, 16 neurons at a time; group g of four warps
         // takes the 16-neuron column blocks g, g + G, ...
         const int lb = 32 * (warp & 3);
@@ -702,13 +762,13 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
             const bool row_ok = ok && m < p.M;
             float thr = INFINITY;
             if (row_ok) thr = (p.perm ? m < nd : (p.dense_flags && p.dense_flags[m])) ? 0.f : p.t_l;
-            const uint32_t dg = tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * 2 * R);
-            for (int c0 = 16 * grp; c0 < R; c0 += 16 * G) {
+            const uint32_t dg = tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * 2 * Rw);
+            for (int c0 = 16 * grp; c0 < Rw; c0 += 16 * G) {
                 float g[16], u[16];
                 tmem_ld16(dg + (uint32_t)c0, g);
-                tmem_ld16(dg + (uint32_t)(R + c0), u);
+                tmem_ld16(dg + (uint32_t)(Rw + c0), u);
                 tmem_ld_wait();
-                const int n = t * R + c0;
+                const int n = t * Rw + c0;
                 if (!row_ok || n >= p.N) continue;
                 uint32_t hw[8], lw[8], kw[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
@@ -768,24 +828,29 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
         tmem_dealloc(tmem, p.tmem_cols);
     }
 }
-
 // ---------------------------------------------------------------------- wide down
 struct WideDownParams {
     const uint16_t *w;    // wd_blk
     int M, H, KBn;
-    int dtiles;           // 128-row hidden tiles per CTA tile (1 or 2: MMA N = 128 dtiles)
-    int kb_per_split;     // K blocks of 64 neurons per split (blockIdx.z)
-    int atomic_out;       // 1: add into out with L2 reductions (split K); 0: one writer per element
-    int add_residual;     // with atomic_out == 0: out += tile, else out = tile
-    float *out;           // [M][H] fp32
+    int dtiles;           // 128-row hidden tiles per unit (1 or 2: MMA N = 128 dtiles)
+    int mtiles, dcols;    // token tiles; unit columns (tc_dt / dtiles)
+    int kb_per_split;     // K blocks of 64 neurons per unit
+    int units;            // mtiles * dcols * splits
+    float *out;           // [M][H] fp32: every unit adds its partial tile with L2 reductions
     const int32_t *perm;  // routed order: row m of h is token perm[m]; or nullptr
     int *ctl;
     int stages, stage_bytes;
+    uint32_t tmem_cols;   // two accumulator buffers of 128 dtiles columns
 };
 
-// One 128-token x (128 dtiles)-column tile of Y = h W_down over one split of
-// the neuron range; h arrives as its high and low bf16 parts (two A tiles).
-// Grid: (ceil(M / 128), tc_dt / dtiles, splits).
+// Persistent: CTA c takes units c, c + G, c + 2G, ...; unit u is the 128-token
+// x (128 dtiles)-column tile (u mod mtiles, (u / mtiles) mod dcols) of
+// Y = h W_down over the neuron split u / (mtiles dcols).  The splits even out the
+// units per CTA (the tile count alone can leave most SMs idle in a last wave),
+// and the units that run together share one split's h and weight tiles through
+// L2.  h arrives as its high and low bf16 parts (two A tiles); the accumulator
+// alternates between two TMEM buffers, so that one unit's epilogue (L2
+// reductions into the output rows) overlaps the next unit's MMAs.
 __global__ void __launch_bounds__(kWideMaxThreads, 1)
     down_wide_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmH2,
                      const WideDownParams p)
@@ -795,27 +860,39 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
     uint8_t *ring = align1024(smem_raw);
     uint64_t *full = reinterpret_cast<uint64_t *>(ring + (size_t)p.stages * p.stage_bytes);
     uint64_t *empty = full + kMaxStages;
-    uint64_t *acc_full = empty + kMaxStages;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_full + 1);
+    uint64_t *acc_full = empty + kMaxStages;   // [2]
+    uint64_t *acc_empty = acc_full + 2;        // [2]
+    uint64_t *mma_done = acc_empty + 2;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mma_done + 1);
     __shared__ int abort_flag, issued_s, consumed_s;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * BM, d0 = blockIdx.y * p.dtiles, S = p.stages;
-    const int BN = BM * p.dtiles;
-    const int kb0 = blockIdx.z * p.kb_per_split;
-    const int kb1 = min(p.KBn, kb0 + p.kb_per_split);
+    const int S = p.stages, BN = BM * p.dtiles, KBn = p.KBn;
+    const int per_split = p.mtiles * p.dcols;
+    // unit u -> its token tile's first row, first hidden tile and K-block range
+    auto unit = [&](int u, int &m0, int &d0, int &kb0, int &kb1) {
+        const int z = u / per_split, rem = u - z * per_split;
+        m0 = (rem % p.mtiles) * BM;
+        d0 = (rem / p.mtiles) * p.dtiles;
+        kb0 = z * p.kb_per_split;
+        kb1 = min(KBn, kb0 + p.kb_per_split);
+    };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
-        mbar_init(acc_full, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], blockDim.x - 64);   // every epilogue thread
+        }
+        mbar_init(mma_done, 1);
         abort_flag = 0;
         issued_s = 0;
         consumed_s = 0;
         mbar_init_fence();
     }
-    if (warp == 1) tmem_alloc(tmem_slot, 256);
+    if (warp == 1) tmem_alloc(tmem_slot, p.tmem_cols);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -823,75 +900,114 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
 
     if (warp == 0 && lane == 0) {
         const uint32_t load_bytes = (uint32_t)(2 * kA + BN * kTileBytes);
-        // L2 prefetch kWidePrefetch stages ahead: the weight tiles by the CTAs of the first two
-        // token tiles, the h tiles by every fourth hidden-tile column of CTAs
-        int pkb = kb0;
+        // L2 prefetch kWidePrefetch stages ahead (this CTA's own sequence of units): the weight
+        // tiles by the CTAs of the first two token tiles, the h tiles by every fourth unit column;
+        // the cursor's unit is decoded once per unit
+        int pu = blockIdx.x, pkb = 0, pkb1 = 0, pm0 = 0, pd0 = 0;
+        bool pf_w = false, pf_h = false;
+        auto prefetch_unit = [&]() {
+            if (pu >= p.units) return;
+            unit(pu, pm0, pd0, pkb, pkb1);
+            pf_w = pm0 < 2 * BM;
+            pf_h = (pd0 / p.dtiles) % 4 == 0;
+        };
+        prefetch_unit();
         auto prefetch_ahead = [&]() {
-            if (pkb >= kb1) return;
-            if (blockIdx.x < 2)
+            if (pu >= p.units) return;
+            if (pf_w)
                 for (int q = 0; q < p.dtiles; ++q)
-                    bulk_prefetch_l2(p.w + ((size_t)(d0 + q) * p.KBn + pkb) * BM * BK, (uint32_t)kA);
-            if (blockIdx.y % 4 == 0) {
-                tma_prefetch_l2(&tmH, pkb * BK, m0);
-                tma_prefetch_l2(&tmH2, pkb * BK, m0);
+                    bulk_prefetch_l2(p.w + ((size_t)(pd0 + q) * KBn + pkb) * BM * BK, (uint32_t)kA);
+            if (pf_h) {
+                tma_prefetch_l2(&tmH, pkb * BK, pm0);
+                tma_prefetch_l2(&tmH2, pkb * BK, pm0);
             }
-            ++pkb;
+            if (++pkb == pkb1) {
+                pu += gridDim.x;
+                prefetch_unit();
+            }
         };
         for (int j = 0; j < kWidePrefetch; ++j) prefetch_ahead();
-        int i = 0;
-        for (int s = 0, ph = 0; kb0 + i < kb1; ++i) {
-            if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
-            const int kb = kb0 + i;
-            uint8_t *st = ring + (size_t)s * p.stage_bytes;
-            mbar_arrive_expect_tx(&full[s], load_bytes);
-            tma_load(st, &tmH, kb * BK, m0, &full[s]);
-            tma_load(st + kA, &tmH2, kb * BK, m0, &full[s]);
-            for (int q = 0; q < p.dtiles; ++q)
-                bulk_load_shared(st + 2 * kA + q * kA, p.w + ((size_t)(d0 + q) * p.KBn + kb) * BM * BK,
-                                 (uint32_t)kA, &full[s]);
-            prefetch_ahead();
-            if (++s == S) { s = 0; ph ^= 1; }
+        int i = 0, s = 0, ph = 0;
+        bool stop = false;
+        for (int u = blockIdx.x; u < p.units && !stop; u += gridDim.x) {
+            int m0, d0, kb0, kb1;
+            unit(u, m0, d0, kb0, kb1);
+            for (int kb = kb0; kb < kb1; ++kb, ++i) {
+                if (!mbar_wait(&empty[s], (uint32_t)ph ^ 1u, &abort_flag)) {
+                    set_timeout(p.ctl, &abort_flag);
+                    stop = true;
+                    break;
+                }
+                uint8_t *st = ring + (size_t)s * p.stage_bytes;
+                mbar_arrive_expect_tx(&full[s], load_bytes);
+                tma_load(st, &tmH, kb * BK, m0, &full[s]);
+                tma_load(st + kA, &tmH2, kb * BK, m0, &full[s]);
+                for (int q = 0; q < p.dtiles; ++q)
+                    bulk_load_shared(st + 2 * kA + q * kA, p.w + ((size_t)(d0 + q) * KBn + kb) * BM * BK,
+                                     (uint32_t)kA, &full[s]);
+                prefetch_ahead();
+                if (++s == S) { s = 0; ph ^= 1; }
+            }
         }
         issued_s = i;
     } else if (warp == 1 && lane == 0) {
         const uint32_t idesc = instr_desc(BM, BN);
-        int i = 0;
-        for (int s = 0, ph = 0; kb0 + i < kb1; ++i) {
-            if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) { set_timeout(p.ctl, &abort_flag); break; }
-            tc_fence_after();
-            const uint32_t st = smem_addr(ring + (size_t)s * p.stage_bytes);
-#pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk) {
-                const uint64_t w = smem_desc(st + 2 * kA + kk * 32);
-                mma_bf16(tmem, smem_desc(st + kk * 32), w, idesc, (i | kk) ? 1u : 0u);
-                mma_bf16(tmem, smem_desc(st + kA + kk * 32), w, idesc, 1u);
+        int i = 0, s = 0, ph = 0, it = 0;
+        bool stop = false;
+        for (int u = blockIdx.x; u < p.units && !stop; u += gridDim.x, ++it) {
+            int m0, d0, kb0, kb1;
+            unit(u, m0, d0, kb0, kb1);
+            const int buf = it & 1;
+            if (!mbar_wait(&acc_empty[buf], (uint32_t)((it >> 1) & 1) ^ 1u, &abort_flag)) {
+                set_timeout(p.ctl, &abort_flag);
+                break;
             }
-            mma_commit(&empty[s]);
-            if (++s == S) { s = 0; ph ^= 1; }
+            tc_fence_after();
+            const uint32_t d = tmem + (uint32_t)(buf * BN);
+            for (int kb = kb0; kb < kb1; ++kb, ++i) {
+                if (!mbar_wait(&full[s], (uint32_t)ph, &abort_flag)) {
+                    set_timeout(p.ctl, &abort_flag);
+                    stop = true;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t st = smem_addr(ring + (size_t)s * p.stage_bytes);
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk) {
+                    const uint64_t w = smem_desc(st + 2 * kA + kk * 32);
+                    mma_bf16(d, smem_desc(st + kk * 32), w, idesc, (kb > kb0 || kk) ? 1u : 0u);
+                    mma_bf16(d, smem_desc(st + kA + kk * 32), w, idesc, 1u);
+                }
+                mma_commit(&empty[s]);
+                if (++s == S) { s = 0; ph ^= 1; }
+            }
+            mma_commit(&acc_full[buf]);
         }
         consumed_s = i;
-        mma_commit(acc_full);
+        mma_commit(mma_done);
     } else if (warp >= 2) {
-        const int m_row = m0 + 32 * (warp & 3) + lane;   // this thread's token row, and its output row (read early)
-        const int out_row = (p.perm && m_row < p.M) ? p.perm[m_row] : m_row;
-        const bool ok = mbar_wait(acc_full, 0u, &abort_flag) && kb1 > kb0;
-        tc_fence_after();
-        // thread = token row of the tile; group g of four warps takes the 16-column blocks g, g + G, ...
-        // (the epilogue follows the tile's last MMA, so its time adds to the CTA's)
+        // thread = token row of the unit's tile; group g of four warps takes the 16-column blocks
+        // g, g + G, ...
         const int lb = 32 * (warp & 3);
         const int G = ((int)blockDim.x - 64) / 128, grp = (warp - 2) >> 2;
-        const int m = m0 + lb + lane;
-        const bool row_ok = ok && m < p.M;
-        for (int c0 = 16 * grp; c0 < BN; c0 += 16 * G) {
-            float v[16];
-            tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)c0, v);
-            tmem_ld_wait();
-            const int h = d0 * BM + c0;
-            if (!row_ok || h >= p.H) continue;
-            float *dst = p.out + (size_t)out_row * p.H + h;
-            const bool vec = h + 16 <= p.H;   // H is a multiple of 8: dst is 16-byte aligned
-            if (p.atomic_out) {
-                if (vec) {
+        int it = 0;
+        for (int u = blockIdx.x; u < p.units; u += gridDim.x, ++it) {
+            int m0, d0, kb0, kb1;
+            unit(u, m0, d0, kb0, kb1);
+            const int buf = it & 1;
+            const int m = m0 + lb + lane;
+            const int out_row = (p.perm && m < p.M) ? p.perm[m] : m;   // read before the wait
+            const bool ok = mbar_wait(&acc_full[buf], (uint32_t)((it >> 1) & 1), &abort_flag);
+            tc_fence_after();
+            const bool row_ok = ok && m < p.M;
+            for (int c0 = 16 * grp; c0 < BN; c0 += 16 * G) {
+                float v[16];
+                tmem_ld16(tmem + ((uint32_t)lb << 16) + (uint32_t)(buf * BN + c0), v);
+                tmem_ld_wait();
+                const int h = d0 * BM + c0;
+                if (!row_ok || h >= p.H) continue;
+                float *dst = p.out + (size_t)out_row * p.H + h;
+                if (h + 16 <= p.H) {   // H is a multiple of 8: dst is 16-byte aligned
 #pragma unroll
                     for (int q = 0; q < 4; ++q) red_add_v4(dst + 4 * q, v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
                 } else {
@@ -899,31 +1015,24 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
                     for (int e = 0; e < 16; ++e)
                         if (h + e < p.H) atomicAdd(dst + e, v[e]);
                 }
-            } else if (vec) {
-                float4 *d4 = reinterpret_cast<float4 *>(dst);
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    float4 o = p.add_residual ? d4[q] : make_float4(0.f, 0.f, 0.f, 0.f);
-                    o.x += v[4 * q];
-                    o.y += v[4 * q + 1];
-                    o.z += v[4 * q + 2];
-                    o.w += v[4 * q + 3];
-                    d4[q] = o;
-                }
-            } else {
-#pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    if (h + e < p.H) dst[e] = p.add_residual ? dst[e] + v[e] : v[e];
             }
+            tc_fence_before();
+            mbar_arrive(&acc_empty[buf]);
+            if (!ok) break;
         }
-        tc_fence_before();
     }
     __syncthreads();
-    if (abort_flag && threadIdx.x == 0) drain_after_abort(full, S, issued_s, consumed_s, acc_full);
+    if (threadIdx.x == 0) {
+        // the arrival on mma_done must land before this CTA's shared memory is released
+        int never = 0;
+        if (abort_flag)
+            for (int k = consumed_s; k < issued_s; ++k) mbar_wait(&full[k % S], (uint32_t)((k / S) & 1), &never);
+        mbar_wait(mma_done, 0u, &never);
+    }
     __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem, 256);
+        tmem_dealloc(tmem, p.tmem_cols);
     }
 }
 
@@ -1233,9 +1342,11 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.N = N;
         gp.R = R;
         gp.KBh = layer->tc_kbh;
+        gp.T = layer->tc_T;
+        gp.Rw = wide_rows(N, R, mtiles, sms, split);
         gp.mtiles = mtiles;
-        gp.tiles = mtiles * layer->tc_T;
-        gp.tmem_cols = tmem_cols_for(4 * R);
+        gp.tiles = mtiles * ((N + gp.Rw - 1) / gp.Rw);
+        gp.tmem_cols = tmem_cols_for(4 * gp.Rw);
         gp.split = split ? 1 : 0;
         gp.t_l = t_l;
         gp.dense_flags = dense_flags;
@@ -1248,42 +1359,44 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.keep_stride = kstride;
         gp.keep_trace = keep_trace;
         gp.ctl = ctl;
-        gp.stage_bytes = BM * kTileBytes * (split ? 2 : 1) + 2 * R * kTileBytes;
+        gp.zero = out_mode == kOutY ? out : nullptr;   // the down projection adds into y
+        gp.zero_count = B * H;
+        gp.stage_bytes = BM * kTileBytes * (split ? 2 : 1) + 2 * gp.Rw * kTileBytes;
         gp.stages = stages_for(gp.stage_bytes, wide_budget());
+        // epilogue groups: the tile's 16-neuron column blocks split evenly over at most kWideGuGroups
+        const int blocks16 = gp.Rw / 16, per_group = (blocks16 + kWideGuGroups - 1) / kWideGuGroups;
+        const int gu_groups = (blocks16 + per_group - 1) / per_group;
         static std::atomic<int> cfg_gu[64];
         if ((e = set_smem(gu_wide_kernel, smem_for(gp.stages, gp.stage_bytes), cfg_gu)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
-        gu_wide_kernel<<<dim3(gp.tiles < sms ? gp.tiles : sms), 64 + 128 * kWideGuGroups, smem_for(gp.stages, gp.stage_bytes),
+        gu_wide_kernel<<<dim3(gp.tiles < sms ? gp.tiles : sms), 64 + 128 * gu_groups, smem_for(gp.stages, gp.stage_bytes),
                          stream>>>(mX, mX2, gp);
         if ((e = cudaGetLastError()) != cudaSuccess) return fail(e, "gate/up kernel launch");
 
-        // down projection: 256 output columns per tile when the hidden tiles pair up;
-        // split K (neurons) when the tile grid alone leaves SMs idle
+        // down projection: 256 output columns per unit when the hidden tiles pair up; the neuron
+        // range split so that the persistent CTAs' units come out even; every unit adds into the
+        // output (y cleared by the gate/up kernel, or the residual stream)
         WideDownParams dp{};
         dp.w = layer->wd_blk;
         dp.M = B;
         dp.H = H;
         dp.KBn = layer->tc_kbn;
         dp.dtiles = (layer->tc_dt % 2 == 0) ? 2 : 1;
-        const int tiles = mtiles * (layer->tc_dt / dp.dtiles);
-        int splits = tiles >= sms ? 1 : (sms + tiles - 1) / tiles;
-        if (splits > dp.KBn) splits = dp.KBn;
+        dp.mtiles = mtiles;
+        dp.dcols = layer->tc_dt / dp.dtiles;
+        const int splits = wide_down_splits(mtiles * dp.dcols, dp.KBn, sms);
         dp.kb_per_split = (dp.KBn + splits - 1) / splits;
-        splits = (dp.KBn + dp.kb_per_split - 1) / dp.kb_per_split;
-        dp.atomic_out = splits > 1 ? 1 : 0;
-        dp.add_residual = out_mode == kOutResid ? 1 : 0;
+        dp.units = mtiles * dp.dcols * splits;
         dp.out = out;
         dp.perm = perm;
         dp.ctl = ctl;
         dp.stage_bytes = BM * kTileBytes * (2 + dp.dtiles);
         dp.stages = stages_for(dp.stage_bytes, wide_budget());
-        if (splits > 1 && out_mode == kOutY &&
-            (e = cudaMemsetAsync(out, 0, (size_t)B * H * sizeof(float), stream)) != cudaSuccess)
-            return fail(e, "y clear");
+        dp.tmem_cols = tmem_cols_for(2 * BM * dp.dtiles);
         static std::atomic<int> cfg_dn[64];
         if ((e = set_smem(down_wide_kernel, smem_for(dp.stages, dp.stage_bytes), cfg_dn)) != cudaSuccess)
             return fail(e, "shared-memory attribute");
-        down_wide_kernel<<<dim3(mtiles, layer->tc_dt / dp.dtiles, splits), 64 + 128 * kWideDownGroups,
+        down_wide_kernel<<<dim3(dp.units < sms ? dp.units : sms), 64 + 128 * kWideDownGroups,
                            smem_for(dp.stages, dp.stage_bytes), stream>>>(mH, mH2, dp);
         if ((e = cudaGetLastError()) != cudaSuccess) return fail(e, "down kernel launch");
     }

@@ -26,7 +26,7 @@ constexpr int BK = 64;               // K per TMA box: one 128-byte swizzle row 
 constexpr int kThreads = 192;
 // Epilogue groups of four warps in the prefill kernels: the last tile's epilogue of the
 // persistent gate/up kernel, and every tile's of the down projection, follow their MMAs.
-constexpr int kWideGuGroups = 3;     // R = 96: two 16-neuron blocks each
+constexpr int kWideGuGroups = 4;     // at most: 128-neuron tiles, two 16-neuron blocks each
 constexpr int kWideDownGroups = 4;   // 256 columns: four 16-column blocks each
 constexpr int kWideMaxThreads = 64 + 128 * 4;
 constexpr int kSkinnyMaxGroups = 6;                             // epilogue groups of four warps
@@ -312,6 +312,54 @@ int choose_rows(int N, int sms)
         if (best_cost < 0 || cost <= best_cost) {
             best_cost = cost;
             best = R;
+        }
+    }
+    return best;
+}
+
+// Neurons per tile of the prefill gate/up kernel: the multiple of 16 (<= 128,
+// spanning at most two of the packed R-neuron tiles) that minimises waves x
+// shared-memory bytes per K step.  Each operand byte is
+// written to shared memory once by the copy engine and read once by the MMA; that
+// traffic (the x tile, twice for split activations, plus 2 Rw weight rows) paces
+// the MMA loop, while the tile's work grows with Rw.
+int wide_rows(int N, int R, int mtiles, int sms, bool split)
+{
+    int best = 16;
+    long long best_cost = -1;
+    for (int Rw = 16; Rw <= BM; Rw += 16) {
+        int g = Rw, r = R;   // gcd(Rw, R): a wide tile then spans at most two tiles of R neurons
+        while (r) {
+            const int t = g % r;
+            g = r;
+            r = t;
+        }
+        if (Rw - g > R) continue;
+        const long long tiles = (long long)mtiles * ((N + Rw - 1) / Rw);
+        const long long cost = ((tiles + sms - 1) / sms) * (BM * (split ? 2 : 1) + 2 * Rw);
+        if (best_cost < 0 || cost <= best_cost) {
+            best_cost = cost;
+            best = Rw;
+        }
+    }
+    return best;
+}
+
+// Splits of the neuron range in the prefill down projection: the count (<= 8,
+// none empty) that minimises waves x (K blocks per unit + 4), the 4 standing for
+// a unit's fixed cost (its accumulator's reductions into the output).
+int wide_down_splits(int tiles, int KBn, int sms)
+{
+    int best = 1;
+    long long best_cost = -1;
+    for (int s = 1; s <= 8 && s <= KBn; ++s) {
+        const int kps = (KBn + s - 1) / s;
+        if ((KBn + kps - 1) / kps != s) continue;
+        const long long units = (long long)tiles * s;
+        const long long cost = ((units + sms - 1) / sms) * (kps + 4);
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best = s;
         }
     }
     return best;
