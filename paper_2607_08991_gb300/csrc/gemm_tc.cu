@@ -22,9 +22,10 @@
 // threshold 0, and outputs, keep traces and kept lists go back to token perm[i].
 //
 // Two orientations:
-//  - skinny (M <= 256 tokens, bandwidth-bound): the weights are the MMA's A
-//    operand (128 rows: neurons, or hidden units for the down projection) and
-//    the tokens its N dimension, so no MMA row is spent on absent tokens.  The
+//  - skinny (M <= 256 tokens, 224 with fp32 activations; bandwidth-bound): the
+//    weights are the MMA's A operand (128 rows: neurons, or hidden units for the
+//    down projection) and the tokens its N dimension, so no MMA row is spent on
+//    absent tokens.  The
 //    down projection splits its 64-neuron K blocks evenly over one CTA per SM
 //    and adds partial sums into y with L2 reductions.
 //  - wide (prefill): tokens are the A operand in tiles of 128, the weights the
@@ -1259,7 +1260,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         e = launch_union_tail(layer, B, xa, split ? xlo : nullptr, uflag, ulist, ucount, a_keep, ldn, u, ldn, out, ctl,
                               stream);
         if (e != cudaSuccess) return fail(e, "union kernels launch");
-    } else if (B <= kMaxSkinny) {
+    } else if (B <= (split ? kMaxSkinnySplit : kMaxSkinny)) {
         const int NT = (B + 15) & ~15;
         CUtensorMap mX, mX2, mH, mH2;
         if (!make_map(&mX, xa, B, H, (uint64_t)H * 2, NT) || !make_map(&mX2, split ? xlo : xa, B, H, (uint64_t)H * 2, NT) ||

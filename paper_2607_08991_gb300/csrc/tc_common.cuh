@@ -35,6 +35,10 @@ constexpr int kSmemBudget = 196608;  // stage ring (one CTA per SM)
 constexpr int kSmemWide = 225280;    // stage ring of the persistent prefill kernels, at most
 constexpr int kMaxStages = 8;
 constexpr int kMaxSkinny = 256;      // largest batch on the skinny orientation (MMA N <= 256)
+// with fp32 activations (bf16 high and low parts), larger batches run faster on the prefill
+// kernels: at hidden 4096 / intermediate 14336, 256 tokens took 135 us skinny and 129 us wide
+// (224 tokens: 125 and 126 us); with bf16 activations the skinny kernels stay ahead up to 256
+constexpr int kMaxSkinnySplit = 224;
 constexpr int kMaxUnion = 8;         // largest batch on the union path (sparse-path tokens only)
 constexpr int kTileBytes = BK * 2;   // bytes of one tile row
 // The prefill kernels bring their weight stages into L2 this many stages ahead of

@@ -112,6 +112,7 @@ def test_tensor_core_batches_match_oracle(sats, oracle, H, N, B, k):
     (1024, 777, 40),
     (512, 1408, 128),   # 128 columns: the largest merged MMA (N = 256; 512 TMEM columns)
     (512, 1408, 200),   # 208 columns: two MMAs per step, hi and lo into the same accumulator
+    (1024, 777, 240),   # above 224 fp32 tokens: the prefill kernels, the second token tile partial
 ])
 def test_tensor_core_fp32_activations(sats, oracle, H, N, B):
     """fp32 x split into bf16 hi + lo parts: the gate keeps ~fp32 accuracy."""
