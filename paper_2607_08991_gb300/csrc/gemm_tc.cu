@@ -649,18 +649,22 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
         };
         const size_t kb_rows = (size_t)2 * R;   // rows of a gu_blk tile per K block
         // L2 prefetch of the weight stage kWidePrefetch loads ahead (this CTA's own sequence of
-        // tiles); of the CTAs that share a weight tile, those of its first two token tiles ask
-        int pq = blockIdx.x, pkb = 0;
-        bool pf_on = false;
+        // tiles); of the CTAs that share a weight tile, one asks for each stage, in turn (the CTA
+        // of token tile m takes the K blocks kb with (m + kb) mod mtiles = 0), so that the
+        // prefetches add the same work to every CTA's load thread
+        int pq = blockIdx.x, pkb = 0, prot = 0;
         Pieces pf{};
         auto prefetch_tile = [&]() {
-            pf_on = pq < p.tiles && pq % p.mtiles < 2;
-            if (pf_on) pf = pieces_of(pq / p.mtiles);
+            if (pq >= p.tiles) return;
+            prot = pq % p.mtiles;
+            pf = pieces_of(pq / p.mtiles);
         };
         prefetch_tile();
         auto prefetch_ahead = [&]() {
             if (pq >= p.tiles) return;
-            if (pf_on) {
+            const bool go = prot == 0;
+            if (++prot == p.mtiles) prot = 0;
+            if (go) {
                 const size_t o = (size_t)pkb * kb_rows;
                 for (int g = 0; g < 2; ++g) {
                     bulk_prefetch_l2(p.w + (pf.a + o + g * R) * BK, (uint32_t)(pf.la * kTileBytes));
