@@ -571,7 +571,7 @@ struct WideGuParams {
     uint8_t *keep_trace;
     int *ctl;
     float *zero;                  // y [M][H] to clear for the down projection's additions, or nullptr
-    int zero_count;               // M H (a multiple of 8)
+    long long zero_count;         // M H (a multiple of 8; M H can exceed 2^31 at prefill sizes)
     int stages, stage_bytes;
     uint32_t tmem_cols;           // two accumulator buffers of 2 Rw columns
 };
@@ -747,10 +747,10 @@ __global__ void __launch_bounds__(kWideMaxThreads, 1)
         if (p.zero) {
             // this CTA's share of y, cleared for the down projection's additions while the first
             // tile's MMAs run
-            const int per = (((p.zero_count + (int)gridDim.x - 1) / (int)gridDim.x) + 7) & ~7;
-            const int z0 = (int)blockIdx.x * per, z1 = min(p.zero_count, z0 + per);
+            const long long per = ((p.zero_count + gridDim.x - 1) / gridDim.x + 7) & ~7LL;
+            const long long z0 = (long long)blockIdx.x * per, z1 = min(p.zero_count, z0 + per);
             float4 *z = reinterpret_cast<float4 *>(p.zero);
-            for (int i = z0 / 4 + (int)threadIdx.x - 64; i < z1 / 4; i += (int)blockDim.x - 64)
+            for (long long i = z0 / 4 + (int)threadIdx.x - 64; i < z1 / 4; i += (int)blockDim.x - 64)
                 z[i] = make_float4(0.f, 0.f, 0.f, 0.f);
         }
         // epilogue: thread = token row of the tile, 16 neurons at a time; group g of four warps
@@ -1365,7 +1365,7 @@ cudaError_t run_tc_layer(const sats_layer *layer, int x_mode, const void *x, int
         gp.keep_trace = keep_trace;
         gp.ctl = ctl;
         gp.zero = out_mode == kOutY ? out : nullptr;   // the down projection adds into y
-        gp.zero_count = B * H;
+        gp.zero_count = (long long)B * H;
         gp.stage_bytes = BM * kTileBytes * (split ? 2 : 1) + 2 * gp.Rw * kTileBytes;
         gp.stages = stages_for(gp.stage_bytes, wide_budget());
         // epilogue groups: the tile's 16-neuron column blocks split evenly over at most kWideGuGroups
